@@ -1,0 +1,239 @@
+/*
+ * optr.h -- C ABI of the rotated INT2 paged KV-cache hot path of OptR
+ * ("Output-Aware Rotation for INT2 KV-Cache Quantization", arXiv 2608.02691).
+ *
+ * Two operations are exported:
+ *
+ *   optr_kv_append         cache write: center keys by mu, rotate K by R_k and
+ *                          V by R_v, group-wise asymmetric INT2 quantize, pack
+ *                          four codes per byte, scatter into paged blocks.
+ *   optr_decode_attention  decode read: rotate each GQA query by its KV head's
+ *                          R_k, stream the paged INT2 cache, dequantize in
+ *                          registers, split-K online softmax, combine, apply
+ *                          R_v^T to the attention output.
+ *
+ * Conventions (fixed for every entry point)
+ * ------------------------------------------
+ *  - Vectors are ROW vectors and a rotation acts on the right: z' = z R, i.e.
+ *    z'[j] = sum_i z[i] * R[i][j]  (paper, Introduction and Sec. 3.1, Eq. 4).
+ *    Every matrix argument is row-major float32, R[i][j] at offset i*D + j.
+ *  - GQA grouping is contiguous: query head j reads KV head j / (h_q / h_kv)
+ *    (Sec. 3, "Preliminaries": the set G_h of query heads sharing KV head h).
+ *  - Attention logits use the scale 1/sqrt(D) (Sec. 3, Eq. 1).
+ *  - Supported shape: head_dim D = 128, group G = 32, page_size P = 16.
+ *    Anything else returns OPTR_ERR_UNSUPPORTED.
+ *
+ * Quantizer Q2 (Sec. 3.1 "group-wise affine INT2 with clipping ratio c and
+ * group size G"; Table "Default experimental settings").  The paper does not
+ * write the formula out; this library fixes the following reading.  For one
+ * token, one KV head and one group of G = 32 consecutive ROTATED channels
+ * z_0..z_31, evaluated in IEEE float32 arithmetic:
+ *      mn = c * min_i z_i,  mx = c * max_i z_i          (c = clip ratio)
+ *      r  = mx - mn
+ *      degenerate group (r is not > 1e-30 or r is not finite):
+ *          all codes 0, scale = 0, min = fp16_rn(mn)
+ *      otherwise:
+ *          inv    = 3.0f / r
+ *          u_i    = (clamp(z_i, mn, mx) - mn) * inv
+ *          code_i = clamp(round_half_even(u_i), 0, 3)
+ *          scale  = fp16_rn(r / 3.0f),  min = fp16_rn(mn)
+ *      dequantized value: zhat_i = code_i * scale + min
+ * Codes are decided from the unrounded range, never from the fp16 scale.
+ * Inputs must be finite; NaN or Inf inputs give unspecified codes.
+ *
+ * Cache write (Sec. 4.1, "Rotated INT2 Cache Reparameterization"; Appendix,
+ * "Key-mean estimation and application"):
+ *      keys:   z_K = k R_k[h] - (mu[h] R_k[h])   ( = (k - mu[h]) R_k[h] )
+ *      values: z_V = v R_v[h]
+ * then Q2 with clip_k / clip_v.  mu[h] R_k[h] is precomputed once per head by
+ * optr_params_create.  The dequantized rotated key is what the decode
+ * attends with (Appendix, "Rotated-query implementation").
+ *
+ * Decode (Sec. 3 Eq. 1-2; Appendix, "Rotated-query implementation" and
+ * "Equivalent Inference Implementation"), for sequence b, query head j,
+ * KV head h = j / (h_q / h_kv), cached tokens s = 0 .. seq_lens[b]-1:
+ *      q'_j  = q_j R_k[h]
+ *      l_s   = <q'_j, khat_R,s> / sqrt(D)
+ *      p     = softmax_s(l)
+ *      o'_j  = sum_s p_s vhat_R,s
+ *      out_j = o'_j R_v[h]^T                                   (float32)
+ * The constant -q.mu term of the centered logits is omitted: softmax is
+ * invariant to it (Appendix, "Equivalent Inference Implementation").
+ * A sequence with seq_lens[b] == 0 gets an all-zero output.
+ *
+ * Paged pool layout (this library's choice; the paper inherits its layout
+ * from its serving stack).  The pool is a byte array
+ *      pool[num_pages][h_kv][OPTR_PAGE_HEAD_BYTES = 1536],
+ * 16-byte aligned, and token position pos of sequence b lives in physical
+ * page block_table[b * max_pages + pos / 16], slot pos % 16.  One
+ * (page, KV head) chunk is:
+ *      offset    0: K codes  [16 slots][32 bytes]
+ *      offset  512: V codes  [16 slots][32 bytes]
+ *      offset 1024: K meta   [16 slots][4 groups] {fp16 scale, fp16 min}
+ *      offset 1280: V meta   [16 slots][4 groups] {fp16 scale, fp16 min}
+ * Within a slot's 32 code bytes the groups are interleaved word-major:
+ * channel ch = 32*g + 4*w + r  (group g in 0..3, w in 0..7, r in 0..3) is
+ * stored in byte 4*w + g, bits [2r, 2r+1].  Byte 4*w + g therefore holds the
+ * four codes of channels 32g+4w .. 32g+4w+3, lowest channel in the lowest
+ * bits.  (Interleaving lets one decode lane fetch whole 32/64-bit words that
+ * carry every group it needs.)  Every slot owns whole bytes, so appends to
+ * different slots of one page never touch the same byte.
+ *
+ * Ownership and synchronisation
+ * -----------------------------
+ * The caller owns every tensor: q, k, v, tables, pool, out and workspace.
+ * The library owns only optr_params (device copies of R_k, R_v, mu R_k, the
+ * tensor-core splits of R, and a device error word).  optr_kv_append and
+ * optr_decode_attention allocate nothing and never synchronise; they enqueue
+ * kernels on the given stream and return.  Pointers named "device" must be
+ * device memory of the current CUDA device; "host" pointers are read
+ * synchronously before the call returns.
+ *
+ * Errors
+ * ------
+ * Argument errors are detected on the host before any launch and return a
+ * negative status; nothing is enqueued then.  Table contents (page ids,
+ * positions, sequence lengths) live in device memory and are checked by the
+ * kernels: an out-of-range entry is skipped (never dereferenced) and a bit is
+ * set in the params' device error word, read with optr_device_error().  No
+ * kernel traps, asserts or waits without bound.  A failed launch returns
+ * OPTR_ERR_CUDA.
+ */
+#ifndef OPTR_H_
+#define OPTR_H_
+
+#include <stddef.h>
+#include <stdint.h>
+#include <cuda_runtime_api.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define OPTR_HEAD_DIM 128
+#define OPTR_GROUP 32
+#define OPTR_PAGE_SIZE 16
+#define OPTR_PAGE_HEAD_BYTES 1536
+#define OPTR_K_CODES_OFFSET 0
+#define OPTR_V_CODES_OFFSET 512
+#define OPTR_K_META_OFFSET 1024
+#define OPTR_V_META_OFFSET 1280
+
+typedef enum {
+  OPTR_OK = 0,
+  OPTR_ERR_INVALID_ARG = -1, /* null pointer, non-positive size, bad ratio */
+  OPTR_ERR_UNSUPPORTED = -2, /* D, G or P other than 128 / 32 / 16        */
+  OPTR_ERR_OUT_OF_RANGE = -3,/* a size exceeds what the library handles    */
+  OPTR_ERR_WORKSPACE = -4,   /* workspace null or smaller than required    */
+  OPTR_ERR_CUDA = -5         /* a CUDA runtime call or launch failed        */
+} optr_status;
+
+/* Bits of the device error word (optr_device_error). */
+#define OPTR_DEVERR_PAGE_ID 1u   /* block_table entry < 0 or >= num_pages  */
+#define OPTR_DEVERR_POSITION 2u  /* append position >= max_pages * 16 or <0 */
+#define OPTR_DEVERR_SEQ_LEN 4u   /* seq_lens[b] < 0 or > max_pages * 16     */
+#define OPTR_DEVERR_CU_NEW 8u    /* cu_new not non-decreasing within n_tok  */
+
+/* Kernel variants (for measurement; 0 picks the library default). */
+#define OPTR_VARIANT_DEFAULT 0
+#define OPTR_VARIANT_CUDA_CORE 1  /* float32 FMA on CUDA cores             */
+#define OPTR_VARIANT_TENSOR 2     /* tensor-core path                      */
+
+typedef struct optr_params optr_params; /* opaque, library-owned */
+
+typedef struct {
+  int h_q;            /* query heads; a positive multiple of h_kv          */
+  int h_kv;           /* KV heads                                          */
+  int head_dim;       /* must be 128                                       */
+  int group;          /* must be 32                                        */
+  int page_size;      /* must be 16                                        */
+  float clip_k;       /* key clip ratio c_K in (0, 1]; 1 = min-max          */
+  float clip_v;       /* value clip ratio c_V in (0, 1]; 1 = min-max        */
+  int append_variant; /* OPTR_VARIANT_*                                    */
+  int decode_variant; /* OPTR_VARIANT_*                                    */
+} optr_config;
+
+/*
+ * Create the per-layer rotation state (paper Algorithm "OptR offline
+ * calibration": its output {R_K, R_V, mu} per KV head is this call's input).
+ *   cfg   host; shapes and clip ratios (copied).
+ *   R_k   host float32 [h_kv][D][D]: key rotation per KV head (orthogonal;
+ *         orthogonality is the caller's contract and is not checked).
+ *   R_v   host float32 [h_kv][D][D]: value rotation per KV head.
+ *   mu    host float32 [h_kv][D]: per-channel key mean (Appendix, key-mean
+ *         estimation).  Pass all zeros for no centering.
+ *   out   host; receives the new handle, or NULL on error.
+ * Allocates device memory on the current device (about h_kv * 200 KB) and
+ * copies synchronously.  Returns OPTR_OK or a negative status.
+ */
+optr_status optr_params_create(const optr_config* cfg, const float* R_k,
+                               const float* R_v, const float* mu,
+                               optr_params** out);
+
+/* Free a handle (NULL is ignored).  The caller ensures no enqueued work
+ * still uses it. */
+void optr_params_destroy(optr_params* p);
+
+/* Bytes of one page across all KV heads: h_kv * 1536. */
+size_t optr_page_bytes(const optr_params* p);
+
+/*
+ * Cache write (Sec. 4.1; Appendix, key-mean estimation and application).
+ *   k, v        device bf16 [n_tok][h_kv][D]: new keys (post-RoPE) and values.
+ *   n_tok       host; total new tokens (0 is a no-op).
+ *   cu_new      device int32 [B+1]: tokens of sequence b are rows
+ *               cu_new[b] .. cu_new[b+1]-1 of k / v; cu_new[0] = 0,
+ *               non-decreasing, cu_new[B] = n_tok.
+ *   pos0        device int32 [B]: cache position of sequence b's first new
+ *               token; token i of the sequence goes to position pos0[b] + i.
+ *   block_table device int32 [B][max_pages]: logical page -> physical page.
+ *   pool        device bytes [num_pages][h_kv][1536], written in place.
+ * Each written slot's codes and metadata are replaced entirely.  Two appends
+ * that target the same slot concurrently race.  Out-of-range table entries
+ * or positions skip that token and set a device error bit.
+ */
+optr_status optr_kv_append(const optr_params* p, const void* k, const void* v,
+                           int n_tok, const int32_t* cu_new,
+                           const int32_t* pos0, const int32_t* block_table,
+                           int B, int max_pages, uint8_t* pool, int num_pages,
+                           cudaStream_t stream);
+
+/* Workspace bytes optr_decode_attention needs for this batch shape on the
+ * current device (split-K partials and the rotated queries). */
+size_t optr_decode_workspace_size(const optr_params* p, int B, int max_pages);
+
+/*
+ * Decode attention over the paged INT2 cache (Sec. 3 Eq. 1-2; Appendix,
+ * rotated-query implementation and equivalent inference implementation).
+ *   q           device bf16 [B][h_q][D]: post-RoPE queries, one per sequence.
+ *   block_table device int32 [B][max_pages].
+ *   seq_lens    device int32 [B]: cached tokens per sequence, 0 .. max_pages*16.
+ *   pool        device bytes [num_pages][h_kv][1536] (read only).
+ *   out         device float32 [B][h_q][D]: attention output o = o' R_v^T.
+ *   workspace   device, at least optr_decode_workspace_size(p, B, max_pages)
+ *               bytes, 256-byte aligned; contents need no initialisation and
+ *               are scratch between calls (concurrent calls need distinct
+ *               workspaces).
+ */
+optr_status optr_decode_attention(const optr_params* p, const void* q,
+                                  const int32_t* block_table,
+                                  const int32_t* seq_lens, int B,
+                                  int max_pages, const uint8_t* pool,
+                                  int num_pages, float* out, void* workspace,
+                                  size_t ws_bytes, cudaStream_t stream);
+
+/*
+ * Read and clear the device error word of p (OPTR_DEVERR_* bits).
+ * Synchronises the device.  *flags receives 0 when no kernel reported a
+ * table error since the last call.
+ */
+optr_status optr_device_error(const optr_params* p, uint32_t* flags);
+
+/* Static description of a status code. */
+const char* optr_strerror(optr_status s);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* OPTR_H_ */
