@@ -1,0 +1,556 @@
+"""Benchmark of the rotated INT2 paged KV-cache hot path on one GB300.
+
+One step = one decode step of the Qwen3-8B-shaped layer (batch 16, 32 query /
+8 KV heads, head dim 128, context 8192 per sequence, page size 16, shuffled
+pages): append the step's new token of every sequence (center, rotate,
+INT2-quantize, pack, scatter) and run decode attention over the 8193 cached
+tokens (rotate queries, stream the INT2 pages, split-K online softmax,
+combine, apply R_v^T).  The cache is pre-filled by the library's append
+before timing.  Metric: algorithmic HBM bytes of the step per second (codes
+and fp16 scale/min read, bf16 query read, fp32 output written, plus the
+appended token's bf16 K/V read and INT2 record written).
+
+Extra measurements in the same JSON line: the prefill append workload
+(4 x 32768 tokens) in tokens/s, the long-context (131072) and ragged
+(batch 128) decode workloads, and the CPU oracle on a bounded sample.
+
+Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+Multi-GPU (weak scaling, no data-path collective): torchrun ... bench.py --gpus N.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+D = 128
+CHUNK = 1536
+L2_FLUSH_BYTES = 512 << 20
+
+
+# ------------------------------------------------------------------ utils
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+class Clocks:
+    """nvidia-smi sampling of SM clocks and throttle reasons during timing."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.lines = []
+        self.thread = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index),
+                 f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=subprocess.PIPE,
+                stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+        time.sleep(0.3)
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if not self.proc:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        sm, smax, reasons = [], 0.0, set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown",
+                 "sw_power_cap")
+        for ln in self.lines:
+            parts = [x.strip() for x in ln.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                smax = max(smax, float(parts[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[4:8]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": smax,
+                "samples": len(sm), "reasons": sorted(reasons)}
+
+
+def kernel_source_hash(files):
+    h = hashlib.sha256()
+    for f in files:
+        with open(os.path.join(ROOT, "paper_2608_02691_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def traffic_for(kernel_key, files):
+    """dram bytes per launch from the committed ncu summary, if the kernel's
+    source is unchanged since the counters were taken (else None)."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        e = d[kernel_key]
+        if e.get("source_sha") == kernel_source_hash(files):
+            return float(e["dram_bytes_per_launch"])
+    except Exception:
+        pass
+    return None
+
+
+# ------------------------------------------------------------ byte counts
+
+def decode_bytes(seq_lens, h_kv, h_q):
+    """Algorithmic bytes of one decode: 96 B per cached token and KV head
+    (32 + 32 code bytes, 16 + 16 metadata bytes), bf16 query, fp32 output."""
+    toks = int(sum(int(x) for x in seq_lens))
+    B = len(seq_lens)
+    return toks * h_kv * 96 + B * h_q * D * 2 + B * h_q * D * 4
+
+
+def decode_stream_bytes(seq_lens, h_kv):
+    """Bytes the split-K partial kernel streams: codes + metadata only."""
+    return int(sum(int(x) for x in seq_lens)) * h_kv * 96
+
+
+def append_bytes(n_tok, h_kv):
+    """Append: bf16 K and V read (512 B) + 96 B written per token and head."""
+    return n_tok * h_kv * (512 + 96)
+
+
+# ------------------------------------------------------------------- ours
+
+class Flusher:
+    def __init__(self, dev):
+        self.buf = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+
+    def __call__(self):
+        self.buf.fill_(1.0)
+
+
+def setup_decode(name, seed, dev, variant, append_variant):
+    from paper_2608_02691_gb300 import optr, synth
+    wl = synth.workload(name, seed)
+    case = synth.build_case(wl, seed, device=dev)
+    p = optr.optr_params_create(case["R_k"], case["R_v"], case["mu"],
+                                case["h_q"], decode_variant=variant,
+                                append_variant=append_variant)
+    pool = optr.new_pool(p, case["num_pages"], device=dev)
+    bt = case["block_table"].to(dev)
+    cu = case["cu_ctx"]
+    cl = cu.tolist()
+    # prefill in chunks of whole sequences (bounded temporary memory): the
+    # chunk's token rows are cu[b0]..cu[b1]; clamping the cumulative counts
+    # to that window gives every other sequence zero new tokens.
+    step = max(1, (1 << 21) // max(1, max(wl.ctx)))
+    for b0 in range(0, case["B"], step):
+        b1 = min(case["B"], b0 + step)
+        if cl[b1] == cl[b0]:
+            continue
+        cu_sub = (cu.clamp(cl[b0], cl[b1]) - cl[b0]).to(torch.int32)
+        optr.optr_kv_append(p, case["k_ctx"][cl[b0]:cl[b1]],
+                            case["v_ctx"][cl[b0]:cl[b1]], cu_sub.to(dev),
+                            case["pos0_ctx"].to(dev), bt, pool)
+    torch.cuda.synchronize()
+    return wl, case, p, pool, bt
+
+
+def run_ours(args, rank, world, dev):
+    from paper_2608_02691_gb300 import optr, synth
+    hbm_peak, peak_src = peaks()
+    flush = Flusher(dev)
+    result = {}
+
+    # ---------------- main step: decode8k (append 1 token/seq + decode)
+    wl, case, p, pool, bt = setup_decode("decode8k", args.seed, dev,
+                                         args.variant, args.append_variant)
+    B, h_q, h_kv = case["B"], case["h_q"], case["h_kv"]
+    seq = case["seq_lens"].to(dev)
+    q = case["q"].to(dev)
+    k_new, v_new = case["k_new"].to(dev), case["v_new"].to(dev)
+    cu_new, pos0 = case["cu_new"].to(dev), case["pos0_new"].to(dev)
+    out = torch.empty(B, h_q, D, dtype=torch.float32, device=dev)
+    ws = optr.new_workspace(p, B, bt.shape[1], device=dev)
+    stream = torch.cuda.current_stream()
+
+    def step():
+        optr.optr_kv_append(p, k_new, v_new, cu_new, pos0, bt, pool)
+        optr.optr_decode_attention(p, q, bt, seq, pool, out, ws)
+
+    step_bytes = (decode_bytes(case["seq_lens"].tolist(), h_kv, h_q) +
+                  append_bytes(k_new.shape[0], h_kv))
+    for _ in range(args.warmup):
+        flush()
+        step()
+    torch.cuda.synchronize()
+    assert optr.optr_device_error(p) == 0
+
+    evs = [(torch.cuda.Event(enable_timing=True),
+            torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    clocks = Clocks(torch.cuda.current_device()) if rank == 0 else None
+    if clocks:
+        clocks.start()
+    barrier(world)
+    torch.cuda.synchronize()
+    for i in range(args.steps):
+        flush()
+        evs[i][0].record(stream)
+        step()
+        evs[i][1].record(stream)
+    torch.cuda.synchronize()
+    barrier(world)
+    clk = clocks.stop() if clocks else None
+    ms = float(np.mean([a.elapsed_time(b) for a, b in evs]))
+    ms_max = allreduce_max(ms, world, dev)
+
+    # stage breakdown (one step at a time, events recorded by the library)
+    optr.optr_profile_enable(p, True)
+    stages = {"append": [], "qrot": [], "partial": [], "combine": []}
+    for _ in range(args.steps):
+        flush()
+        step()
+        st = optr.optr_profile_last(p)
+        for k2 in stages:
+            stages[k2].append(st[k2])
+    optr.optr_profile_enable(p, False)
+    stage_ms = {k2: float(np.mean(v)) for k2, v in stages.items()}
+
+    # end to end through the public API with host buffers
+    q_h = case["q"].pin_memory()
+    k_h, v_h = case["k_new"].pin_memory(), case["v_new"].pin_memory()
+    out_h = torch.empty(B, h_q, D, dtype=torch.float32).pin_memory()
+    h2d = q_h.numel() * 2 + k_h.numel() * 2 + v_h.numel() * 2
+    d2h = out_h.numel() * 4
+    q_d, k_d, v_d = torch.empty_like(q), torch.empty_like(k_new), torch.empty_like(v_new)
+
+    def e2e_step():
+        q_d.copy_(q_h, non_blocking=True)
+        k_d.copy_(k_h, non_blocking=True)
+        v_d.copy_(v_h, non_blocking=True)
+        optr.optr_kv_append(p, k_d, v_d, cu_new, pos0, bt, pool)
+        optr.optr_decode_attention(p, q_d, bt, seq, pool, out, ws)
+        out_h.copy_(out, non_blocking=True)
+
+    for _ in range(args.warmup):
+        flush()
+        e2e_step()
+    torch.cuda.synchronize()
+    e2e_ev = [(torch.cuda.Event(enable_timing=True),
+               torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    for i in range(args.steps):
+        flush()
+        e2e_ev[i][0].record(stream)
+        e2e_step()
+        e2e_ev[i][1].record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = float(np.mean([a.elapsed_time(b) for a, b in e2e_ev]))
+    e2e_ms = allreduce_max(e2e_ms, world, dev)
+
+    # roofline of the dominant kernel (split-K partial)
+    part_bytes = decode_stream_bytes(case["seq_lens"].tolist(), h_kv)
+    achieved = part_bytes / (stage_ms["partial"] * 1e-3) / 1e9
+    variant_files = (["decode_tc.cu", "decode_common.cuh"]
+                     if args.variant != 1 else ["decode.cu", "decode_common.cuh"])
+    key = "partial_tensor" if args.variant != 1 else "partial_cuda_core"
+    traffic = traffic_for(key, variant_files)
+    roofline = {"bound": "hbm", "kernel": key, "achieved": round(achieved, 1),
+                "peak": hbm_peak, "peak_source": peak_src, "unit": "GB/s",
+                "frac": round(achieved / hbm_peak, 4),
+                "frac_of_nominal_8000": round(achieved / 8000.0, 4),
+                "traffic": traffic,
+                "algorithmic_bytes_per_launch": part_bytes,
+                "launch_ms": round(stage_ms["partial"], 5)}
+
+    result["main"] = dict(ms=ms_max, bytes=step_bytes, stage_ms=stage_ms,
+                          e2e_ms=e2e_ms, h2d=h2d, d2h=d2h, roofline=roofline,
+                          clocks=clk, case=case, pool=pool, p=p)
+    return result
+
+
+def extra_workloads(args, dev):
+    """Prefill append throughput and the other decode workloads."""
+    from paper_2608_02691_gb300 import optr, synth
+    hbm_peak, _ = peaks()
+    flush = Flusher(dev)
+    res = {}
+    # prefill append: 4 x 32768 tokens
+    wl = synth.workload("prefill", args.seed)
+    case = synth.build_case(wl, args.seed, device=dev)
+    p = optr.optr_params_create(case["R_k"], case["R_v"], case["mu"],
+                                case["h_q"], append_variant=args.append_variant)
+    pool = optr.new_pool(p, case["num_pages"], device=dev)
+    bt = case["block_table"].to(dev)
+    k, v = case["k_new"].to(dev), case["v_new"].to(dev)
+    cu, pos0 = case["cu_new"].to(dev), case["pos0_new"].to(dev)
+    for _ in range(3):
+        optr.optr_kv_append(p, k, v, cu, pos0, bt, pool)
+    optr.optr_profile_enable(p, True)
+    t = []
+    for _ in range(max(5, args.steps // 4)):
+        flush()
+        optr.optr_kv_append(p, k, v, cu, pos0, bt, pool)
+        t.append(optr.optr_profile_last(p)["append"])
+    optr.optr_profile_enable(p, False)
+    ms = float(np.mean(t))
+    n_tok = k.shape[0]
+    nb = append_bytes(n_tok, case["h_kv"])
+    res["prefill_append"] = {
+        "tokens": n_tok, "ms": round(ms, 4),
+        "tokens_per_s": round(n_tok / (ms * 1e-3), 1),
+        "gbs": round(nb / (ms * 1e-3) / 1e9, 1),
+        "frac": round(nb / (ms * 1e-3) / 1e9 / hbm_peak, 4)}
+    del pool, k, v, case
+    torch.cuda.empty_cache()
+
+    for name in ("long128k", "ragged"):
+        wl, case, p, pool, bt = setup_decode(name, args.seed, dev, args.variant,
+                                             args.append_variant)
+        seq = case["seq_lens"].to(dev)
+        q = case["q"].to(dev)
+        out = torch.empty(case["B"], case["h_q"], D, device=dev)
+        ws = optr.new_workspace(p, case["B"], bt.shape[1], device=dev)
+        if case["k_new"].shape[0]:
+            optr.optr_kv_append(p, case["k_new"].to(dev), case["v_new"].to(dev),
+                                case["cu_new"].to(dev), case["pos0_new"].to(dev),
+                                bt, pool)
+        else:
+            seq = case["seq_lens_ctx"].to(dev)
+        for _ in range(3):
+            optr.optr_decode_attention(p, q, bt, seq, pool, out, ws)
+        optr.optr_profile_enable(p, True)
+        st = []
+        for _ in range(max(5, args.steps // 4)):
+            flush()
+            optr.optr_decode_attention(p, q, bt, seq, pool, out, ws)
+            st.append(optr.optr_profile_last(p))
+        optr.optr_profile_enable(p, False)
+        lens = seq.cpu().tolist()
+        tot = sum(np.mean([s[k2] for s in st]) for k2 in ("qrot", "partial", "combine"))
+        part = float(np.mean([s["partial"] for s in st]))
+        nb = decode_bytes(lens, case["h_kv"], case["h_q"])
+        sb = decode_stream_bytes(lens, case["h_kv"])
+        res[name] = {"decode_ms": round(tot, 4), "gbs": round(nb / (tot * 1e-3) / 1e9, 1),
+                     "partial_ms": round(part, 4),
+                     "partial_gbs": round(sb / (part * 1e-3) / 1e9, 1),
+                     "partial_frac": round(sb / (part * 1e-3) / 1e9 / hbm_peak, 4)}
+        del pool, case
+        torch.cuda.empty_cache()
+    return res
+
+
+# ---------------------------------------------------------- CPU baseline
+
+def cpu_baseline(case, pool_gpu, n_groups, threads):
+    """The oracle, as it stands, on a bounded sample of the main workload:
+    the decode of n_groups (sequence, KV head) groups (4 query heads each)
+    over their full contexts.  Returns GB/s on the same byte accounting."""
+    from oracle import oracle
+    from paper_2608_02691_gb300 import synth
+    oracle.build()
+    oracle.set_threads(threads)
+    pool = pool_gpu.cpu().numpy()
+    rows = []
+    B, h_kv = case["B"], case["h_kv"]
+    groups = [(b, h) for b in range(B) for h in range(h_kv)][:n_groups]
+    for b, h in groups:
+        rows += [(b, 4 * h + r) for r in range(4)]
+    qb = synth.bf16_bits(case["q"])
+    t0 = time.perf_counter()
+    oracle.decode_attention(qb, case["block_table"].numpy(),
+                            case["seq_lens"].numpy(), pool, case["R_k"].numpy(),
+                            case["R_v"].numpy(), h_kv, rows=rows)
+    dt = time.perf_counter() - t0
+    lens = case["seq_lens"].tolist()
+    nb = sum(lens[b] * 96 + 4 * D * 6 for b, _ in groups)
+    return {"value": round(nb / dt / 1e9, 4), "unit": "GB/s", "cores": threads,
+            "kind": "oracle", "seconds": round(dt, 2),
+            "sample": f"oracle decode of {len(groups)} of {B * h_kv} (sequence, KV head) "
+                      f"groups of the batch-16 x 8193-token step (4 query heads each)"}
+
+
+# ------------------------------------------------------------- reference
+
+def run_reference(args, rank, world):
+    """The oracle as the reference arm: each step = oracle append of the new
+    token of the sampled sequences + oracle decode of those sequences."""
+    if rank != 0:
+        return None
+    from oracle import oracle
+    from paper_2608_02691_gb300 import synth
+    oracle.build()
+    threads = os.cpu_count() or 1
+    oracle.set_threads(threads)
+    wl = synth.workload("decode8k", args.seed)
+    wl.B = args.ref_seqs
+    wl.ctx = wl.ctx[:args.ref_seqs]
+    case = synth.build_case(wl, args.seed)
+    bt = case["block_table"].numpy()
+    pool = np.zeros((case["num_pages"], case["h_kv"], CHUNK), np.uint8)
+    R = (case["R_k"].numpy(), case["R_v"].numpy(), case["mu"].numpy())
+    oracle.kv_append(synth.bf16_bits(case["k_ctx"]), synth.bf16_bits(case["v_ctx"]),
+                     case["cu_ctx"].numpy(), case["pos0_ctx"].numpy(), bt, pool, *R)
+    qb = synth.bf16_bits(case["q"])
+    kb, vb = synth.bf16_bits(case["k_new"]), synth.bf16_bits(case["v_new"])
+
+    def step():
+        oracle.kv_append(kb, vb, case["cu_new"].numpy(), case["pos0_new"].numpy(),
+                         bt, pool, *R)
+        oracle.decode_attention(qb, bt, case["seq_lens"].numpy(), pool,
+                                case["R_k"].numpy(), case["R_v"].numpy(),
+                                case["h_kv"])
+
+    for _ in range(args.warmup):
+        step()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        step()
+    dt = (time.perf_counter() - t0) / args.steps
+    nb = (decode_bytes(case["seq_lens"].tolist(), case["h_kv"], case["h_q"]) +
+          append_bytes(case["k_new"].shape[0], case["h_kv"]))
+    v = nb / dt / 1e9
+    sample = (f"{args.ref_seqs} of 16 sequences of the batch-16 x 8193-token "
+              f"decode step (append 1 token + decode, all 8 KV heads)")
+    return {"impl": "reference", "metric": METRIC, "value": round(v, 4),
+            "unit": "GB/s", "n_gpus": 1, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": round(dt * 1e3, 3),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "f64", "data": "synthetic",
+            "config": {"workload": "decode8k: batch 16, 32 q / 8 kv heads, "
+                                   "head_dim 128, context 8192+1, page 16",
+                       "sample_sequences": args.ref_seqs},
+            "cpu_baseline": {"value": round(v, 4), "unit": "GB/s",
+                             "cores": threads, "kind": "oracle", "sample": sample},
+            "e2e": {"value": round(v, 4), "unit": "GB/s",
+                    "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+
+
+METRIC = "decode-attention HBM GB/s (decode step: append 1 token/seq + decode)"
+
+
+# ------------------------------------------------------------- dist glue
+
+def barrier(world):
+    if world > 1:
+        torch.distributed.barrier()
+
+
+def allreduce_max(x, world, dev):
+    if world <= 1:
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--variant", type=int, default=0)
+    ap.add_argument("--append-variant", type=int, default=0)
+    ap.add_argument("--ref-seqs", type=int, default=2)
+    ap.add_argument("--cpu-groups", type=int, default=128)
+    ap.add_argument("--no-extra", action="store_true")
+    ap.add_argument("--no-cpu", action="store_true")
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+
+    if args.impl == "reference":
+        if world > 1:
+            os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+        line = run_reference(args, rank, world)
+        if line is not None:
+            print(json.dumps(line), flush=True)
+        return
+
+    if world > 1:
+        torch.distributed.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    import __graft_entry__
+    __graft_entry__.build()
+
+    res = run_ours(args, rank, world, dev)
+    m = res["main"]
+    extra = extra_workloads(args, dev) if (rank == 0 and not args.no_extra) else None
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu:
+        cpu = cpu_baseline(m["case"], m["pool"], args.cpu_groups, os.cpu_count() or 1)
+    if rank == 0:
+        value = m["bytes"] * world / (m["ms"] * 1e-3) / 1e9
+        e2e = m["bytes"] * world / (m["e2e_ms"] * 1e-3) / 1e9
+        line = {
+            "metric": METRIC, "value": round(value, 2), "unit": "GB/s",
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(m["ms"], 5), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "int2+fp16 meta, f32 math",
+            "data": "synthetic",
+            "config": {"workload": "decode8k: batch 16 x context 8192 (+1 appended "
+                                   "token per sequence), 32 q / 8 kv heads, head_dim 128, "
+                                   "page 16, shuffled pages, Student-t(4) K/V",
+                       "bytes_per_step": m["bytes"], "l2": "flushed (512 MiB write) "
+                       "before every timed step; step timed alone with CUDA events",
+                       "decode_variant": args.variant, "append_variant": args.append_variant},
+            "gpu_launches": 4 * args.steps,
+            "stage_ms": {k: round(v, 5) for k, v in m["stage_ms"].items()},
+            "roofline": m["roofline"],
+            "e2e": {"value": round(e2e, 2), "unit": "GB/s",
+                    "h2d_bytes_per_step": m["h2d"], "d2h_bytes_per_step": m["d2h"],
+                    "ms_per_step": round(m["e2e_ms"], 5)},
+            "clocks": m["clocks"],
+            "cpu_baseline": cpu,
+            "workloads": extra,
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

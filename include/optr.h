@@ -229,6 +229,20 @@ optr_status optr_decode_attention(const optr_params* p, const void* q,
  */
 optr_status optr_device_error(const optr_params* p, uint32_t* flags);
 
+/*
+ * Stage timing for measurement (off by default).  optr_profile_enable(p, 1)
+ * creates library-owned CUDA events; afterwards every optr_kv_append and
+ * optr_decode_attention call made with p records an event on its stream
+ * before and after each kernel it launches.  optr_profile_last waits for the
+ * most recent calls' events and returns their durations in milliseconds:
+ *   ms[0] append kernel, ms[1] query rotation + plan, ms[2] split-K partial,
+ *   ms[3] combine (a stage that did not run reports 0).
+ * Calls that overlap on the GPU share the events, so time one call at a
+ * time.  optr_profile_enable(p, 0) destroys the events.
+ */
+optr_status optr_profile_enable(optr_params* p, int on);
+optr_status optr_profile_last(const optr_params* p, float ms[4]);
+
 /* Static description of a status code. */
 const char* optr_strerror(optr_status s);
 

@@ -1,0 +1,355 @@
+// Decode attention over the paged INT2 cache.
+//
+//   qrot     q' = q R_k[h] * log2(e)/sqrt(128) for every query head, per-group
+//            sums of q', and the split-K plan (page prefix sums over the
+//            batch)  -- paper Appendix, "Rotated-query implementation".
+//   partial  persistent warps; the flattened (sequence, KV head, page) space
+//            is cut into W equal contiguous ranges, one per warp.  A warp runs
+//            an online softmax over each (sequence, KV head) segment of its
+//            range and writes one partial (m, l, o') per segment.
+//   combine  per (sequence, KV head): log-sum-exp merge of the segment
+//            partials, then o = o' R_v^T (Appendix, "Equivalent Inference
+//            Implementation": o' = o R_V, recovered with R_V^T).
+//
+// Logits are kept in the log2 domain: q' carries log2(e)/sqrt(d), so
+// softmax weights are exp2(l - m) (Sec. 3 Eq. 1 with the 1/sqrt(d) scale).
+#include "decode_common.cuh"
+
+namespace optr {
+namespace {
+
+constexpr float kLog2e = 1.4426950408889634f;
+
+// ---------------------------------------------------------------- qrot
+
+__global__ void __launch_bounds__(128)
+qrot_kernel(const __nv_bfloat16* __restrict__ q, const float* __restrict__ R_k,
+            int B, int h_q, int h_kv, float qscale,
+            const int32_t* __restrict__ seq_lens, int max_pages,
+            float* __restrict__ qf, float* __restrict__ qs,
+            int* __restrict__ pref, int* __restrict__ nzpref, unsigned* err) {
+  __shared__ float qsm[4][kD];
+  __shared__ int warp_tot[2][4];
+  const int b = blockIdx.x, h = blockIdx.y, j = threadIdx.x;
+  const int warp = j >> 5, lane = j & 31;
+#pragma unroll
+  for (int r = 0; r < 4; ++r)
+    qsm[r][j] = __bfloat162float(q[((size_t)b * h_q + 4 * h + r) * kD + j]);
+  __syncthreads();
+  float acc[4] = {0.f, 0.f, 0.f, 0.f};
+  const float* R = R_k + (size_t)h * kD * kD;
+  for (int i = 0; i < kD; ++i) {
+    const float rij = __ldg(R + i * kD + j);
+#pragma unroll
+    for (int r = 0; r < 4; ++r) acc[r] = fmaf(qsm[r][i], rij, acc[r]);
+  }
+#pragma unroll
+  for (int r = 0; r < 4; ++r) {
+    const float x = acc[r] * qscale;
+    const size_t row = (size_t)b * h_q + 4 * h + r;
+    qf[row * kD + j] = x;
+    float s = x;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    if (lane == 0) qs[row * kGroups + warp] = s;  // warp == group
+  }
+
+  if (b != 0 || h != 0) return;
+  // Split-K plan: pref[b] = pages of sequences < b, nzpref[b] = non-empty
+  // sequences < b.  Invalid lengths count as empty and are flagged.
+  int run_p = 0, run_n = 0;
+  for (int base = 0; base < B; base += 128) {
+    const int bb = base + j;
+    int np = 0;
+    if (bb < B) {
+      const int len = seq_lens[bb];
+      if (len < 0 || (long long)len > (long long)max_pages * kPage)
+        atomicOr(err, OPTR_DEVERR_SEQ_LEN);
+      else
+        np = (len + kPage - 1) / kPage;
+    }
+    int xp = np, xn = np > 0;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int yp = __shfl_up_sync(0xffffffffu, xp, o);
+      const int yn = __shfl_up_sync(0xffffffffu, xn, o);
+      if (lane >= o) { xp += yp; xn += yn; }
+    }
+    if (lane == 31) { warp_tot[0][warp] = xp; warp_tot[1][warp] = xn; }
+    __syncthreads();
+    int op = run_p, on = run_n;
+    for (int w = 0; w < warp; ++w) { op += warp_tot[0][w]; on += warp_tot[1][w]; }
+    if (bb < B) { pref[bb + 1] = op + xp; nzpref[bb + 1] = on + xn; }
+    if (bb == 0) { pref[0] = 0; nzpref[0] = 0; }
+    for (int w = 0; w < 4; ++w) { run_p += warp_tot[0][w]; run_n += warp_tot[1][w]; }
+    __syncthreads();
+  }
+}
+
+// ------------------------------------------------- CUDA-core partial kernel
+
+struct WarpSmemCC {
+  alignas(16) uint8_t stage[2][kChunk];
+  float qv[4][kD];
+  float qsum[4][kGroups];
+  float p[kPage][4];
+};
+
+__global__ void __launch_bounds__(128)
+partial_cuda_core_kernel(const uint8_t* __restrict__ pool,
+                         const int32_t* __restrict__ bt,
+                         const int32_t* __restrict__ seq_lens, int B,
+                         int max_pages, int num_pages, int h_q, int h_kv,
+                         const float* __restrict__ qf,
+                         const float* __restrict__ qs,
+                         const int* __restrict__ pref,
+                         const int* __restrict__ nzpref,
+                         float* __restrict__ part, int W, unsigned* err) {
+  __shared__ WarpSmemCC smem[4];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  WarpSmemCC& S = smem[warp];
+  const int w = blockIdx.x * 4 + warp;
+  const long long F = (long long)__ldg(pref + B) * h_kv;
+  long long f = w * F / W;
+  const long long f1 = (w + 1) * F / W;
+
+  while (f < f1) {
+    Segment sg = locate_segment(f, f1, pref, B, h_kv);
+    const int b = sg.b, h = sg.h;
+    const int len = __ldg(seq_lens + b);
+    // rotated queries of the GQA group
+    for (int i = lane; i < 4 * kD; i += 32)
+      S.qv[i / kD][i % kD] = __ldg(qf + ((size_t)b * h_q + 4 * h) * kD + i);
+    if (lane < 16)
+      S.qsum[lane / 4][lane % 4] = __ldg(qs + ((size_t)b * h_q + 4 * h) * kGroups + lane);
+    float m[4], l[4], acc[4][4];
+#pragma unroll
+    for (int r = 0; r < 4; ++r) {
+      m[r] = -INFINITY;
+      l[r] = 0.f;
+#pragma unroll
+      for (int c = 0; c < 4; ++c) acc[r][c] = 0.f;
+    }
+    const int32_t* btb = bt + (size_t)b * max_pages;
+    // 2-stage cp.async pipeline over the segment's pages
+    bool ok0 = issue_page(S.stage[0], pool, btb, sg.p0, num_pages, h_kv, h, lane, err);
+    bool okn = false;
+    for (int i = 0; i < sg.n; ++i) {
+      const bool ok = (i == 0) ? ok0 : okn;
+      if (i + 1 < sg.n)
+        okn = issue_page(S.stage[(i + 1) & 1], pool, btb, sg.p0 + i + 1,
+                         num_pages, h_kv, h, lane, err);
+      else
+        cp_async_commit();
+      cp_async_wait_1();
+      __syncwarp();
+      const uint8_t* st = S.stage[i & 1];
+      const int page = sg.p0 + i;
+      int nvalid = ok ? min(kPage, len - page * kPage) : 0;
+      __syncwarp();
+
+      // logits: lane -> token t, heads hp and hp+1
+      const int t = lane & 15, hp = (lane >> 4) * 2;
+      float lg0 = -INFINITY, lg1 = -INFINITY;
+      if (t < nvalid) {
+        float a0 = 0.f, a1 = 0.f;
+        const uint8_t* kc = st + OPTR_K_CODES_OFFSET + t * 32;
+        const __half2* km = reinterpret_cast<const __half2*>(st + OPTR_K_META_OFFSET + t * 16);
+#pragma unroll
+        for (int G = 0; G < kGroups; ++G) {
+          float d0 = 0.f, d1 = 0.f;
+#pragma unroll
+          for (int wd = 0; wd < 8; ++wd) {
+            const unsigned byte = kc[4 * wd + G];
+#pragma unroll
+            for (int r = 0; r < 4; ++r) {
+              const float c = (float)((byte >> (2 * r)) & 3u);
+              const int ch = 32 * G + 4 * wd + r;
+              d0 = fmaf(S.qv[hp][ch], c, d0);
+              d1 = fmaf(S.qv[hp + 1][ch], c, d1);
+            }
+          }
+          const float2 sm = __half22float2(km[G]);
+          a0 += sm.x * d0 + sm.y * S.qsum[hp][G];
+          a1 += sm.x * d1 + sm.y * S.qsum[hp + 1][G];
+        }
+        lg0 = a0;
+        lg1 = a1;
+      }
+      // online softmax over the 16 tokens of each head
+      float t0 = lg0, t1 = lg1;
+#pragma unroll
+      for (int o = 1; o < 16; o <<= 1) {
+        t0 = fmaxf(t0, __shfl_xor_sync(0xffffffffu, t0, o));
+        t1 = fmaxf(t1, __shfl_xor_sync(0xffffffffu, t1, o));
+      }
+      float tmax[4];
+      tmax[0] = __shfl_sync(0xffffffffu, t0, 0);
+      tmax[1] = __shfl_sync(0xffffffffu, t1, 0);
+      tmax[2] = __shfl_sync(0xffffffffu, t0, 16);
+      tmax[3] = __shfl_sync(0xffffffffu, t1, 16);
+      float alpha[4], mnew[4];
+#pragma unroll
+      for (int r = 0; r < 4; ++r) {
+        mnew[r] = fmaxf(m[r], tmax[r]);
+        alpha[r] = (mnew[r] == -INFINITY) ? 1.f : exp2f(m[r] - mnew[r]);
+      }
+      const float p0 = (lg0 == -INFINITY) ? 0.f : exp2f(lg0 - mnew[hp]);
+      const float p1 = (lg1 == -INFINITY) ? 0.f : exp2f(lg1 - mnew[hp + 1]);
+      S.p[t][hp] = p0;
+      S.p[t][hp + 1] = p1;
+      float s0 = p0, s1 = p1;
+#pragma unroll
+      for (int o = 1; o < 16; o <<= 1) {
+        s0 += __shfl_xor_sync(0xffffffffu, s0, o);
+        s1 += __shfl_xor_sync(0xffffffffu, s1, o);
+      }
+      float psum[4];
+      psum[0] = __shfl_sync(0xffffffffu, s0, 0);
+      psum[1] = __shfl_sync(0xffffffffu, s1, 0);
+      psum[2] = __shfl_sync(0xffffffffu, s0, 16);
+      psum[3] = __shfl_sync(0xffffffffu, s1, 16);
+#pragma unroll
+      for (int r = 0; r < 4; ++r) {
+        l[r] = l[r] * alpha[r] + psum[r];
+        m[r] = mnew[r];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) acc[r][c] *= alpha[r];
+      }
+      __syncwarp();
+      // PV: lane -> byte `lane` of the value codes (4 channels of group lane%4)
+      const int G = lane & 3;
+      for (int tt = 0; tt < nvalid; ++tt) {
+        const unsigned byte = st[OPTR_V_CODES_OFFSET + tt * 32 + lane];
+        const float2 sm = __half22float2(
+            reinterpret_cast<const __half2*>(st + OPTR_V_META_OFFSET + tt * 16)[G]);
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          const float vv = fmaf((float)((byte >> (2 * c)) & 3u), sm.x, sm.y);
+#pragma unroll
+          for (int r = 0; r < 4; ++r) acc[r][c] = fmaf(S.p[tt][r], vv, acc[r][c]);
+        }
+      }
+      __syncwarp();
+    }
+    // partial slot of this segment
+    float* dst = part + (size_t)(w + nzpref[b] * h_kv + h) * kPartFloats;
+    const int wd = lane >> 2, G = lane & 3;
+#pragma unroll
+    for (int r = 0; r < 4; ++r)
+#pragma unroll
+      for (int c = 0; c < 4; ++c) dst[r * (kD + 2) + 32 * G + 4 * wd + c] = acc[r][c];
+    if (lane < 4) {
+      dst[lane * (kD + 2) + kD] = m[lane];
+      dst[lane * (kD + 2) + kD + 1] = l[lane];
+    }
+    f = sg.f_end;
+  }
+}
+
+// ------------------------------------------------------------- combine
+
+__global__ void __launch_bounds__(128)
+combine_kernel(const float* __restrict__ part, const int* __restrict__ pref,
+               const int* __restrict__ nzpref, int B, int h_q, int h_kv, int W,
+               const float* __restrict__ R_vT, float* __restrict__ out) {
+  __shared__ float orot[4][kD];
+  __shared__ float coef[4][2];
+  const int b = blockIdx.x, h = blockIdx.y, j = threadIdx.x;
+  const int np = __ldg(pref + b + 1) - __ldg(pref + b);
+  float* ob = out + ((size_t)b * h_q + 4 * h) * kD;
+  if (np == 0) {
+#pragma unroll
+    for (int r = 0; r < 4; ++r) ob[r * kD + j] = 0.f;
+    return;
+  }
+  const long long F = (long long)__ldg(pref + B) * h_kv;
+  const long long fs = (long long)__ldg(pref + b) * h_kv + (long long)h * np;
+  const int w0 = warp_of(fs, F, W), w1 = warp_of(fs + np - 1, F, W);
+  const size_t base = (size_t)__ldg(nzpref + b) * h_kv + h;
+  if (j < 4) {
+    float M = -INFINITY;
+    for (int w = w0; w <= w1; ++w)
+      if (!warp_empty(w, F, W))
+        M = fmaxf(M, part[(base + w) * kPartFloats + j * (kD + 2) + kD]);
+    float L = 0.f;
+    for (int w = w0; w <= w1; ++w) {
+      if (warp_empty(w, F, W)) continue;
+      const float* pp = part + (base + w) * kPartFloats + j * (kD + 2);
+      L += pp[kD + 1] * merge_weight(pp[kD], M);
+    }
+    coef[j][0] = M;
+    coef[j][1] = L > 0.f ? 1.f / L : 0.f;
+  }
+  __syncthreads();
+#pragma unroll
+  for (int r = 0; r < 4; ++r) {
+    const float M = coef[r][0];
+    float o = 0.f;
+    for (int w = w0; w <= w1; ++w) {
+      if (warp_empty(w, F, W)) continue;
+      const float* pp = part + (base + w) * kPartFloats + r * (kD + 2);
+      o += pp[j] * merge_weight(pp[kD], M);
+    }
+    orot[r][j] = o * coef[r][1];
+  }
+  __syncthreads();
+  const float* RT = R_vT + (size_t)h * kD * kD;
+  float acc[4] = {0.f, 0.f, 0.f, 0.f};
+  for (int jj = 0; jj < kD; ++jj) {
+    const float rt = __ldg(RT + jj * kD + j);  // R_v[h][j][jj]
+#pragma unroll
+    for (int r = 0; r < 4; ++r) acc[r] = fmaf(orot[r][jj], rt, acc[r]);
+  }
+#pragma unroll
+  for (int r = 0; r < 4; ++r) ob[r * kD + j] = acc[r];
+}
+
+}  // namespace
+
+cudaError_t launch_partial_tensor(const optr_params* p, const uint8_t* pool,
+                                  const int32_t* bt, const int32_t* seq_lens,
+                                  int B, int max_pages, int num_pages,
+                                  const float* qf, const float* qs,
+                                  const int* pref, const int* nzpref,
+                                  float* part, int W, cudaStream_t s);
+
+cudaError_t launch_decode(const optr_params* p, int variant,
+                          const __nv_bfloat16* q, const int32_t* bt,
+                          const int32_t* seq_lens, int B, int max_pages,
+                          const uint8_t* pool, int num_pages, float* out,
+                          void* ws, const DecodePlan& plan, cudaStream_t s) {
+  char* w = static_cast<char*>(ws);
+  float* qf = reinterpret_cast<float*>(w + plan.off_qf);
+  float* qs = reinterpret_cast<float*>(w + plan.off_qs);
+  int* pref = reinterpret_cast<int*>(w + plan.off_pref);
+  int* nzpref = pref + (B + 1);
+  float* part = reinterpret_cast<float*>(w + plan.off_part);
+  const int h_q = p->cfg.h_q, h_kv = p->cfg.h_kv;
+  const float qscale = kLog2e / sqrtf((float)kD);
+
+  prof_mark(p, 2, s);
+  qrot_kernel<<<dim3(B, h_kv), 128, 0, s>>>(q, p->R_k, B, h_q, h_kv, qscale,
+                                            seq_lens, max_pages, qf, qs, pref,
+                                            nzpref, p->err);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  prof_mark(p, 3, s);
+  if (variant == OPTR_VARIANT_TENSOR) {
+    e = launch_partial_tensor(p, pool, bt, seq_lens, B, max_pages, num_pages,
+                              qf, qs, pref, nzpref, part, plan.W, s);
+  } else {
+    partial_cuda_core_kernel<<<plan.W / 4, 128, 0, s>>>(
+        pool, bt, seq_lens, B, max_pages, num_pages, h_q, h_kv, qf, qs, pref,
+        nzpref, part, plan.W, p->err);
+    e = cudaGetLastError();
+  }
+  if (e != cudaSuccess) return e;
+  prof_mark(p, 4, s);
+  combine_kernel<<<dim3(B, h_kv), 128, 0, s>>>(part, pref, nzpref, B, h_q,
+                                               h_kv, plan.W, p->R_vT, out);
+  prof_mark(p, 5, s);
+  return cudaGetLastError();
+}
+
+}  // namespace optr

@@ -1,0 +1,251 @@
+// Host side of the C ABI declared in include/optr.h: argument validation,
+// library-owned state (optr_params) and kernel launches.  No entry point
+// here allocates or synchronises except optr_params_create/destroy and
+// optr_device_error.
+#include <math.h>
+#include <stdlib.h>
+#include <string.h>
+
+#include <vector>
+
+#include "optr_internal.cuh"
+
+using namespace optr;
+
+namespace {
+
+bool aligned(const void* ptr, size_t a) {
+  return (reinterpret_cast<uintptr_t>(ptr) % a) == 0;
+}
+
+optr_status cuda_status(cudaError_t e) {
+  return e == cudaSuccess ? OPTR_OK : OPTR_ERR_CUDA;
+}
+
+size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+}  // namespace
+
+namespace optr {
+
+// Workspace of one decode call (all offsets 256-byte aligned):
+//   qf   float [B][h_q][128]   rotated, pre-scaled queries
+//   qs   float [B][h_q][4]     per-group sums of qf
+//   pref int   [2][B+1]        page prefix sums / non-empty prefix counts
+//   part float [W + B*h_kv][4][130] split-K partials
+DecodePlan decode_plan(const optr_params* p, int B, int max_pages) {
+  DecodePlan d;
+  d.B = B;
+  d.h_q = p->cfg.h_q;
+  d.h_kv = p->cfg.h_kv;
+  d.max_pages = max_pages;
+  d.W = p->num_sms * kDecodeWarpsPerSm;
+  size_t o = 0;
+  d.off_qf = o;
+  o = round_up(o + sizeof(float) * (size_t)B * d.h_q * kD, 256);
+  d.off_qs = o;
+  o = round_up(o + sizeof(float) * (size_t)B * d.h_q * kGroups, 256);
+  d.off_pref = o;
+  o = round_up(o + sizeof(int) * 2 * (size_t)(B + 1), 256);
+  d.off_part = o;
+  o = round_up(o + sizeof(float) * kPartFloats *
+                       ((size_t)d.W + (size_t)B * d.h_kv), 256);
+  d.total = o;
+  return d;
+}
+
+}  // namespace optr
+
+extern "C" {
+
+const char* optr_strerror(optr_status s) {
+  switch (s) {
+    case OPTR_OK: return "ok";
+    case OPTR_ERR_INVALID_ARG: return "invalid argument";
+    case OPTR_ERR_UNSUPPORTED: return "unsupported shape (need D=128, G=32, P=16, h_q = 4*h_kv)";
+    case OPTR_ERR_OUT_OF_RANGE: return "size out of the supported range";
+    case OPTR_ERR_WORKSPACE: return "workspace missing or too small";
+    case OPTR_ERR_CUDA: return "CUDA runtime error";
+  }
+  return "unknown status";
+}
+
+optr_status optr_params_create(const optr_config* cfg, const float* R_k,
+                               const float* R_v, const float* mu,
+                               optr_params** out) {
+  if (out) *out = nullptr;
+  if (!cfg || !R_k || !R_v || !mu || !out) return OPTR_ERR_INVALID_ARG;
+  if (cfg->h_kv <= 0 || cfg->h_q <= 0 || cfg->h_q % cfg->h_kv != 0)
+    return OPTR_ERR_INVALID_ARG;
+  if (cfg->head_dim != kD || cfg->group != kG || cfg->page_size != kPage ||
+      cfg->h_q / cfg->h_kv != 4)
+    return OPTR_ERR_UNSUPPORTED;
+  if (!(cfg->clip_k > 0.f && cfg->clip_k <= 1.f) ||
+      !(cfg->clip_v > 0.f && cfg->clip_v <= 1.f))
+    return OPTR_ERR_INVALID_ARG;
+  if (cfg->h_kv > 1024) return OPTR_ERR_OUT_OF_RANGE;
+
+  const int H = cfg->h_kv;
+  const size_t mat = (size_t)kD * kD;
+  // Host-side preparation: mu R_k in fp64, R_v transposed.
+  std::vector<float> muR((size_t)H * kD), RvT((size_t)H * mat);
+  for (int h = 0; h < H; ++h) {
+    const float* R = R_k + h * mat;
+    for (int j = 0; j < kD; ++j) {
+      double acc = 0.0;
+      for (int i = 0; i < kD; ++i)
+        acc += (double)mu[h * kD + i] * (double)R[(size_t)i * kD + j];
+      muR[(size_t)h * kD + j] = (float)acc;
+    }
+    const float* Rv = R_v + h * mat;
+    for (int i = 0; i < kD; ++i)
+      for (int j = 0; j < kD; ++j)
+        RvT[h * mat + (size_t)j * kD + i] = Rv[(size_t)i * kD + j];
+  }
+
+  optr_params* p = (optr_params*)calloc(1, sizeof(optr_params));
+  if (!p) return OPTR_ERR_OUT_OF_RANGE;
+  p->cfg = *cfg;
+  p->ratio = cfg->h_q / cfg->h_kv;
+  cudaError_t e = cudaGetDevice(&p->device);
+  if (e == cudaSuccess)
+    e = cudaDeviceGetAttribute(&p->num_sms, cudaDevAttrMultiProcessorCount,
+                               p->device);
+  if (e == cudaSuccess) e = cudaMalloc(&p->R_k, sizeof(float) * H * mat);
+  if (e == cudaSuccess) e = cudaMalloc(&p->R_v, sizeof(float) * H * mat);
+  if (e == cudaSuccess) e = cudaMalloc(&p->R_vT, sizeof(float) * H * mat);
+  if (e == cudaSuccess) e = cudaMalloc(&p->muR, sizeof(float) * H * kD);
+  if (e == cudaSuccess) e = cudaMalloc(&p->err, sizeof(unsigned));
+  if (e == cudaSuccess)
+    e = cudaMemcpy(p->R_k, R_k, sizeof(float) * H * mat, cudaMemcpyHostToDevice);
+  if (e == cudaSuccess)
+    e = cudaMemcpy(p->R_v, R_v, sizeof(float) * H * mat, cudaMemcpyHostToDevice);
+  if (e == cudaSuccess)
+    e = cudaMemcpy(p->R_vT, RvT.data(), sizeof(float) * H * mat,
+                   cudaMemcpyHostToDevice);
+  if (e == cudaSuccess)
+    e = cudaMemcpy(p->muR, muR.data(), sizeof(float) * H * kD,
+                   cudaMemcpyHostToDevice);
+  if (e == cudaSuccess) e = cudaMemset(p->err, 0, sizeof(unsigned));
+  if (e != cudaSuccess) {
+    optr_params_destroy(p);
+    return OPTR_ERR_CUDA;
+  }
+  *out = p;
+  return OPTR_OK;
+}
+
+void optr_params_destroy(optr_params* p) {
+  if (!p) return;
+  optr_profile_enable(p, 0);
+  cudaFree(p->R_k);
+  cudaFree(p->R_v);
+  cudaFree(p->R_vT);
+  cudaFree(p->muR);
+  cudaFree(p->Rk_tc);
+  cudaFree(p->Rv_tc);
+  cudaFree(p->err);
+  free(p);
+}
+
+size_t optr_page_bytes(const optr_params* p) {
+  return p ? (size_t)p->cfg.h_kv * kChunk : 0;
+}
+
+optr_status optr_kv_append(const optr_params* p, const void* k, const void* v,
+                           int n_tok, const int32_t* cu_new,
+                           const int32_t* pos0, const int32_t* block_table,
+                           int B, int max_pages, uint8_t* pool, int num_pages,
+                           cudaStream_t stream) {
+  if (!p || n_tok < 0 || B <= 0 || max_pages <= 0 || num_pages <= 0)
+    return OPTR_ERR_INVALID_ARG;
+  if (n_tok == 0) return OPTR_OK;
+  if (!k || !v || !cu_new || !pos0 || !block_table || !pool)
+    return OPTR_ERR_INVALID_ARG;
+  if (!aligned(pool, 16) || !aligned(k, 16) || !aligned(v, 16))
+    return OPTR_ERR_INVALID_ARG;
+  if ((long long)max_pages * kPage > (1LL << 30)) return OPTR_ERR_OUT_OF_RANGE;
+  int variant = p->cfg.append_variant;
+  (void)variant;
+  prof_mark(p, 0, stream);
+  cudaError_t e = launch_append_cuda_core(
+      p, (const __nv_bfloat16*)k, (const __nv_bfloat16*)v, n_tok, cu_new, pos0,
+      block_table, B, max_pages, pool, num_pages, stream);
+  prof_mark(p, 1, stream);
+  if (p->prof) const_cast<optr_params*>(p)->ran[0] = 1;
+  return cuda_status(e);
+}
+
+size_t optr_decode_workspace_size(const optr_params* p, int B, int max_pages) {
+  if (!p || B <= 0 || max_pages <= 0) return 0;
+  return decode_plan(p, B, max_pages).total;
+}
+
+optr_status optr_decode_attention(const optr_params* p, const void* q,
+                                  const int32_t* block_table,
+                                  const int32_t* seq_lens, int B,
+                                  int max_pages, const uint8_t* pool,
+                                  int num_pages, float* out, void* workspace,
+                                  size_t ws_bytes, cudaStream_t stream) {
+  if (!p || B <= 0 || max_pages <= 0 || num_pages <= 0)
+    return OPTR_ERR_INVALID_ARG;
+  if (!q || !block_table || !seq_lens || !pool || !out)
+    return OPTR_ERR_INVALID_ARG;
+  if (!aligned(pool, 16) || !aligned(q, 16) || !aligned(out, 16))
+    return OPTR_ERR_INVALID_ARG;
+  if ((long long)max_pages * kPage > (1LL << 30) || B > (1 << 24))
+    return OPTR_ERR_OUT_OF_RANGE;
+  DecodePlan plan = decode_plan(p, B, max_pages);
+  if (!workspace || ws_bytes < plan.total || !aligned(workspace, 256))
+    return OPTR_ERR_WORKSPACE;
+  int variant = p->cfg.decode_variant;
+  cudaError_t e = launch_decode(p, variant, (const __nv_bfloat16*)q,
+                                block_table, seq_lens, B, max_pages, pool,
+                                num_pages, out, workspace, plan, stream);
+  if (p->prof) const_cast<optr_params*>(p)->ran[1] = 1;
+  return cuda_status(e);
+}
+
+optr_status optr_profile_enable(optr_params* p, int on) {
+  if (!p) return OPTR_ERR_INVALID_ARG;
+  if (on && !p->prof) {
+    for (int i = 0; i < 6; ++i)
+      if (cudaEventCreate(&p->ev[i]) != cudaSuccess) return OPTR_ERR_CUDA;
+    p->ran[0] = p->ran[1] = 0;
+    p->prof = 1;
+  } else if (!on && p->prof) {
+    for (int i = 0; i < 6; ++i) cudaEventDestroy(p->ev[i]);
+    p->prof = 0;
+  }
+  return OPTR_OK;
+}
+
+optr_status optr_profile_last(const optr_params* p, float ms[4]) {
+  if (!p || !ms) return OPTR_ERR_INVALID_ARG;
+  for (int i = 0; i < 4; ++i) ms[i] = 0.f;
+  if (!p->prof) return OPTR_ERR_INVALID_ARG;
+  cudaError_t e = cudaSuccess;
+  if (p->ran[0]) {
+    e = cudaEventSynchronize(p->ev[1]);
+    if (e == cudaSuccess) e = cudaEventElapsedTime(&ms[0], p->ev[0], p->ev[1]);
+  }
+  if (e == cudaSuccess && p->ran[1]) {
+    e = cudaEventSynchronize(p->ev[5]);
+    for (int i = 0; i < 3 && e == cudaSuccess; ++i)
+      e = cudaEventElapsedTime(&ms[1 + i], p->ev[2 + i], p->ev[3 + i]);
+  }
+  return cuda_status(e);
+}
+
+optr_status optr_device_error(const optr_params* p, uint32_t* flags) {
+  if (!p || !flags) return OPTR_ERR_INVALID_ARG;
+  unsigned h = 0;
+  cudaError_t e = cudaDeviceSynchronize();
+  if (e == cudaSuccess)
+    e = cudaMemcpy(&h, p->err, sizeof(unsigned), cudaMemcpyDeviceToHost);
+  if (e == cudaSuccess) e = cudaMemset(p->err, 0, sizeof(unsigned));
+  *flags = h;
+  return cuda_status(e);
+}
+
+}  // extern "C"

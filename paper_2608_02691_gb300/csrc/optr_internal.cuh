@@ -1,0 +1,79 @@
+// Internal declarations shared by the library's translation units.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "optr.h"
+
+namespace optr {
+
+constexpr int kD = OPTR_HEAD_DIM;        // 128
+constexpr int kG = OPTR_GROUP;           // 32
+constexpr int kGroups = kD / kG;         // 4
+constexpr int kPage = OPTR_PAGE_SIZE;    // 16
+constexpr int kChunk = OPTR_PAGE_HEAD_BYTES;
+constexpr int kMaxRatio = 8;             // largest supported h_q / h_kv
+
+// Decode split-K: every decode launch uses this many warps per SM for the
+// partial kernel; the workspace holds one partial slot per warp plus one per
+// (sequence, KV head), see DecodePlan.
+constexpr int kDecodeWarpsPerSm = 16;
+
+}  // namespace optr
+
+struct optr_params {
+  optr_config cfg;
+  int device;
+  int num_sms;
+  int ratio;           // h_q / h_kv
+  float* R_k;          // device [h_kv][D][D]
+  float* R_v;          // device [h_kv][D][D]
+  float* R_vT;         // device [h_kv][D][D], R_vT[h][j][i] = R_v[h][i][j]
+  float* muR;          // device [h_kv][D], mu R_k computed in fp64
+  __half* Rk_tc;       // device tensor-core operand of R_k (see append.cu)
+  __half* Rv_tc;       // device tensor-core operand of R_v
+  unsigned* err;       // device error word
+  // stage timing (optr_profile_enable): ev[0..1] bracket the append kernel,
+  // ev[2..5] the decode stages (before qrot, partial, combine, after).
+  int prof;
+  cudaEvent_t ev[6];
+  int ran[2];          // append ran / decode ran since enable
+};
+
+namespace optr {
+// Record stage event i on stream s when profiling is on.
+inline void prof_mark(const optr_params* p, int i, cudaStream_t s) {
+  if (p->prof) cudaEventRecord(p->ev[i], s);
+}
+}  // namespace optr
+
+namespace optr {
+
+// Byte offsets of the decode workspace for a batch shape.
+struct DecodePlan {
+  int B, h_q, h_kv, max_pages, W;  // W = partial-kernel warps
+  size_t off_qf, off_qs, off_pref, off_part, total;
+};
+DecodePlan decode_plan(const optr_params* p, int B, int max_pages);
+
+// One split-K partial: per query head of the GQA group, running max m
+// (log2 domain), sum l, and the unnormalised rotated output o'[128].
+constexpr int kPartFloats = 4 * (kD + 2);
+
+// Launchers (return cudaGetLastError()).
+cudaError_t launch_append_cuda_core(const optr_params* p, const __nv_bfloat16* k,
+                                    const __nv_bfloat16* v, int n_tok,
+                                    const int32_t* cu_new, const int32_t* pos0,
+                                    const int32_t* bt, int B, int max_pages,
+                                    uint8_t* pool, int num_pages,
+                                    cudaStream_t s);
+cudaError_t launch_decode(const optr_params* p, int variant,
+                          const __nv_bfloat16* q, const int32_t* bt,
+                          const int32_t* seq_lens, int B, int max_pages,
+                          const uint8_t* pool, int num_pages, float* out,
+                          void* ws, const DecodePlan& plan, cudaStream_t s);
+
+}  // namespace optr

@@ -1,0 +1,223 @@
+"""Thin ctypes binding of the C ABI in ``include/optr.h``.
+
+Function names match the C entry points.  The binding only marshals
+arguments: torch tensors become raw device pointers, the current torch CUDA
+stream becomes the ``cudaStream_t``, and negative status codes raise
+``OptrError``.  Every step of the computation runs in ``liboptr.so``; if the
+library has not been built, the first call raises instead of falling back to
+anything else.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import torch
+
+from . import build as _build
+
+_lib = None
+_lock = threading.Lock()
+
+OPTR_VARIANT_DEFAULT = 0
+OPTR_VARIANT_CUDA_CORE = 1
+OPTR_VARIANT_TENSOR = 2
+PAGE_HEAD_BYTES = 1536
+HEAD_DIM = 128
+
+
+class OptrError(RuntimeError):
+    def __init__(self, status: int, what: str):
+        super().__init__(f"{what}: {optr_strerror(status)} (status {status})")
+        self.status = status
+
+
+class optr_config(ctypes.Structure):
+    _fields_ = [("h_q", ctypes.c_int), ("h_kv", ctypes.c_int),
+                ("head_dim", ctypes.c_int), ("group", ctypes.c_int),
+                ("page_size", ctypes.c_int), ("clip_k", ctypes.c_float),
+                ("clip_v", ctypes.c_float), ("append_variant", ctypes.c_int),
+                ("decode_variant", ctypes.c_int)]
+
+
+_V = ctypes.c_void_p
+_I = ctypes.c_int
+_SIG = {
+    "optr_params_create": (_I, [ctypes.POINTER(optr_config), _V, _V, _V,
+                                ctypes.POINTER(_V)]),
+    "optr_params_destroy": (None, [_V]),
+    "optr_page_bytes": (ctypes.c_size_t, [_V]),
+    "optr_kv_append": (_I, [_V, _V, _V, _I, _V, _V, _V, _I, _I, _V, _I, _V]),
+    "optr_decode_workspace_size": (ctypes.c_size_t, [_V, _I, _I]),
+    "optr_decode_attention": (_I, [_V, _V, _V, _V, _I, _I, _V, _I, _V, _V,
+                                   ctypes.c_size_t, _V]),
+    "optr_device_error": (_I, [_V, ctypes.POINTER(ctypes.c_uint32)]),
+    "optr_strerror": (ctypes.c_char_p, [_I]),
+    "optr_profile_enable": (_I, [_V, _I]),
+    "optr_profile_last": (_I, [_V, ctypes.POINTER(ctypes.c_float)]),
+}
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def lib():
+    """The loaded ``liboptr.so``; raises if it has not been built."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            path = _build.LIB
+            if not os.path.exists(path):
+                raise RuntimeError(
+                    f"{path} is missing: build the CUDA library first "
+                    "(python -c 'import __graft_entry__ as g; g.build()')")
+            L = ctypes.CDLL(path)
+            for name, (res, args) in _SIG.items():
+                fn = getattr(L, name)
+                fn.restype = res
+                fn.argtypes = args
+            _lib = L
+    return _lib
+
+
+def optr_strerror(status: int) -> str:
+    return lib().optr_strerror(int(status)).decode()
+
+
+def _check(status: int, what: str):
+    if status != 0:
+        raise OptrError(status, what)
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _dev(t, dtype, name):
+    if not (t.is_cuda and t.dtype == dtype and t.is_contiguous()):
+        raise ValueError(f"{name} must be a contiguous CUDA {dtype} tensor")
+    return t
+
+
+class Params:
+    """Owner of an ``optr_params*`` handle (destroyed with the object)."""
+
+    def __init__(self, handle, cfg: optr_config):
+        self.handle = handle
+        self.cfg = cfg
+
+    def __del__(self):
+        h, self.handle = getattr(self, "handle", None), None
+        if h and _lib is not None:
+            _lib.optr_params_destroy(h)
+
+    @property
+    def h_q(self):
+        return self.cfg.h_q
+
+    @property
+    def h_kv(self):
+        return self.cfg.h_kv
+
+
+def optr_params_create(R_k, R_v, mu, h_q: int, clip_k: float = 1.0,
+                       clip_v: float = 1.0,
+                       append_variant: int = OPTR_VARIANT_DEFAULT,
+                       decode_variant: int = OPTR_VARIANT_DEFAULT) -> Params:
+    """R_k, R_v float32 [h_kv][128][128] and mu float32 [h_kv][128] (host
+    tensors); the library copies them to the current CUDA device."""
+    R_k = R_k.detach().to("cpu", torch.float32).contiguous()
+    R_v = R_v.detach().to("cpu", torch.float32).contiguous()
+    mu = mu.detach().to("cpu", torch.float32).contiguous()
+    h_kv = R_k.shape[0]
+    if R_k.shape != (h_kv, 128, 128) or R_v.shape != R_k.shape or \
+            mu.shape != (h_kv, 128):
+        raise ValueError("R_k, R_v must be [h_kv][128][128], mu [h_kv][128]")
+    cfg = optr_config(h_q, h_kv, 128, 32, 16, clip_k, clip_v, append_variant,
+                      decode_variant)
+    h = ctypes.c_void_p()
+    _check(lib().optr_params_create(ctypes.byref(cfg), _ptr(R_k), _ptr(R_v),
+                                    _ptr(mu), ctypes.byref(h)),
+           "optr_params_create")
+    return Params(h, cfg)
+
+
+def optr_page_bytes(p: Params) -> int:
+    return int(lib().optr_page_bytes(p.handle))
+
+
+def optr_kv_append(p: Params, k, v, cu_new, pos0, block_table, pool,
+                   stream=None) -> None:
+    """k, v bf16 [n_tok][h_kv][128]; cu_new int32 [B+1]; pos0 int32 [B];
+    block_table int32 [B][max_pages]; pool uint8 [num_pages][h_kv][1536]."""
+    _dev(k, torch.bfloat16, "k")
+    _dev(v, torch.bfloat16, "v")
+    _dev(cu_new, torch.int32, "cu_new")
+    _dev(pos0, torch.int32, "pos0")
+    _dev(block_table, torch.int32, "block_table")
+    _dev(pool, torch.uint8, "pool")
+    B, max_pages = block_table.shape
+    _check(lib().optr_kv_append(p.handle, _ptr(k), _ptr(v), k.shape[0],
+                                _ptr(cu_new), _ptr(pos0), _ptr(block_table),
+                                B, max_pages, _ptr(pool), pool.shape[0],
+                                _stream(stream)),
+           "optr_kv_append")
+
+
+def optr_decode_workspace_size(p: Params, B: int, max_pages: int) -> int:
+    return int(lib().optr_decode_workspace_size(p.handle, B, max_pages))
+
+
+def optr_decode_attention(p: Params, q, block_table, seq_lens, pool, out,
+                          workspace, stream=None) -> None:
+    """q bf16 [B][h_q][128]; out float32 [B][h_q][128]; workspace uint8 of
+    at least optr_decode_workspace_size bytes (256-byte aligned)."""
+    _dev(q, torch.bfloat16, "q")
+    _dev(block_table, torch.int32, "block_table")
+    _dev(seq_lens, torch.int32, "seq_lens")
+    _dev(pool, torch.uint8, "pool")
+    _dev(out, torch.float32, "out")
+    _dev(workspace, torch.uint8, "workspace")
+    B, max_pages = block_table.shape
+    _check(lib().optr_decode_attention(
+        p.handle, _ptr(q), _ptr(block_table), _ptr(seq_lens), B, max_pages,
+        _ptr(pool), pool.shape[0], _ptr(out), _ptr(workspace),
+        workspace.numel(), _stream(stream)), "optr_decode_attention")
+
+
+def optr_device_error(p: Params) -> int:
+    flags = ctypes.c_uint32(0)
+    _check(lib().optr_device_error(p.handle, ctypes.byref(flags)),
+           "optr_device_error")
+    return int(flags.value)
+
+
+def optr_profile_enable(p: Params, on: bool = True) -> None:
+    _check(lib().optr_profile_enable(p.handle, int(bool(on))),
+           "optr_profile_enable")
+
+
+def optr_profile_last(p: Params) -> dict:
+    """Durations (ms) of the stages of the most recent append / decode."""
+    ms = (ctypes.c_float * 4)()
+    _check(lib().optr_profile_last(p.handle, ms), "optr_profile_last")
+    return {"append": ms[0], "qrot": ms[1], "partial": ms[2], "combine": ms[3]}
+
+
+def new_pool(p: Params, num_pages: int, device="cuda") -> torch.Tensor:
+    """A zero-filled pool tensor [num_pages][h_kv][1536] (uint8)."""
+    return torch.zeros(num_pages, p.h_kv, PAGE_HEAD_BYTES, dtype=torch.uint8,
+                       device=device)
+
+
+def new_workspace(p: Params, B: int, max_pages: int, device="cuda"):
+    n = optr_decode_workspace_size(p, B, max_pages)
+    return torch.empty(n, dtype=torch.uint8, device=device)
