@@ -167,9 +167,12 @@ class Flusher:
         self.buf.fill_(1.0)
 
 
-def setup_decode(name, seed, dev, variant, append_variant):
+def setup_decode(name, seed, dev, variant, append_variant, batch=None):
     from paper_2608_02691_gb300 import optr, synth
     wl = synth.workload(name, seed)
+    if batch:
+        wl.B = batch
+        wl.ctx = [wl.ctx[0]] * batch
     case = synth.build_case(wl, seed, device=dev)
     p = optr.optr_params_create(case["R_k"], case["R_v"], case["mu"],
                                 case["h_q"], decode_variant=variant,
@@ -202,7 +205,8 @@ def run_ours(args, rank, world, dev):
 
     # ---------------- main step: decode8k (append 1 token/seq + decode)
     wl, case, p, pool, bt = setup_decode("decode8k", args.seed, dev,
-                                         args.variant, args.append_variant)
+                                         args.variant, args.append_variant,
+                                         args.batch)
     B, h_q, h_kv = case["B"], case["h_q"], case["h_kv"]
     seq = case["seq_lens"].to(dev)
     q = case["q"].to(dev)
@@ -254,13 +258,46 @@ def run_ours(args, rank, world, dev):
     optr.optr_profile_enable(p, False)
     stage_ms = {k2: float(np.mean(v)) for k2, v in stages.items()}
 
-    # end to end through the public API with host buffers
-    q_h = case["q"].pin_memory()
-    k_h, v_h = case["k_new"].pin_memory(), case["v_new"].pin_memory()
+    if args.no_e2e:
+        e2e_ms, h2d, d2h = float("nan"), 0, 0
+    else:
+        e2e_ms, h2d, d2h = e2e_time(args, case, p, pool, bt, seq, cu_new, pos0,
+                                    out, ws, flush, stream, world, dev)
+    # roofline of the dominant kernel (split-K partial)
+    part_bytes = decode_stream_bytes(case["seq_lens"].tolist(), h_kv)
+    achieved = part_bytes / (stage_ms["partial"] * 1e-3) / 1e9
+    variant_files = (["decode_tc.cu", "decode_common.cuh"]
+                     if args.variant != 1 else ["decode.cu", "decode_common.cuh"])
+    key = "partial_tensor" if args.variant != 1 else "partial_cuda_core"
+    traffic = traffic_for(key, variant_files)
+    roofline = {"bound": "hbm", "kernel": key, "achieved": round(achieved, 1),
+                "peak": hbm_peak, "peak_source": peak_src, "unit": "GB/s",
+                "frac": round(achieved / hbm_peak, 4),
+                "frac_of_nominal_8000": round(achieved / 8000.0, 4),
+                "traffic": traffic,
+                "algorithmic_bytes_per_launch": part_bytes,
+                "launch_ms": round(stage_ms["partial"], 5)}
+
+    result["main"] = dict(ms=ms_max, bytes=step_bytes, stage_ms=stage_ms,
+                          e2e_ms=e2e_ms, h2d=h2d, d2h=d2h, roofline=roofline,
+                          clocks=clk, case=case, pool=pool, p=p)
+    return result
+
+
+def e2e_time(args, case, p, pool, bt, seq, cu_new, pos0, out, ws, flush,
+             stream, world, dev):
+    """The step through the public API with inputs from pinned host memory
+    (query and the new K/V token of every sequence) and the output read
+    back to pinned host memory, all inside the timed region."""
+    from paper_2608_02691_gb300 import optr
+    B, h_q = case["B"], case["h_q"]
+    q_h = case["q"].cpu().pin_memory()
+    k_h, v_h = case["k_new"].cpu().pin_memory(), case["v_new"].cpu().pin_memory()
     out_h = torch.empty(B, h_q, D, dtype=torch.float32).pin_memory()
     h2d = q_h.numel() * 2 + k_h.numel() * 2 + v_h.numel() * 2
     d2h = out_h.numel() * 4
-    q_d, k_d, v_d = torch.empty_like(q), torch.empty_like(k_new), torch.empty_like(v_new)
+    q_d = torch.empty_like(q_h, device=dev)
+    k_d, v_d = torch.empty_like(k_h, device=dev), torch.empty_like(v_h, device=dev)
 
     def e2e_step():
         q_d.copy_(q_h, non_blocking=True)
@@ -283,27 +320,7 @@ def run_ours(args, rank, world, dev):
         e2e_ev[i][1].record(stream)
     torch.cuda.synchronize()
     e2e_ms = float(np.mean([a.elapsed_time(b) for a, b in e2e_ev]))
-    e2e_ms = allreduce_max(e2e_ms, world, dev)
-
-    # roofline of the dominant kernel (split-K partial)
-    part_bytes = decode_stream_bytes(case["seq_lens"].tolist(), h_kv)
-    achieved = part_bytes / (stage_ms["partial"] * 1e-3) / 1e9
-    variant_files = (["decode_tc.cu", "decode_common.cuh"]
-                     if args.variant != 1 else ["decode.cu", "decode_common.cuh"])
-    key = "partial_tensor" if args.variant != 1 else "partial_cuda_core"
-    traffic = traffic_for(key, variant_files)
-    roofline = {"bound": "hbm", "kernel": key, "achieved": round(achieved, 1),
-                "peak": hbm_peak, "peak_source": peak_src, "unit": "GB/s",
-                "frac": round(achieved / hbm_peak, 4),
-                "frac_of_nominal_8000": round(achieved / 8000.0, 4),
-                "traffic": traffic,
-                "algorithmic_bytes_per_launch": part_bytes,
-                "launch_ms": round(stage_ms["partial"], 5)}
-
-    result["main"] = dict(ms=ms_max, bytes=step_bytes, stage_ms=stage_ms,
-                          e2e_ms=e2e_ms, h2d=h2d, d2h=d2h, roofline=roofline,
-                          clocks=clk, case=case, pool=pool, p=p)
-    return result
+    return allreduce_max(e2e_ms, world, dev), h2d, d2h
 
 
 def extra_workloads(args, dev):
@@ -379,90 +396,93 @@ def extra_workloads(args, dev):
 
 # ---------------------------------------------------------- CPU baseline
 
-def cpu_baseline(case, pool_gpu, n_groups, threads):
-    """The oracle, as it stands, on a bounded sample of the main workload:
-    the decode of n_groups (sequence, KV head) groups (4 query heads each)
-    over their full contexts.  Returns GB/s on the same byte accounting."""
+def oracle_sample(case, n_seqs, threads):
+    """The oracle, as it stands, on the first n_seqs sequences of a decode
+    workload: its own cache write of their context (untimed set-up), then a
+    step() closure = oracle append of their new token + oracle decode of all
+    their query heads over the full context.  Inputs come from the seeded
+    generator only.  Returns (step, bytes_per_step, description)."""
     from oracle import oracle
     from paper_2608_02691_gb300 import synth
     oracle.build()
     oracle.set_threads(threads)
-    pool = pool_gpu.cpu().numpy()
-    rows = []
-    B, h_kv = case["B"], case["h_kv"]
-    groups = [(b, h) for b in range(B) for h in range(h_kv)][:n_groups]
-    for b, h in groups:
-        rows += [(b, 4 * h + r) for r in range(4)]
-    qb = synth.bf16_bits(case["q"])
+    B = n_seqs
+    cu = case["cu_ctx"][:B + 1]
+    n_ctx = int(cu[-1])
+    h_kv, h_q = case["h_kv"], case["h_q"]
+    bt = case["block_table"][:B].numpy()
+    used = np.unique(bt[bt >= 0])
+    remap = np.full(case["num_pages"], -1, np.int64)
+    remap[used] = np.arange(used.size)
+    bt = np.where(bt >= 0, remap[np.maximum(bt, 0)], -1).astype(np.int32)
+    pool = np.zeros((used.size, h_kv, CHUNK), np.uint8)
+    R = (case["R_k"].numpy(), case["R_v"].numpy(), case["mu"].numpy())
+    oracle.kv_append(synth.bf16_bits(case["k_ctx"][:n_ctx]),
+                     synth.bf16_bits(case["v_ctx"][:n_ctx]), cu.numpy(),
+                     case["pos0_ctx"][:B].numpy(), bt, pool, *R)
+    n_new = int(case["cu_new"][B])
+    kb = synth.bf16_bits(case["k_new"][:n_new])
+    vb = synth.bf16_bits(case["v_new"][:n_new])
+    qb = synth.bf16_bits(case["q"][:B])
+    cu_new = case["cu_new"][:B + 1].numpy()
+    pos0 = case["pos0_new"][:B].numpy()
+    lens = case["seq_lens"][:B].numpy()
+
+    def step():
+        oracle.kv_append(kb, vb, cu_new, pos0, bt, pool, *R)
+        oracle.decode_attention(qb, bt, lens, pool, R[0], R[1], h_kv)
+
+    nb = decode_bytes(lens.tolist(), h_kv, h_q) + append_bytes(n_new, h_kv)
+    desc = (f"{B} of {case['B']} sequences of the batch-{case['B']} x "
+            f"{int(lens[0])}-token decode step (append 1 token + decode, all "
+            f"{h_kv} KV heads / {h_q} query heads)")
+    return step, nb, desc
+
+
+def cpu_baseline(case, n_seqs, threads, reps=2):
+    step, nb, desc = oracle_sample(case, n_seqs, threads)
+    step()
     t0 = time.perf_counter()
-    oracle.decode_attention(qb, case["block_table"].numpy(),
-                            case["seq_lens"].numpy(), pool, case["R_k"].numpy(),
-                            case["R_v"].numpy(), h_kv, rows=rows)
-    dt = time.perf_counter() - t0
-    lens = case["seq_lens"].tolist()
-    nb = sum(lens[b] * 96 + 4 * D * 6 for b, _ in groups)
+    for _ in range(reps):
+        step()
+    dt = (time.perf_counter() - t0) / reps
     return {"value": round(nb / dt / 1e9, 4), "unit": "GB/s", "cores": threads,
-            "kind": "oracle", "seconds": round(dt, 2),
-            "sample": f"oracle decode of {len(groups)} of {B * h_kv} (sequence, KV head) "
-                      f"groups of the batch-16 x 8193-token step (4 query heads each)"}
+            "kind": "oracle", "seconds_per_step": round(dt, 3), "sample": desc}
 
 
 # ------------------------------------------------------------- reference
 
 def run_reference(args, rank, world):
-    """The oracle as the reference arm: each step = oracle append of the new
-    token of the sampled sequences + oracle decode of those sequences."""
+    """The oracle as the reference arm, on the same workload, metric and
+    unit: each step is the oracle's decode step on a bounded sample."""
     if rank != 0:
         return None
-    from oracle import oracle
     from paper_2608_02691_gb300 import synth
-    oracle.build()
     threads = os.cpu_count() or 1
-    oracle.set_threads(threads)
-    wl = synth.workload("decode8k", args.seed)
-    wl.B = args.ref_seqs
-    wl.ctx = wl.ctx[:args.ref_seqs]
-    case = synth.build_case(wl, args.seed)
-    bt = case["block_table"].numpy()
-    pool = np.zeros((case["num_pages"], case["h_kv"], CHUNK), np.uint8)
-    R = (case["R_k"].numpy(), case["R_v"].numpy(), case["mu"].numpy())
-    oracle.kv_append(synth.bf16_bits(case["k_ctx"]), synth.bf16_bits(case["v_ctx"]),
-                     case["cu_ctx"].numpy(), case["pos0_ctx"].numpy(), bt, pool, *R)
-    qb = synth.bf16_bits(case["q"])
-    kb, vb = synth.bf16_bits(case["k_new"]), synth.bf16_bits(case["v_new"])
-
-    def step():
-        oracle.kv_append(kb, vb, case["cu_new"].numpy(), case["pos0_new"].numpy(),
-                         bt, pool, *R)
-        oracle.decode_attention(qb, bt, case["seq_lens"].numpy(), pool,
-                                case["R_k"].numpy(), case["R_v"].numpy(),
-                                case["h_kv"])
-
+    case = synth.build_case(synth.workload("decode8k", args.seed), args.seed)
+    step, nb, desc = oracle_sample(case, args.ref_seqs, threads)
     for _ in range(args.warmup):
         step()
     t0 = time.perf_counter()
     for _ in range(args.steps):
         step()
     dt = (time.perf_counter() - t0) / args.steps
-    nb = (decode_bytes(case["seq_lens"].tolist(), case["h_kv"], case["h_q"]) +
-          append_bytes(case["k_new"].shape[0], case["h_kv"]))
     v = nb / dt / 1e9
-    sample = (f"{args.ref_seqs} of 16 sequences of the batch-16 x 8193-token "
-              f"decode step (append 1 token + decode, all 8 KV heads)")
     return {"impl": "reference", "metric": METRIC, "value": round(v, 4),
             "unit": "GB/s", "n_gpus": 1, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": round(dt * 1e3, 3),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "f64", "data": "synthetic",
-            "config": {"workload": "decode8k: batch 16, 32 q / 8 kv heads, "
-                                   "head_dim 128, context 8192+1, page 16",
-                       "sample_sequences": args.ref_seqs},
+            "config": {"workload": WORKLOAD_DESC, "sample_sequences": args.ref_seqs},
             "cpu_baseline": {"value": round(v, 4), "unit": "GB/s",
-                             "cores": threads, "kind": "oracle", "sample": sample},
+                             "cores": threads, "kind": "oracle", "sample": desc},
             "e2e": {"value": round(v, 4), "unit": "GB/s",
                     "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
 
 
+WORKLOAD_DESC = ("decode8k: batch 16 x context 8192 (+1 appended token per "
+                 "sequence), 32 q / 8 kv heads, head_dim 128, page 16, "
+                 "shuffled pages, Student-t(4) K/V")
 METRIC = "decode-attention HBM GB/s (decode step: append 1 token/seq + decode)"
 
 
@@ -490,10 +510,13 @@ def main():
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--variant", type=int, default=0)
     ap.add_argument("--append-variant", type=int, default=0)
-    ap.add_argument("--ref-seqs", type=int, default=2)
-    ap.add_argument("--cpu-groups", type=int, default=128)
+    ap.add_argument("--ref-seqs", type=int, default=4)
+    ap.add_argument("--cpu-seqs", type=int, default=16)
     ap.add_argument("--no-extra", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--batch", type=int, default=0,
+                    help="override the decode8k batch (profiling cases)")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
 
@@ -521,28 +544,31 @@ def main():
     extra = extra_workloads(args, dev) if (rank == 0 and not args.no_extra) else None
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu:
-        cpu = cpu_baseline(m["case"], m["pool"], args.cpu_groups, os.cpu_count() or 1)
+        case_cpu = {k: (v.cpu() if torch.is_tensor(v) else v)
+                    for k, v in m["case"].items()}
+        del m["pool"], m["case"]
+        cpu = cpu_baseline(case_cpu, args.cpu_seqs, os.cpu_count() or 1)
     if rank == 0:
         value = m["bytes"] * world / (m["ms"] * 1e-3) / 1e9
-        e2e = m["bytes"] * world / (m["e2e_ms"] * 1e-3) / 1e9
+        e2e = (None if not np.isfinite(m["e2e_ms"]) else
+               m["bytes"] * world / (m["e2e_ms"] * 1e-3) / 1e9)
         line = {
             "metric": METRIC, "value": round(value, 2), "unit": "GB/s",
             "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": round(m["ms"], 5), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "int2+fp16 meta, f32 math",
             "data": "synthetic",
-            "config": {"workload": "decode8k: batch 16 x context 8192 (+1 appended "
-                                   "token per sequence), 32 q / 8 kv heads, head_dim 128, "
-                                   "page 16, shuffled pages, Student-t(4) K/V",
+            "config": {"workload": WORKLOAD_DESC,
                        "bytes_per_step": m["bytes"], "l2": "flushed (512 MiB write) "
                        "before every timed step; step timed alone with CUDA events",
                        "decode_variant": args.variant, "append_variant": args.append_variant},
             "gpu_launches": 4 * args.steps,
             "stage_ms": {k: round(v, 5) for k, v in m["stage_ms"].items()},
             "roofline": m["roofline"],
-            "e2e": {"value": round(e2e, 2), "unit": "GB/s",
-                    "h2d_bytes_per_step": m["h2d"], "d2h_bytes_per_step": m["d2h"],
-                    "ms_per_step": round(m["e2e_ms"], 5)},
+            "e2e": None if e2e is None else {
+                "value": round(e2e, 2), "unit": "GB/s",
+                "h2d_bytes_per_step": m["h2d"], "d2h_bytes_per_step": m["d2h"],
+                "ms_per_step": round(m["e2e_ms"], 5)},
             "clocks": m["clocks"],
             "cpu_baseline": cpu,
             "workloads": extra,

@@ -103,6 +103,7 @@ append_cuda_core_kernel(const __nv_bfloat16* __restrict__ k,
   float acc[T];
 #pragma unroll
   for (int t = 0; t < T; ++t) acc[t] = 0.f;
+#pragma unroll 8
   for (int i = 0; i < kD; ++i) {
     float r = __ldg(R + i * kD + j);
 #pragma unroll
@@ -147,12 +148,22 @@ cudaError_t launch_append_cuda_core(const optr_params* p,
                                     const int32_t* bt, int B, int max_pages,
                                     uint8_t* pool, int num_pages,
                                     cudaStream_t s) {
-  constexpr int T = 32;
-  dim3 grid((n_tok + T - 1) / T, p->cfg.h_kv);
-  append_cuda_core_kernel<T><<<grid, 256, 0, s>>>(
-      k, v, n_tok, cu_new, pos0, bt, B, max_pages, pool, num_pages,
-      p->cfg.h_kv, p->R_k, p->R_v, p->muR, p->cfg.clip_k, p->cfg.clip_v,
-      p->err);
+  // few tokens (decode steps): small tiles for more blocks in flight
+  if (n_tok <= 2048) {
+    constexpr int T = 4;
+    dim3 grid((n_tok + T - 1) / T, p->cfg.h_kv);
+    append_cuda_core_kernel<T><<<grid, 256, 0, s>>>(
+        k, v, n_tok, cu_new, pos0, bt, B, max_pages, pool, num_pages,
+        p->cfg.h_kv, p->R_k, p->R_v, p->muR, p->cfg.clip_k, p->cfg.clip_v,
+        p->err);
+  } else {
+    constexpr int T = 32;
+    dim3 grid((n_tok + T - 1) / T, p->cfg.h_kv);
+    append_cuda_core_kernel<T><<<grid, 256, 0, s>>>(
+        k, v, n_tok, cu_new, pos0, bt, B, max_pages, pool, num_pages,
+        p->cfg.h_kv, p->R_k, p->R_v, p->muR, p->cfg.clip_k, p->cfg.clip_v,
+        p->err);
+  }
   return cudaGetLastError();
 }
 

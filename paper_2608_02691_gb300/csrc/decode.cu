@@ -27,8 +27,11 @@ qrot_kernel(const __nv_bfloat16* __restrict__ q, const float* __restrict__ R_k,
             int B, int h_q, int h_kv, float qscale,
             const int32_t* __restrict__ seq_lens, int max_pages,
             float* __restrict__ qf, float* __restrict__ qs,
+            uint32_t* __restrict__ frag, float* __restrict__ invs,
             int* __restrict__ pref, int* __restrict__ nzpref, unsigned* err) {
   __shared__ float qsm[4][kD];
+  __shared__ float qrs[4][kD];
+  __shared__ float hmax[4][4];
   __shared__ int warp_tot[2][4];
   const int b = blockIdx.x, h = blockIdx.y, j = threadIdx.x;
   const int warp = j >> 5, lane = j & 31;
@@ -48,10 +51,49 @@ qrot_kernel(const __nv_bfloat16* __restrict__ q, const float* __restrict__ R_k,
     const float x = acc[r] * qscale;
     const size_t row = (size_t)b * h_q + 4 * h + r;
     qf[row * kD + j] = x;
-    float s = x;
+    qrs[r][j] = x;
+    float s = x, a = fabsf(x);
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-    if (lane == 0) qs[row * kGroups + warp] = s;  // warp == group
+    for (int o = 16; o > 0; o >>= 1) {
+      s += __shfl_xor_sync(0xffffffffu, s, o);
+      a = fmaxf(a, __shfl_xor_sync(0xffffffffu, a, o));
+    }
+    if (lane == 0) {
+      qs[row * kGroups + warp] = s;  // warp == group
+      hmax[r][warp] = a;
+    }
+  }
+  __syncthreads();
+  // Tensor-core B fragments (see decode_tc.cu): per head a power-of-two
+  // prescale 2^e keeps |q'| * 2^e below 2^14, so that the fp16 hi/lo split
+  // (and the 4^-r factors that undo the unshifted code masks) stay normal.
+  int e[4];
+#pragma unroll
+  for (int r = 0; r < 4; ++r) {
+    const float mx = fmaxf(fmaxf(hmax[r][0], hmax[r][1]), fmaxf(hmax[r][2], hmax[r][3]));
+    e[r] = mx > 0.f ? 13 - ilogbf(mx) : 0;
+    e[r] = max(-100, min(100, e[r]));
+  }
+  if (j < 4) invs[(size_t)b * h_q + 4 * h + j] = ldexpf(1.f, 24 - e[j]);
+  uint32_t* fb = frag + ((size_t)b * h_kv + h) * 512;
+#pragma unroll
+  for (int t = 0; t < 4; ++t) {
+    const int ridx = j + 128 * t;          // 512 fragment registers
+    const int L = ridx >> 4, reg = ridx & 15;
+    const int G = reg >> 2, kk = (reg >> 1) & 1, which = reg & 1;
+    const int g = L >> 2, c = L & 3;
+    const int head = g >> 1, part = g & 1;
+    const int ch = 32 * G + 8 * c + 2 * kk + which;   // low half; +4 high
+    const float sc = ldexpf(1.f, e[head] - 2 * (2 * kk + which));
+    const float x0 = qrs[head][ch] * sc, x1 = qrs[head][ch + 4] * sc;
+    const __half h0 = __float2half_rn(x0), h1 = __float2half_rn(x1);
+    __half v0 = h0, v1 = h1;
+    if (part) {
+      v0 = __float2half_rn(x0 - __half2float(h0));
+      v1 = __float2half_rn(x1 - __half2float(h1));
+    }
+    fb[L * 16 + reg] = (uint32_t)__half_as_ushort(v0) |
+                       ((uint32_t)__half_as_ushort(v1) << 16);
   }
 
   if (b != 0 || h != 0) return;
@@ -238,10 +280,10 @@ partial_cuda_core_kernel(const uint8_t* __restrict__ pool,
 #pragma unroll
     for (int r = 0; r < 4; ++r)
 #pragma unroll
-      for (int c = 0; c < 4; ++c) dst[r * (kD + 2) + 32 * G + 4 * wd + c] = acc[r][c];
+      for (int c = 0; c < 4; ++c) dst[r * kD + 32 * G + 4 * wd + c] = acc[r][c];
     if (lane < 4) {
-      dst[lane * (kD + 2) + kD] = m[lane];
-      dst[lane * (kD + 2) + kD + 1] = l[lane];
+      dst[kPartM + lane] = m[lane];
+      dst[kPartL + lane] = l[lane];
     }
     f = sg.f_end;
   }
@@ -249,60 +291,100 @@ partial_cuda_core_kernel(const uint8_t* __restrict__ pool,
 
 // ------------------------------------------------------------- combine
 
-__global__ void __launch_bounds__(128)
+// One CTA per (sequence b, KV head h, query head r of the group); 1024
+// threads = 8 slices x 128 channels.  Merge weights exp2(m_i - M) / L of the
+// segment partials are computed once into shared memory (W + 1 floats of
+// dynamic shared memory), then every slice sums a strided subset of the
+// partials, and the merged o' is rotated back: out = o' R_v^T.
+constexpr int kCombineThreads = 1024;
+constexpr int kSlices = kCombineThreads / kD;
+
+__device__ __forceinline__ float block_reduce(float v, bool is_max, float* red) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float u = __shfl_xor_sync(0xffffffffu, v, o);
+    v = is_max ? fmaxf(v, u) : v + u;
+  }
+  __syncthreads();
+  if (lane == 0) red[warp] = v;
+  __syncthreads();
+  float t = red[0];
+  for (int i = 1; i < kCombineThreads / 32; ++i) t = is_max ? fmaxf(t, red[i]) : t + red[i];
+  return t;
+}
+
+__global__ void __launch_bounds__(kCombineThreads)
 combine_kernel(const float* __restrict__ part, const int* __restrict__ pref,
                const int* __restrict__ nzpref, int B, int h_q, int h_kv, int W,
                const float* __restrict__ R_vT, float* __restrict__ out) {
-  __shared__ float orot[4][kD];
-  __shared__ float coef[4][2];
-  const int b = blockIdx.x, h = blockIdx.y, j = threadIdx.x;
+  extern __shared__ float wts[];  // [W + 1]
+  __shared__ float red[kCombineThreads / 32];
+  __shared__ float osl[kSlices][kD];
+  __shared__ float orot[kD];
+  const int b = blockIdx.x, h = blockIdx.y, r = blockIdx.z;
+  const int tid = threadIdx.x, sl = tid / kD, j = tid % kD;
   const int np = __ldg(pref + b + 1) - __ldg(pref + b);
-  float* ob = out + ((size_t)b * h_q + 4 * h) * kD;
+  float* ob = out + ((size_t)b * h_q + 4 * h + r) * kD;
   if (np == 0) {
-#pragma unroll
-    for (int r = 0; r < 4; ++r) ob[r * kD + j] = 0.f;
+    if (tid < kD) ob[tid] = 0.f;
     return;
   }
   const long long F = (long long)__ldg(pref + B) * h_kv;
   const long long fs = (long long)__ldg(pref + b) * h_kv + (long long)h * np;
   const int w0 = warp_of(fs, F, W), w1 = warp_of(fs + np - 1, F, W);
-  const size_t base = (size_t)__ldg(nzpref + b) * h_kv + h;
-  if (j < 4) {
-    float M = -INFINITY;
-    for (int w = w0; w <= w1; ++w)
-      if (!warp_empty(w, F, W))
-        M = fmaxf(M, part[(base + w) * kPartFloats + j * (kD + 2) + kD]);
-    float L = 0.f;
-    for (int w = w0; w <= w1; ++w) {
-      if (warp_empty(w, F, W)) continue;
-      const float* pp = part + (base + w) * kPartFloats + j * (kD + 2);
-      L += pp[kD + 1] * merge_weight(pp[kD], M);
+  const int n = w1 - w0 + 1;
+  const float* pbase = part + ((size_t)__ldg(nzpref + b) * h_kv + h + w0) * kPartFloats;
+
+  float mloc = -INFINITY;
+  for (int i = tid; i < n; i += kCombineThreads)
+    if (!warp_empty(w0 + i, F, W))
+      mloc = fmaxf(mloc, __ldg(pbase + (size_t)i * kPartFloats + kPartM + r));
+  const float M = block_reduce(mloc, true, red);
+  float lloc = 0.f;
+  for (int i = tid; i < n; i += kCombineThreads) {
+    float wgt = 0.f;
+    if (!warp_empty(w0 + i, F, W)) {
+      const float* pp = pbase + (size_t)i * kPartFloats;
+      wgt = merge_weight(__ldg(pp + kPartM + r), M);
+      lloc += __ldg(pp + kPartL + r) * wgt;
     }
-    coef[j][0] = M;
-    coef[j][1] = L > 0.f ? 1.f / L : 0.f;
+    wts[i] = wgt;
   }
+  const float L = block_reduce(lloc, false, red);
+  const float invL = L > 0.f ? 1.f / L : 0.f;
+
+  float o = 0.f;
+#pragma unroll 4
+  for (int i = sl; i < n; i += kSlices) {
+    const float wgt = wts[i];
+    if (wgt != 0.f) o = fmaf(__ldg(pbase + (size_t)i * kPartFloats + r * kD + j), wgt, o);
+  }
+  osl[sl][j] = o;
   __syncthreads();
+  if (tid < kD) {
+    float t = 0.f;
 #pragma unroll
-  for (int r = 0; r < 4; ++r) {
-    const float M = coef[r][0];
-    float o = 0.f;
-    for (int w = w0; w <= w1; ++w) {
-      if (warp_empty(w, F, W)) continue;
-      const float* pp = part + (base + w) * kPartFloats + r * (kD + 2);
-      o += pp[j] * merge_weight(pp[kD], M);
-    }
-    orot[r][j] = o * coef[r][1];
+    for (int k = 0; k < kSlices; ++k) t += osl[k][tid];
+    orot[tid] = t * invL;
   }
   __syncthreads();
+  // out[i] = sum_jj o'[jj] R_v[i][jj] = sum_jj o'[jj] R_vT[jj][i]
   const float* RT = R_vT + (size_t)h * kD * kD;
-  float acc[4] = {0.f, 0.f, 0.f, 0.f};
-  for (int jj = 0; jj < kD; ++jj) {
-    const float rt = __ldg(RT + jj * kD + j);  // R_v[h][j][jj]
+  float acc = 0.f;
+  const int jj0 = sl * (kD / kSlices);
 #pragma unroll
-    for (int r = 0; r < 4; ++r) acc[r] = fmaf(orot[r][jj], rt, acc[r]);
+  for (int k = 0; k < kD / kSlices; ++k)
+    acc = fmaf(orot[jj0 + k], __ldg(RT + (jj0 + k) * kD + j), acc);
+  __syncthreads();
+  osl[sl][j] = acc;
+  __syncthreads();
+  if (tid < kD) {
+    float t = 0.f;
+#pragma unroll
+    for (int k = 0; k < kSlices; ++k) t += osl[k][tid];
+    ob[tid] = t;
   }
-#pragma unroll
-  for (int r = 0; r < 4; ++r) ob[r * kD + j] = acc[r];
 }
 
 }  // namespace
@@ -310,9 +392,10 @@ combine_kernel(const float* __restrict__ part, const int* __restrict__ pref,
 cudaError_t launch_partial_tensor(const optr_params* p, const uint8_t* pool,
                                   const int32_t* bt, const int32_t* seq_lens,
                                   int B, int max_pages, int num_pages,
-                                  const float* qf, const float* qs,
-                                  const int* pref, const int* nzpref,
-                                  float* part, int W, cudaStream_t s);
+                                  const uint32_t* frag, const float* invs,
+                                  const float* qs, const int* pref,
+                                  const int* nzpref, float* part, int W,
+                                  cudaStream_t s);
 
 cudaError_t launch_decode(const optr_params* p, int variant,
                           const __nv_bfloat16* q, const int32_t* bt,
@@ -322,6 +405,8 @@ cudaError_t launch_decode(const optr_params* p, int variant,
   char* w = static_cast<char*>(ws);
   float* qf = reinterpret_cast<float*>(w + plan.off_qf);
   float* qs = reinterpret_cast<float*>(w + plan.off_qs);
+  uint32_t* frag = reinterpret_cast<uint32_t*>(w + plan.off_frag);
+  float* invs = reinterpret_cast<float*>(w + plan.off_invs);
   int* pref = reinterpret_cast<int*>(w + plan.off_pref);
   int* nzpref = pref + (B + 1);
   float* part = reinterpret_cast<float*>(w + plan.off_part);
@@ -330,14 +415,14 @@ cudaError_t launch_decode(const optr_params* p, int variant,
 
   prof_mark(p, 2, s);
   qrot_kernel<<<dim3(B, h_kv), 128, 0, s>>>(q, p->R_k, B, h_q, h_kv, qscale,
-                                            seq_lens, max_pages, qf, qs, pref,
-                                            nzpref, p->err);
+                                            seq_lens, max_pages, qf, qs, frag,
+                                            invs, pref, nzpref, p->err);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   prof_mark(p, 3, s);
-  if (variant == OPTR_VARIANT_TENSOR) {
+  if (variant != OPTR_VARIANT_CUDA_CORE) {
     e = launch_partial_tensor(p, pool, bt, seq_lens, B, max_pages, num_pages,
-                              qf, qs, pref, nzpref, part, plan.W, s);
+                              frag, invs, qs, pref, nzpref, part, plan.W, s);
   } else {
     partial_cuda_core_kernel<<<plan.W / 4, 128, 0, s>>>(
         pool, bt, seq_lens, B, max_pages, num_pages, h_q, h_kv, qf, qs, pref,
@@ -346,8 +431,10 @@ cudaError_t launch_decode(const optr_params* p, int variant,
   }
   if (e != cudaSuccess) return e;
   prof_mark(p, 4, s);
-  combine_kernel<<<dim3(B, h_kv), 128, 0, s>>>(part, pref, nzpref, B, h_q,
-                                               h_kv, plan.W, p->R_vT, out);
+  combine_kernel<<<dim3(B, h_kv, 4), kCombineThreads,
+                   sizeof(float) * (plan.W + 1), s>>>(part, pref, nzpref, B,
+                                                      h_q, h_kv, plan.W,
+                                                      p->R_vT, out);
   prof_mark(p, 5, s);
   return cudaGetLastError();
 }

@@ -1,13 +1,364 @@
-// Tensor-core split-K partial kernel (placeholder until implemented).
+// Tensor-core split-K partial kernel of the decode attention.
+//
+// Work partition, partial format and combine are those of decode.cu: the
+// flattened (sequence, KV head, page) space is cut into W equal contiguous
+// ranges, one per warp; a warp writes one partial (m, l, o') per
+// (sequence, KV head) segment of its range.
+//
+// Per 16-token page a warp runs two tiny GEMMs on mma.sync.m16n8k16
+// (f16 inputs, f32 accumulate), N = 8 = 4 GQA query heads x {hi, lo}:
+//
+//   logits   S[tok][n] = sum_ch code[tok][ch] * q'[n][ch], one accumulator
+//            per 32-channel group, then l = sum_g scale_g * S_g
+//            + sum_g min_g * sum(q' over group g)      (Sec. 3 Eq. 1 on the
+//            dequantized rotated key, Appendix "Rotated-query implementation")
+//   values   O[ch][n] += code[ch][tok] * (p[tok] * scale_g[tok])_{hi,lo}, plus
+//            sum_tok p * min_g[tok] per group              (Sec. 3 Eq. 2)
+//
+// The 2-bit codes enter the MMA as exact fp16 subnormals: masking a code
+// field at bit 2r of a 16-bit half gives the value code * 4^r * 2^-24.  The
+// 4^r factor is undone on the other operand (query fragments are prescaled
+// by 4^-r, see qrot in decode.cu) or on the output row (values).  q' and
+// p*scale are split into fp16 hi + lo parts, which fill the 8 MMA columns
+// and keep ~22 bits of the float32 operands.
 #include "decode_common.cuh"
 
 namespace optr {
+namespace {
 
-cudaError_t launch_partial_tensor(const optr_params*, const uint8_t*,
-                                  const int32_t*, const int32_t*, int, int,
-                                  int, const float*, const float*, const int*,
-                                  const int*, float*, int, cudaStream_t) {
-  return cudaErrorNotSupported;
+constexpr int kStages = 4;            // cp.async pages in flight per warp
+constexpr int kWarps = 4;             // warps per CTA
+constexpr float kLazyTau = 8.f;       // log2-domain slack before rescaling
+
+struct WarpSmemTC {
+  alignas(16) uint8_t stage[kStages][kChunk];
+  alignas(16) uint32_t pt[kGroups][kPage][4];  // p*scale_v (hi, lo) per head
+};
+
+__device__ __forceinline__ void mma16816(float* d, uint32_t a0, uint32_t a1,
+                                         uint32_t a2, uint32_t a3, uint32_t b0,
+                                         uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 "
+      "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};\n"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+__device__ __forceinline__ void ldsm_x4_trans(uint32_t& r0, uint32_t& r1,
+                                              uint32_t& r2, uint32_t& r3,
+                                              const void* smem_row) {
+  const unsigned a = static_cast<unsigned>(__cvta_generic_to_shared(smem_row));
+  asm volatile(
+      "ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];\n"
+      : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+      : "r"(a));
+}
+
+__device__ __forceinline__ float2 h2f(uint32_t u) {
+  return __half22float2(*reinterpret_cast<const __half2*>(&u));
+}
+
+// fp16 hi / lo split of x, packed (hi in the low half).
+__device__ __forceinline__ uint32_t split_hilo(float x) {
+  const __half hi = __float2half_rn(x);
+  const __half lo = __float2half_rn(x - __half2float(hi));
+  return (uint32_t)__half_as_ushort(hi) | ((uint32_t)__half_as_ushort(lo) << 16);
+}
+
+// Iterator over a warp's flat page range: yields (b, h, page) and marks the
+// first page of each (sequence, KV head) segment.
+struct PageIter {
+  long long f, f1, seg_end;
+  int b, h, page;
+  __device__ void init(long long f0, long long fend, const int* pref, int B,
+                       int h_kv) {
+    f = f0;
+    f1 = fend;
+    seg_end = f0;
+    b = h = page = 0;
+    if (f < f1) seek(pref, B, h_kv);
+  }
+  __device__ void seek(const int* pref, int B, int h_kv) {
+    Segment s = locate_segment(f, f1, pref, B, h_kv);
+    b = s.b;
+    h = s.h;
+    page = s.p0;
+    seg_end = s.f_end;
+  }
+  __device__ bool valid() const { return f < f1; }
+  __device__ void next(const int* pref, int B, int h_kv) {
+    ++f;
+    ++page;
+    if (f < f1 && f == seg_end) seek(pref, B, h_kv);
+  }
+};
+
+__global__ void __launch_bounds__(kWarps * 32, 4)
+partial_tensor_kernel(const uint8_t* __restrict__ pool,
+                      const int32_t* __restrict__ bt,
+                      const int32_t* __restrict__ seq_lens, int B,
+                      int max_pages, int num_pages, int h_q, int h_kv,
+                      const uint32_t* __restrict__ frag,
+                      const float* __restrict__ invs,
+                      const float* __restrict__ qs,
+                      const int* __restrict__ pref,
+                      const int* __restrict__ nzpref,
+                      float* __restrict__ part, int W, unsigned* err) {
+  __shared__ WarpSmemTC smem[kWarps];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int g = lane >> 2, c = lane & 3;
+  WarpSmemTC& S = smem[warp];
+  const int w = blockIdx.x * kWarps + warp;
+  const long long F = (long long)__ldg(pref + B) * h_kv;
+  const long long f0 = w * F / W, f1 = (w + 1) * F / W;
+  if (f0 >= f1) return;
+
+  // issue iterator runs kStages-1 pages ahead of the compute iterator
+  PageIter is, cs;
+  is.init(f0, f1, pref, B, h_kv);
+  cs = is;
+  unsigned okmask = 0;  // bit s: stage s holds a page that was read
+#pragma unroll
+  for (int s = 0; s < kStages - 1; ++s) {
+    if (is.valid()) {
+      if (issue_page(S.stage[s], pool, bt + (size_t)is.b * max_pages,
+                     is.page, num_pages, h_kv, is.h, lane, err))
+        okmask |= 1u << s;
+      is.next(pref, B, h_kv);
+    } else {
+      cp_async_commit();
+    }
+  }
+
+  // per-segment state
+  uint32_t bq[kGroups][2][2];  // query B fragments [group][kk][reg]
+  float qsum[kGroups];         // sum of q' over each group, head c
+  float inv_s = 0.f;           // 2^24 / prescale of head c
+  float acc_o[kGroups][2][4];  // values: [group][half][c-frag]
+  float mv[kGroups];           // sum_tok p * min_v per group (this lane)
+  float m_run = -INFINITY, l_lane = 0.f;
+  int cur_b = -1, cur_h = -1, len = 0;
+
+  auto flush = [&]() {
+    // reduce l and the min-terms over the 8 lanes of head c, then write
+    float l = l_lane;
+#pragma unroll
+    for (int o = 4; o < 32; o <<= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
+#pragma unroll
+    for (int G = 0; G < kGroups; ++G)
+#pragma unroll
+      for (int o = 4; o < 32; o <<= 1)
+        mv[G] += __shfl_xor_sync(0xffffffffu, mv[G], o);
+    float* slot = part + (size_t)(w + __ldg(nzpref + cur_b) * h_kv + cur_h) * kPartFloats;
+    float* dst = slot + c * kD;
+#pragma unroll
+    for (int G = 0; G < kGroups; ++G) {
+      // rows g (r = 2*half) and g+8 (r = 2*half+1) of tile (G, half) are
+      // channels 32G + 4g + r; their codes carried 4^r * 2^-24
+      float4 o4;
+      o4.x = (acc_o[G][0][0] + acc_o[G][0][1]) * 16777216.f + mv[G];
+      o4.y = (acc_o[G][0][2] + acc_o[G][0][3]) * 4194304.f + mv[G];
+      o4.z = (acc_o[G][1][0] + acc_o[G][1][1]) * 1048576.f + mv[G];
+      o4.w = (acc_o[G][1][2] + acc_o[G][1][3]) * 262144.f + mv[G];
+      *reinterpret_cast<float4*>(dst + 32 * G + 4 * g) = o4;
+    }
+    if (g == 0) {
+      slot[kPartM + c] = m_run;
+      slot[kPartL + c] = l;
+    }
+  };
+
+  for (int i = 0; cs.valid(); ++i) {
+    // keep kStages-1 pages in flight
+    const int slot_issue = (i + kStages - 1) % kStages;
+    okmask &= ~(1u << slot_issue);
+    if (is.valid()) {
+      if (issue_page(S.stage[slot_issue], pool, bt + (size_t)is.b * max_pages,
+                     is.page, num_pages, h_kv, is.h, lane, err))
+        okmask |= 1u << slot_issue;
+      is.next(pref, B, h_kv);
+    } else {
+      cp_async_commit();
+    }
+    cp_async_wait<kStages - 1>();
+    __syncwarp();
+
+    if (cs.b != cur_b || cs.h != cur_h) {
+      if (cur_b >= 0) flush();
+      cur_b = cs.b;
+      cur_h = cs.h;
+      len = __ldg(seq_lens + cur_b);
+      const uint4* fq = reinterpret_cast<const uint4*>(
+          frag + (((size_t)cur_b * h_kv + cur_h) * 32 + lane) * 16);
+#pragma unroll
+      for (int G = 0; G < kGroups; ++G) {
+        const uint4 v = __ldg(fq + G);
+        bq[G][0][0] = v.x;
+        bq[G][0][1] = v.y;
+        bq[G][1][0] = v.z;
+        bq[G][1][1] = v.w;
+      }
+      const size_t row = (size_t)cur_b * h_q + 4 * cur_h + c;
+      const float4 q4 = __ldg(reinterpret_cast<const float4*>(qs + row * kGroups));
+      qsum[0] = q4.x;
+      qsum[1] = q4.y;
+      qsum[2] = q4.z;
+      qsum[3] = q4.w;
+      inv_s = __ldg(invs + row);
+#pragma unroll
+      for (int G = 0; G < kGroups; ++G) {
+        mv[G] = 0.f;
+#pragma unroll
+        for (int hf = 0; hf < 2; ++hf)
+#pragma unroll
+          for (int k = 0; k < 4; ++k) acc_o[G][hf][k] = 0.f;
+      }
+      m_run = -INFINITY;
+      l_lane = 0.f;
+    }
+
+    const uint8_t* st = S.stage[i % kStages];
+    const bool ok = (okmask >> (i % kStages)) & 1u;
+    const int nvalid = ok ? min(kPage, len - cs.page * kPage) : 0;
+
+    // ---------------------------------------------------------- logits
+    float sc[2];
+    {
+      const uint2 k0 = *reinterpret_cast<const uint2*>(st + OPTR_K_CODES_OFFSET + g * 32 + 8 * c);
+      const uint2 k1 = *reinterpret_cast<const uint2*>(st + OPTR_K_CODES_OFFSET + (g + 8) * 32 + 8 * c);
+      // bytes [G0 w2c, G1 w2c, G0 w2c+1, G1 w2c+1] and the same for G2/G3
+      const uint32_t y01_0 = __byte_perm(k0.x, k0.y, 0x5410);
+      const uint32_t y23_0 = __byte_perm(k0.x, k0.y, 0x7632);
+      const uint32_t y01_1 = __byte_perm(k1.x, k1.y, 0x5410);
+      const uint32_t y23_1 = __byte_perm(k1.x, k1.y, 0x7632);
+      float s_acc[kGroups][4];
+#pragma unroll
+      for (int G = 0; G < kGroups; ++G) {
+        const uint32_t src0 = (G < 2 ? y01_0 : y23_0) >> (8 * (G & 1));
+        const uint32_t src1 = (G < 2 ? y01_1 : y23_1) >> (8 * (G & 1));
+#pragma unroll
+        for (int k = 0; k < 4; ++k) s_acc[G][k] = 0.f;
+#pragma unroll
+        for (int kk = 0; kk < 2; ++kk) {
+          const uint32_t m0 = 0x00030003u << (2 * (2 * kk));
+          const uint32_t m1 = 0x00030003u << (2 * (2 * kk + 1));
+          mma16816(s_acc[G], src0 & m0, src1 & m0, src0 & m1, src1 & m1,
+                   bq[G][kk][0], bq[G][kk][1]);
+        }
+      }
+      const uint4 km0 = *reinterpret_cast<const uint4*>(st + OPTR_K_META_OFFSET + g * 16);
+      const uint4 km1 = *reinterpret_cast<const uint4*>(st + OPTR_K_META_OFFSET + (g + 8) * 16);
+      const uint32_t kmv0[4] = {km0.x, km0.y, km0.z, km0.w};
+      const uint32_t kmv1[4] = {km1.x, km1.y, km1.z, km1.w};
+      float t0 = 0.f, t1 = 0.f, u0 = 0.f, u1 = 0.f;
+#pragma unroll
+      for (int G = 0; G < kGroups; ++G) {
+        const float2 a = h2f(kmv0[G]);  // (scale, min) of token g
+        const float2 bb = h2f(kmv1[G]); // token g+8
+        t0 = fmaf(a.x, s_acc[G][0] + s_acc[G][1], t0);
+        t1 = fmaf(bb.x, s_acc[G][2] + s_acc[G][3], t1);
+        u0 = fmaf(a.y, qsum[G], u0);
+        u1 = fmaf(bb.y, qsum[G], u1);
+      }
+      sc[0] = g < nvalid ? fmaf(inv_s, t0, u0) : -INFINITY;
+      sc[1] = g + 8 < nvalid ? fmaf(inv_s, t1, u1) : -INFINITY;
+    }
+
+    // ------------------------------------------------ online softmax
+    float tmax = fmaxf(sc[0], sc[1]);
+#pragma unroll
+    for (int o = 4; o < 32; o <<= 1) tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, o));
+    const bool need = tmax > m_run + kLazyTau;
+    if (__any_sync(0xffffffffu, need)) {
+      const float m_new = need ? tmax : m_run;
+      const float alpha = (m_run == -INFINITY) ? 0.f : exp2f(m_run - m_new);
+      if (need) {
+        l_lane *= alpha;
+#pragma unroll
+        for (int G = 0; G < kGroups; ++G) {
+          mv[G] *= alpha;
+#pragma unroll
+          for (int hf = 0; hf < 2; ++hf)
+#pragma unroll
+            for (int k = 0; k < 4; ++k) acc_o[G][hf][k] *= alpha;
+        }
+        m_run = m_new;
+      }
+    }
+    const float p0 = sc[0] == -INFINITY ? 0.f : exp2f(sc[0] - m_run);
+    const float p1 = sc[1] == -INFINITY ? 0.f : exp2f(sc[1] - m_run);
+    l_lane += p0 + p1;
+
+    // ----------------------------------------------------------- values
+    {
+      const uint4 vm0 = *reinterpret_cast<const uint4*>(st + OPTR_V_META_OFFSET + g * 16);
+      const uint4 vm1 = *reinterpret_cast<const uint4*>(st + OPTR_V_META_OFFSET + (g + 8) * 16);
+      const uint32_t vmv0[4] = {vm0.x, vm0.y, vm0.z, vm0.w};
+      const uint32_t vmv1[4] = {vm1.x, vm1.y, vm1.z, vm1.w};
+#pragma unroll
+      for (int G = 0; G < kGroups; ++G) {
+        const float2 a = h2f(vmv0[G]);
+        const float2 bb = h2f(vmv1[G]);
+        // masked tokens: p = 0, and their (possibly garbage) metadata is
+        // never multiplied in
+        const float pt0 = g < nvalid ? p0 * a.x : 0.f;
+        const float pt1 = g + 8 < nvalid ? p1 * bb.x : 0.f;
+        if (g < nvalid) mv[G] = fmaf(p0, a.y, mv[G]);
+        if (g + 8 < nvalid) mv[G] = fmaf(p1, bb.y, mv[G]);
+        S.pt[G][g][c] = split_hilo(pt0);
+        S.pt[G][g + 8][c] = split_hilo(pt1);
+      }
+    }
+    __syncwarp();
+    uint32_t bv[kGroups][2];
+    {
+      // lanes 0-7 address rows 0-7 of group G, 8-15 rows 8-15, 16-31 the
+      // same for group G+1
+      const int r = lane & 15, gsel = lane >> 4;
+      ldsm_x4_trans(bv[0][0], bv[0][1], bv[1][0], bv[1][1], &S.pt[gsel][r][0]);
+      ldsm_x4_trans(bv[2][0], bv[2][1], bv[3][0], bv[3][1], &S.pt[2 + gsel][r][0]);
+    }
+    {
+      const uint8_t* vc = st + OPTR_V_CODES_OFFSET + 4 * g;
+      const uint32_t x0 = *reinterpret_cast<const uint32_t*>(vc + (2 * c) * 32);
+      const uint32_t x1 = *reinterpret_cast<const uint32_t*>(vc + (2 * c + 1) * 32);
+      const uint32_t x2 = *reinterpret_cast<const uint32_t*>(vc + (2 * c + 8) * 32);
+      const uint32_t x3 = *reinterpret_cast<const uint32_t*>(vc + (2 * c + 9) * 32);
+      const uint32_t a01 = __byte_perm(x0, x1, 0x5410), a23 = __byte_perm(x0, x1, 0x7632);
+      const uint32_t b01 = __byte_perm(x2, x3, 0x5410), b23 = __byte_perm(x2, x3, 0x7632);
+#pragma unroll
+      for (int G = 0; G < kGroups; ++G) {
+        const uint32_t sa = (G < 2 ? a01 : a23) >> (8 * (G & 1));
+        const uint32_t sb = (G < 2 ? b01 : b23) >> (8 * (G & 1));
+#pragma unroll
+        for (int hf = 0; hf < 2; ++hf) {
+          const uint32_t mlo = 0x00030003u << (2 * (2 * hf));
+          const uint32_t mhi = 0x00030003u << (2 * (2 * hf + 1));
+          mma16816(acc_o[G][hf], sa & mlo, sa & mhi, sb & mlo, sb & mhi,
+                   bv[G][0], bv[G][1]);
+        }
+      }
+    }
+    __syncwarp();
+    cs.next(pref, B, h_kv);
+  }
+  flush();
+}
+
+}  // namespace
+
+cudaError_t launch_partial_tensor(const optr_params* p, const uint8_t* pool,
+                                  const int32_t* bt, const int32_t* seq_lens,
+                                  int B, int max_pages, int num_pages,
+                                  const uint32_t* frag, const float* invs,
+                                  const float* qs, const int* pref,
+                                  const int* nzpref, float* part, int W,
+                                  cudaStream_t s) {
+  partial_tensor_kernel<<<W / kWarps, kWarps * 32, 0, s>>>(
+      pool, bt, seq_lens, B, max_pages, num_pages, p->cfg.h_q, p->cfg.h_kv,
+      frag, invs, qs, pref, nzpref, part, W, p->err);
+  return cudaGetLastError();
 }
 
 }  // namespace optr

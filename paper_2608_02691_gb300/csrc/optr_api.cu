@@ -31,8 +31,10 @@ namespace optr {
 // Workspace of one decode call (all offsets 256-byte aligned):
 //   qf   float [B][h_q][128]   rotated, pre-scaled queries
 //   qs   float [B][h_q][4]     per-group sums of qf
+//   frag u32   [B][h_kv][32][16] tensor-core B fragments of qf (hi/lo f16)
+//   invs float [B][h_q]         2^24 / (power-of-two prescale of frag)
 //   pref int   [2][B+1]        page prefix sums / non-empty prefix counts
-//   part float [W + B*h_kv][4][130] split-K partials
+//   part float [W + B*h_kv][520] split-K partials (o'[4][128], m[4], l[4])
 DecodePlan decode_plan(const optr_params* p, int B, int max_pages) {
   DecodePlan d;
   d.B = B;
@@ -45,6 +47,10 @@ DecodePlan decode_plan(const optr_params* p, int B, int max_pages) {
   o = round_up(o + sizeof(float) * (size_t)B * d.h_q * kD, 256);
   d.off_qs = o;
   o = round_up(o + sizeof(float) * (size_t)B * d.h_q * kGroups, 256);
+  d.off_frag = o;
+  o = round_up(o + sizeof(uint32_t) * (size_t)B * d.h_kv * 32 * 16, 256);
+  d.off_invs = o;
+  o = round_up(o + sizeof(float) * (size_t)B * d.h_q, 256);
   d.off_pref = o;
   o = round_up(o + sizeof(int) * 2 * (size_t)(B + 1), 256);
   d.off_part = o;

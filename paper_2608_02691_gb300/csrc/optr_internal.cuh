@@ -55,13 +55,16 @@ namespace optr {
 // Byte offsets of the decode workspace for a batch shape.
 struct DecodePlan {
   int B, h_q, h_kv, max_pages, W;  // W = partial-kernel warps
-  size_t off_qf, off_qs, off_pref, off_part, total;
+  size_t off_qf, off_qs, off_frag, off_invs, off_pref, off_part, total;
 };
 DecodePlan decode_plan(const optr_params* p, int B, int max_pages);
 
-// One split-K partial: per query head of the GQA group, running max m
-// (log2 domain), sum l, and the unnormalised rotated output o'[128].
-constexpr int kPartFloats = 4 * (kD + 2);
+// One split-K partial (float32): the unnormalised rotated output o'[4][128]
+// of the 4 query heads of a GQA group, then their running maxima m[4]
+// (log2 domain) and sums l[4].
+constexpr int kPartFloats = 4 * kD + 8;
+constexpr int kPartM = 4 * kD;
+constexpr int kPartL = 4 * kD + 4;
 
 // Launchers (return cudaGetLastError()).
 cudaError_t launch_append_cuda_core(const optr_params* p, const __nv_bfloat16* k,

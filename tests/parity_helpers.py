@@ -55,8 +55,12 @@ def slot_codes(pool, pages, slots, kind):
 
 
 def compare_append(pool_gpu, pool_ref, u, pages, slots):
-    """Returns a dict of counts; raises AssertionError on a violation."""
-    stats = {"codes": 0, "tie_band": 0, "mismatch_in_band": 0}
+    """Returns a dict of counts (and the boolean [n_tok][h_kv] mask of
+    token-heads whose stored record differs within tolerance -- an in-band
+    code or a scale/min ulp -- under key "flipped");
+    raises AssertionError on a violation."""
+    stats = {"codes": 0, "tie_band": 0, "mismatch_in_band": 0,
+             "flipped": np.zeros(u.shape[:2], bool)}
     for kind in (0, 1):
         cg, sg, mg = slot_codes(pool_gpu, pages, slots, kind)
         cr, sr, mr = slot_codes(pool_ref, pages, slots, kind)
@@ -67,6 +71,9 @@ def compare_append(pool_gpu, pool_ref, u, pages, slots):
         stats["codes"] += cg.size
         stats["tie_band"] += int(band.sum())
         stats["mismatch_in_band"] += int(((cg != cr) & band).sum())
+        stats["flipped"] |= ((cg != cr) & band).any(axis=2)
+        # an in-tolerance fp16 ulp of scale or min also changes the output
+        stats["flipped"] |= ((sg != sr) | (mg != mr)).any(axis=2)
         if bad.any():
             i = np.argwhere(bad)[0]
             raise AssertionError(
@@ -114,6 +121,37 @@ def gpu_case(case, variant=optr.OPTR_VARIANT_DEFAULT, append_variant=0,
                                case["seq_lens"].to(dev), pool, out, ws)
     torch.cuda.synchronize()
     return p, pool, out
+
+
+def gpu_decode(case, pool_np, variant=optr.OPTR_VARIANT_DEFAULT,
+               seq_lens=None, dev="cuda"):
+    """GPU decode over a given (oracle-written) host pool."""
+    p = optr.optr_params_create(case["R_k"], case["R_v"], case["mu"],
+                                case["h_q"], decode_variant=variant)
+    pool = torch.from_numpy(pool_np).to(dev)
+    bt = case["block_table"].to(dev)
+    lens = case["seq_lens"] if seq_lens is None else seq_lens
+    out = torch.full((case["B"], case["h_q"], 128), 7.0, dtype=torch.float32,
+                     device=dev)
+    ws = optr.new_workspace(p, case["B"], bt.shape[1], device=dev)
+    optr.optr_decode_attention(p, case["q"].to(dev), bt, lens.to(dev), pool,
+                               out, ws)
+    torch.cuda.synchronize()
+    assert optr.optr_device_error(p) == 0
+    return out.cpu().double().numpy()
+
+
+def flipped_groups(case, stats_ctx, stats_new):
+    """(b, h) groups whose cached codes differ in the tie band somewhere."""
+    out = set()
+    for st, cu in ((stats_ctx, case["cu_ctx"]), (stats_new, case["cu_new"])):
+        if st is None:
+            continue
+        cu = np.asarray(cu)
+        for t, h in np.argwhere(st["flipped"]):
+            b = int(np.searchsorted(cu, t, side="right") - 1)
+            out.add((b, int(h)))
+    return out
 
 
 def oracle_case(case, pool_init=None):

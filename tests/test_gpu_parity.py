@@ -13,7 +13,7 @@ import parity_helpers as ph
 
 pytestmark = pytest.mark.gpu
 
-VARIANTS = [optr.OPTR_VARIANT_CUDA_CORE]
+VARIANTS = [optr.OPTR_VARIANT_CUDA_CORE, optr.OPTR_VARIANT_TENSOR]
 APPEND_VARIANTS = [optr.OPTR_VARIANT_CUDA_CORE]
 CASES = [("tiny", 1.0), ("decode8k", 1 / 16), ("long128k", 1 / 32),
          ("prefill", 1 / 128), ("ragged", 1 / 32)]
@@ -42,36 +42,68 @@ def _case(name, scale, seed=0):
     return _cache[key]
 
 
+_gpu_stats = {}
+
+
 @pytest.mark.parametrize("name,scale", CASES)
 @pytest.mark.parametrize("avar", APPEND_VARIANTS)
 def test_append_matches_oracle(name, scale, avar):
+    """Codes bit-exact outside the tie band, scale/min within tolerance."""
     c, pool_ref, u_ctx, u_new = _case(name, scale)
     p, pool, _ = ph.gpu_case(c, append_variant=avar)
     assert optr.optr_device_error(p) == 0
     pg = pool.cpu().numpy()
+    sts = []
     for k, cu, pos0, u in (("ctx", c["cu_ctx"], c["pos0_ctx"], u_ctx),
                            ("new", c["cu_new"], c["pos0_new"], u_new)):
         if u is None:
+            sts.append(None)
             continue
         pages, slots = ph.token_slots(cu, pos0, c["block_table"])
         st = ph.compare_append(pg, pool_ref, u, pages, slots)
-        print(f"{name} {k}: {st}")
+        sts.append(st)
+        print(f"{name} {k}: codes {st['codes']} tie_band {st['tie_band']} "
+              f"differing_in_band {st['mismatch_in_band']}")
+    _gpu_stats[(name, scale, avar)] = sts
 
 
 @pytest.mark.parametrize("name,scale", CASES)
 @pytest.mark.parametrize("variant", VARIANTS)
 def test_decode_matches_oracle(name, scale, variant):
+    """Decode error alone: the GPU decodes the oracle-written cache."""
     c, pool_ref, _, _ = _case(name, scale)
+    got = ph.gpu_decode(c, pool_ref, variant=variant)
+    ref = ph.oracle_decode(c, pool_ref)
+    r = ph.assert_decode_close(got, ref, f"{name} decode")
+    print(f"{name} variant {variant}: err/rms {r:.2e}")
+
+
+@pytest.mark.parametrize("name,scale", CASES)
+@pytest.mark.parametrize("variant", VARIANTS)
+def test_end_to_end_matches_oracle(name, scale, variant):
+    """GPU append + GPU decode against oracle append + oracle decode, on every
+    (sequence, KV head) whose cached codes agree bit for bit; groups with an
+    in-band rounding difference (both roundings are valid) are counted."""
+    c, pool_ref, u_ctx, u_new = _case(name, scale)
     p, pool, out = ph.gpu_case(c, variant=variant)
-    assert optr.optr_device_error(p) == 0
+    pg = pool.cpu().numpy()
+    sts = []
+    for cu, pos0, u in ((c["cu_ctx"], c["pos0_ctx"], u_ctx),
+                        (c["cu_new"], c["pos0_new"], u_new)):
+        if u is None:
+            sts.append(None)
+            continue
+        pages, slots = ph.token_slots(cu, pos0, c["block_table"])
+        sts.append(ph.compare_append(pg, pool_ref, u, pages, slots))
+    skip = ph.flipped_groups(c, *sts)
     got = out.cpu().double().numpy()
-    # decode error alone: oracle decode over the GPU-written cache
-    ref = ph.oracle_decode(c, pool.cpu().numpy())
-    r1 = ph.assert_decode_close(got, ref, f"{name} decode")
-    # end to end: oracle append + oracle decode
-    ref2 = ph.oracle_decode(c, pool_ref)
-    r2 = ph.assert_decode_close(got, ref2, f"{name} end-to-end")
-    print(f"{name} variant {variant}: err/rms decode {r1:.2e} e2e {r2:.2e}")
+    ref = ph.oracle_decode(c, pool_ref)
+    keep = np.ones(got.shape[:2], bool)
+    for b, h in skip:
+        keep[b, 4 * h:4 * h + 4] = False
+    ph.assert_decode_close(got[keep], ref[keep], f"{name} end-to-end")
+    print(f"{name}: end-to-end over {int(keep.sum())} rows, "
+          f"{len(skip)} groups with in-band code differences skipped")
 
 
 @pytest.mark.parametrize("variant", VARIANTS)
@@ -79,45 +111,45 @@ def test_unused_slots_never_read(variant):
     """Slots past seq_len hold NaN metadata (pool pre-filled with 0xFF): the
     output stays finite and equal to the oracle's."""
     c, _, _, _ = _case("ragged", 1 / 32)
-    p, pool, out = ph.gpu_case(c, variant=variant, poison=True)
-    got = out.cpu().double().numpy()
-    ref = ph.oracle_decode(c, pool.cpu().numpy())
+    poisoned = np.full((c["num_pages"], c["h_kv"], 1536), 0xFF, np.uint8)
+    pool_ref, _, _ = ph.oracle_case(c, pool_init=poisoned)
+    got = ph.gpu_decode(c, pool_ref, variant=variant)
+    ref = ph.oracle_decode(c, pool_ref)
     ph.assert_decode_close(got, ref, "poisoned")
 
 
 @pytest.mark.parametrize("variant", VARIANTS)
 def test_sequence_length_edges(variant):
-    """seq_len 0 (zeros), 1, 15, 16, 17, 31, 33 over one prefilled cache."""
-    c, _, _, _ = _case("decode8k", 1 / 16)
-    p, pool, _ = ph.gpu_case(c, variant=variant)
+    """seq_len 0 (zeros), 1, 15, 16, 17, 31, 33, ... over one cache."""
+    c, pool_ref, _, _ = _case("decode8k", 1 / 16)
     lens = torch.tensor([0, 1, 15, 16, 17, 31, 33, 2, 3, 100, 257, 511, 512,
                          513, 64, 48], dtype=torch.int32)
-    dev = "cuda"
-    out = torch.full((c["B"], c["h_q"], 128), 7.0, device=dev)
-    ws = optr.new_workspace(p, c["B"], c["block_table"].shape[1])
-    optr.optr_decode_attention(p, c["q"].to(dev), c["block_table"].to(dev),
-                               lens.to(dev), pool, out, ws)
-    got = out.cpu().double().numpy()
+    got = ph.gpu_decode(c, pool_ref, variant=variant, seq_lens=lens)
     assert not got[0].any()
-    ref = ph.oracle_decode(c, pool.cpu().numpy(), seq_lens=lens)
+    ref = ph.oracle_decode(c, pool_ref, seq_lens=lens)
     ph.assert_decode_close(got, ref, "length edges")
-    assert optr.optr_device_error(p) == 0
 
 
 @pytest.mark.parametrize("variant", VARIANTS)
 def test_split_invariance(variant):
     """The split-K cut points of a sequence depend on the whole batch; the
     result for one sequence must not (alone vs inside the batch)."""
-    c, _, _, _ = _case("ragged", 1 / 32)
-    p, pool, out = ph.gpu_case(c, variant=variant)
+    c, pool_ref, _, _ = _case("ragged", 1 / 32)
     dev = "cuda"
+    p = optr.optr_params_create(c["R_k"], c["R_v"], c["mu"], c["h_q"],
+                                decode_variant=variant)
+    pool = torch.from_numpy(pool_ref).to(dev)
     bt = c["block_table"]
+    out = torch.empty(c["B"], c["h_q"], 128, device=dev)
+    ws = optr.new_workspace(p, c["B"], bt.shape[1])
+    optr.optr_decode_attention(p, c["q"].to(dev), bt.to(dev),
+                               c["seq_lens"].to(dev), pool, out, ws)
     for b in (0, 7, 127):
         o1 = torch.empty(1, c["h_q"], 128, device=dev)
-        ws = optr.new_workspace(p, 1, bt.shape[1])
+        ws1 = optr.new_workspace(p, 1, bt.shape[1])
         optr.optr_decode_attention(p, c["q"][b:b + 1].to(dev),
                                    bt[b:b + 1].contiguous().to(dev),
-                                   c["seq_lens"][b:b + 1].to(dev), pool, o1, ws)
+                                   c["seq_lens"][b:b + 1].to(dev), pool, o1, ws1)
         torch.cuda.synchronize()
         a, bb = o1[0].double().cpu(), out[b].double().cpu()
         rms = float(a.pow(2).mean().sqrt())
@@ -127,18 +159,15 @@ def test_split_invariance(variant):
 def test_needle_is_retrieved():
     """long-context workload: the planted key wins the softmax of its
     group's first query head, and the GPU output matches the oracle."""
-    c, _, _, _ = _case("long128k", 1 / 16)
-    p, pool, out = ph.gpu_case(c)
-    pn = pool.cpu().numpy()
+    c, pool_ref, _, _ = _case("long128k", 1 / 16)
     for h, pos in enumerate(c["needle"].tolist()):
-        j = 4 * h
         _, prob = oracle.decode_attention(
             synth.bf16_bits(c["q"]), c["block_table"].numpy(),
-            c["seq_lens"].numpy(), pn, c["R_k"].numpy(), c["R_v"].numpy(),
-            c["h_kv"], rows=[(0, j)], want_p=True)
+            c["seq_lens"].numpy(), pool_ref, c["R_k"].numpy(),
+            c["R_v"].numpy(), c["h_kv"], rows=[(0, 4 * h)], want_p=True)
         assert int(np.argmax(prob)) == pos
-    ref = ph.oracle_decode(c, pn)
-    ph.assert_decode_close(out.cpu().double().numpy(), ref, "needle")
+    got = ph.gpu_decode(c, pool_ref)
+    ph.assert_decode_close(got, ph.oracle_decode(c, pool_ref), "needle")
 
 
 def test_bad_tables_are_flagged_not_read():
