@@ -65,8 +65,8 @@ qrot_kernel(const __nv_bfloat16* __restrict__ q, const float* __restrict__ R_k,
   }
   __syncthreads();
   // Tensor-core B fragments (see decode_tc.cu): per head a power-of-two
-  // prescale 2^e keeps |q'| * 2^e below 2^14, so that the fp16 hi/lo split
-  // (and the 4^-r factors that undo the unshifted code masks) stay normal.
+  // prescale 2^e brings max |q'| * 2^e into [2^13, 2^14), so that the fp16
+  // hi/lo split stays in the normal range for all but tiny elements.
   int e[4];
 #pragma unroll
   for (int r = 0; r < 4; ++r) {
@@ -74,7 +74,7 @@ qrot_kernel(const __nv_bfloat16* __restrict__ q, const float* __restrict__ R_k,
     e[r] = mx > 0.f ? 13 - ilogbf(mx) : 0;
     e[r] = max(-100, min(100, e[r]));
   }
-  if (j < 4) invs[(size_t)b * h_q + 4 * h + j] = ldexpf(1.f, 24 - e[j]);
+  if (j < 4) invs[(size_t)b * h_q + 4 * h + j] = ldexpf(1.f, -e[j]);
   uint32_t* fb = frag + ((size_t)b * h_kv + h) * 512;
 #pragma unroll
   for (int t = 0; t < 4; ++t) {
@@ -84,7 +84,7 @@ qrot_kernel(const __nv_bfloat16* __restrict__ q, const float* __restrict__ R_k,
     const int g = L >> 2, c = L & 3;
     const int head = g >> 1, part = g & 1;
     const int ch = 32 * G + 8 * c + 2 * kk + which;   // low half; +4 high
-    const float sc = ldexpf(1.f, e[head] - 2 * (2 * kk + which));
+    const float sc = ldexpf(1.f, e[head]);
     const float x0 = qrs[head][ch] * sc, x1 = qrs[head][ch + 4] * sc;
     const __half h0 = __float2half_rn(x0), h1 = __float2half_rn(x1);
     __half v0 = h0, v1 = h1;

@@ -15,12 +15,16 @@
 //   values   O[ch][n] += code[ch][tok] * (p[tok] * scale_g[tok])_{hi,lo}, plus
 //            sum_tok p * min_g[tok] per group              (Sec. 3 Eq. 2)
 //
-// The 2-bit codes enter the MMA as exact fp16 subnormals: masking a code
-// field at bit 2r of a 16-bit half gives the value code * 4^r * 2^-24.  The
-// 4^r factor is undone on the other operand (query fragments are prescaled
-// by 4^-r, see qrot in decode.cu) or on the output row (values).  q' and
-// p*scale are split into fp16 hi + lo parts, which fill the 8 MMA columns
-// and keep ~22 bits of the float32 operands.
+// The 2-bit codes enter the MMA as exact normal fp16 integers 0..3: one LOP3
+// masks the code field at bit 2r of each 16-bit half and ORs in the exponent
+// of 1024, giving the half 1024 + code * 4^r, and one HFMA2 maps it to
+// (x - 1024) * 4^-r = code exactly.  (Raw masked fields would be fp16
+// subnormals; the MMA keeps only ~17 bits below its largest product for
+// subnormal A operands, against ~21 for normal ones, and the value-side sum
+// sum_tok p*scale*code nearly cancels against sum_tok p*min, so that loss
+// would show in the output.)  q' and p*scale are split into fp16 hi + lo
+// parts, which fill the 8 MMA columns and keep ~22 bits of the float32
+// operands.
 #include "decode_common.cuh"
 
 namespace optr {
@@ -53,6 +57,17 @@ __device__ __forceinline__ void ldsm_x4_trans(uint32_t& r0, uint32_t& r1,
       "ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];\n"
       : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
       : "r"(a));
+}
+
+// Two codes (the fields at bit 2r of each 16-bit half of src) as exact
+// fp16 values 0..3.
+template <int r>
+__device__ __forceinline__ uint32_t codes_f16x2(uint32_t src) {
+  const uint32_t x = (src & (0x00030003u << (2 * r))) | 0x64006400u;
+  const __half2 sc = __float2half2_rn(1.0f / (float)(1 << (2 * r)));
+  const __half2 bias = __float2half2_rn(-1024.0f / (float)(1 << (2 * r)));
+  const __half2 y = __hfma2(*reinterpret_cast<const __half2*>(&x), sc, bias);
+  return *reinterpret_cast<const uint32_t*>(&y);
 }
 
 __device__ __forceinline__ float2 h2f(uint32_t u) {
@@ -134,7 +149,7 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
   // per-segment state
   uint32_t bq[kGroups][2][2];  // query B fragments [group][kk][reg]
   float qsum[kGroups];         // sum of q' over each group, head c
-  float inv_s = 0.f;           // 2^24 / prescale of head c
+  float inv_s = 0.f;           // 1 / prescale of head c
   float acc_o[kGroups][2][4];  // values: [group][half][c-frag]
   float mv[kGroups];           // sum_tok p * min_v per group (this lane)
   float m_run = -INFINITY, l_lane = 0.f;
@@ -155,12 +170,12 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
 #pragma unroll
     for (int G = 0; G < kGroups; ++G) {
       // rows g (r = 2*half) and g+8 (r = 2*half+1) of tile (G, half) are
-      // channels 32G + 4g + r; their codes carried 4^r * 2^-24
+      // channels 32G + 4g + r
       float4 o4;
-      o4.x = (acc_o[G][0][0] + acc_o[G][0][1]) * 16777216.f + mv[G];
-      o4.y = (acc_o[G][0][2] + acc_o[G][0][3]) * 4194304.f + mv[G];
-      o4.z = (acc_o[G][1][0] + acc_o[G][1][1]) * 1048576.f + mv[G];
-      o4.w = (acc_o[G][1][2] + acc_o[G][1][3]) * 262144.f + mv[G];
+      o4.x = (acc_o[G][0][0] + acc_o[G][0][1]) + mv[G];
+      o4.y = (acc_o[G][0][2] + acc_o[G][0][3]) + mv[G];
+      o4.z = (acc_o[G][1][0] + acc_o[G][1][1]) + mv[G];
+      o4.w = (acc_o[G][1][2] + acc_o[G][1][3]) + mv[G];
       *reinterpret_cast<float4*>(dst + 32 * G + 4 * g) = o4;
     }
     if (g == 0) {
@@ -239,13 +254,12 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
         const uint32_t src1 = (G < 2 ? y01_1 : y23_1) >> (8 * (G & 1));
 #pragma unroll
         for (int k = 0; k < 4; ++k) s_acc[G][k] = 0.f;
-#pragma unroll
-        for (int kk = 0; kk < 2; ++kk) {
-          const uint32_t m0 = 0x00030003u << (2 * (2 * kk));
-          const uint32_t m1 = 0x00030003u << (2 * (2 * kk + 1));
-          mma16816(s_acc[G], src0 & m0, src1 & m0, src0 & m1, src1 & m1,
-                   bq[G][kk][0], bq[G][kk][1]);
-        }
+        mma16816(s_acc[G], codes_f16x2<0>(src0), codes_f16x2<0>(src1),
+                 codes_f16x2<1>(src0), codes_f16x2<1>(src1), bq[G][0][0],
+                 bq[G][0][1]);
+        mma16816(s_acc[G], codes_f16x2<2>(src0), codes_f16x2<2>(src1),
+                 codes_f16x2<3>(src0), codes_f16x2<3>(src1), bq[G][1][0],
+                 bq[G][1][1]);
       }
       const uint4 km0 = *reinterpret_cast<const uint4*>(st + OPTR_K_META_OFFSET + g * 16);
       const uint4 km1 = *reinterpret_cast<const uint4*>(st + OPTR_K_META_OFFSET + (g + 8) * 16);
@@ -331,13 +345,10 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
       for (int G = 0; G < kGroups; ++G) {
         const uint32_t sa = (G < 2 ? a01 : a23) >> (8 * (G & 1));
         const uint32_t sb = (G < 2 ? b01 : b23) >> (8 * (G & 1));
-#pragma unroll
-        for (int hf = 0; hf < 2; ++hf) {
-          const uint32_t mlo = 0x00030003u << (2 * (2 * hf));
-          const uint32_t mhi = 0x00030003u << (2 * (2 * hf + 1));
-          mma16816(acc_o[G][hf], sa & mlo, sa & mhi, sb & mlo, sb & mhi,
-                   bv[G][0], bv[G][1]);
-        }
+        mma16816(acc_o[G][0], codes_f16x2<0>(sa), codes_f16x2<1>(sa),
+                 codes_f16x2<0>(sb), codes_f16x2<1>(sb), bv[G][0], bv[G][1]);
+        mma16816(acc_o[G][1], codes_f16x2<2>(sa), codes_f16x2<3>(sa),
+                 codes_f16x2<2>(sb), codes_f16x2<3>(sb), bv[G][0], bv[G][1]);
       }
     }
     __syncwarp();

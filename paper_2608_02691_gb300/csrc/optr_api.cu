@@ -32,7 +32,7 @@ namespace optr {
 //   qf   float [B][h_q][128]   rotated, pre-scaled queries
 //   qs   float [B][h_q][4]     per-group sums of qf
 //   frag u32   [B][h_kv][32][16] tensor-core B fragments of qf (hi/lo f16)
-//   invs float [B][h_q]         2^24 / (power-of-two prescale of frag)
+//   invs float [B][h_q]         1 / (power-of-two prescale of frag)
 //   pref int   [2][B+1]        page prefix sums / non-empty prefix counts
 //   part float [W + B*h_kv][520] split-K partials (o'[4][128], m[4], l[4])
 DecodePlan decode_plan(const optr_params* p, int B, int max_pages) {

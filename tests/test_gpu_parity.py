@@ -81,9 +81,11 @@ def test_decode_matches_oracle(name, scale, variant):
 @pytest.mark.parametrize("name,scale", CASES)
 @pytest.mark.parametrize("variant", VARIANTS)
 def test_end_to_end_matches_oracle(name, scale, variant):
-    """GPU append + GPU decode against oracle append + oracle decode, on every
-    (sequence, KV head) whose cached codes agree bit for bit; groups with an
-    in-band rounding difference (both roundings are valid) are counted."""
+    """GPU append + GPU decode against oracle append + oracle decode.  Rows of
+    (sequence, KV head) groups whose cached records agree bit for bit meet
+    the decode tolerance; every row meets E2E_TOL, since an in-band code or
+    an fp16 ulp of scale/min (both allowed by the append tolerance) moves
+    the output by up to about a quantization step times its weight."""
     c, pool_ref, u_ctx, u_new = _case(name, scale)
     p, pool, out = ph.gpu_case(c, variant=variant)
     pg = pool.cpu().numpy()
@@ -101,9 +103,13 @@ def test_end_to_end_matches_oracle(name, scale, variant):
     keep = np.ones(got.shape[:2], bool)
     for b, h in skip:
         keep[b, 4 * h:4 * h + 4] = False
-    ph.assert_decode_close(got[keep], ref[keep], f"{name} end-to-end")
-    print(f"{name}: end-to-end over {int(keep.sum())} rows, "
-          f"{len(skip)} groups with in-band code differences skipped")
+    if keep.any():
+        ph.assert_decode_close(got[keep], ref[keep], f"{name} end-to-end")
+    rms = float(np.sqrt(np.mean(ref ** 2)))
+    err = float(np.abs(got - ref).max())
+    assert err <= ph.E2E_TOL * rms, f"{name} end-to-end: {err / rms:.2e} of rms"
+    print(f"{name}: strict over {int(keep.sum())} rows ({len(skip)} groups "
+          f"with in-tolerance record differences); all rows err/rms {err / rms:.2e}")
 
 
 @pytest.mark.parametrize("variant", VARIANTS)
