@@ -87,6 +87,24 @@ __device__ __forceinline__ bool issue_page(uint8_t* stage,
   return ok;
 }
 
+// Same as issue_page for a physical page id already in hand.
+__device__ __forceinline__ bool issue_phys(uint8_t* stage,
+                                           const uint8_t* __restrict__ pool,
+                                           int phys, int num_pages, int h_kv,
+                                           int h, int lane, unsigned* err) {
+  const bool ok = phys >= 0 && phys < num_pages;
+  if (ok) {
+    const uint8_t* src = pool + ((size_t)phys * h_kv + h) * kChunk;
+#pragma unroll
+    for (int c = 0; c < 3; ++c)
+      cp_async16(stage + (lane + 32 * c) * 16, src + (lane + 32 * c) * 16);
+  } else if (lane == 0) {
+    atomicOr(err, OPTR_DEVERR_PAGE_ID);
+  }
+  cp_async_commit();
+  return ok;
+}
+
 // exp2(m - M) for a partial whose running max is m, 0 for an empty partial.
 __device__ __forceinline__ float merge_weight(float m, float M) {
   return m == -INFINITY ? 0.f : exp2f(m - M);

@@ -81,8 +81,8 @@ __device__ __forceinline__ uint32_t split_hilo(float x) {
   return (uint32_t)__half_as_ushort(hi) | ((uint32_t)__half_as_ushort(lo) << 16);
 }
 
-// Iterator over a warp's flat page range: yields (b, h, page) and marks the
-// first page of each (sequence, KV head) segment.
+// Iterator over a warp's flat page range: yields (b, h, page) in order,
+// seeking the next (sequence, KV head) segment at each boundary.
 struct PageIter {
   long long f, f1, seg_end;
   int b, h, page;
@@ -102,10 +102,38 @@ struct PageIter {
     seg_end = s.f_end;
   }
   __device__ bool valid() const { return f < f1; }
-  __device__ void next(const int* pref, int B, int h_kv) {
+  // true when the step entered a new segment
+  __device__ bool next(const int* pref, int B, int h_kv) {
     ++f;
     ++page;
-    if (f < f1 && f == seg_end) seek(pref, B, h_kv);
+    if (f < f1 && f == seg_end) {
+      seek(pref, B, h_kv);
+      return true;
+    }
+    return false;
+  }
+};
+
+// The issuing side also holds the block-table entries of the next 32 pages
+// of its segment, one per lane, so that a page issue needs no dependent
+// global load.
+struct IssueIter : PageIter {
+  int chunk_base;
+  int32_t btreg;
+  __device__ void load_chunk(const int32_t* __restrict__ bt, int max_pages,
+                             int lane) {
+    chunk_base = page;
+    const long long left = seg_end - f;  // pages left in this segment
+    btreg = lane < left ? __ldg(bt + (size_t)b * max_pages + page + lane) : -1;
+  }
+  __device__ int phys(const int32_t* __restrict__ bt, int max_pages, int lane) {
+    if (page - chunk_base >= 32) load_chunk(bt, max_pages, lane);
+    return __shfl_sync(0xffffffffu, btreg, page - chunk_base);
+  }
+  __device__ void advance(const int* pref, int B, int h_kv,
+                          const int32_t* __restrict__ bt, int max_pages,
+                          int lane) {
+    if (next(pref, B, h_kv)) load_chunk(bt, max_pages, lane);
   }
 };
 
@@ -130,17 +158,19 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
   if (f0 >= f1) return;
 
   // issue iterator runs kStages-1 pages ahead of the compute iterator
-  PageIter is, cs;
+  IssueIter is;
+  PageIter cs;
   is.init(f0, f1, pref, B, h_kv);
   cs = is;
+  is.load_chunk(bt, max_pages, lane);
   unsigned okmask = 0;  // bit s: stage s holds a page that was read
 #pragma unroll
   for (int s = 0; s < kStages - 1; ++s) {
     if (is.valid()) {
-      if (issue_page(S.stage[s], pool, bt + (size_t)is.b * max_pages,
-                     is.page, num_pages, h_kv, is.h, lane, err))
+      if (issue_phys(S.stage[s], pool, is.phys(bt, max_pages, lane),
+                     num_pages, h_kv, is.h, lane, err))
         okmask |= 1u << s;
-      is.next(pref, B, h_kv);
+      is.advance(pref, B, h_kv, bt, max_pages, lane);
     } else {
       cp_async_commit();
     }
@@ -189,10 +219,10 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
     const int slot_issue = (i + kStages - 1) % kStages;
     okmask &= ~(1u << slot_issue);
     if (is.valid()) {
-      if (issue_page(S.stage[slot_issue], pool, bt + (size_t)is.b * max_pages,
-                     is.page, num_pages, h_kv, is.h, lane, err))
+      if (issue_phys(S.stage[slot_issue], pool, is.phys(bt, max_pages, lane),
+                     num_pages, h_kv, is.h, lane, err))
         okmask |= 1u << slot_issue;
-      is.next(pref, B, h_kv);
+      is.advance(pref, B, h_kv, bt, max_pages, lane);
     } else {
       cp_async_commit();
     }
