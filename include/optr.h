@@ -243,6 +243,38 @@ optr_status optr_device_error(const optr_params* p, uint32_t* flags);
 optr_status optr_profile_enable(optr_params* p, int on);
 optr_status optr_profile_last(const optr_params* p, float ms[4]);
 
+/*
+ * Decode attention without a caller-supplied workspace.  The paper has no
+ * counterpart: this entry point exists for callers that cannot allocate
+ * device memory at decode time -- for example an inference-engine plugin
+ * whose host interface hands it tensors but no allocator, or a latency-
+ * critical decode loop that must never call cudaMalloc (which synchronises
+ * the device and can fail under memory pressure).
+ *
+ * Same arguments, result and errors as optr_decode_attention, minus the
+ * workspace.  The scratch memory is a fixed array of
+ * OPTR_NOALLOC_SCRATCH_BYTES (16 MiB) in the library's device image; every
+ * GPU that loads the library holds it until the process exits.  A batch
+ * whose workspace would exceed it (optr_decode_workspace_size(p, B,
+ * max_pages) > OPTR_NOALLOC_SCRATCH_BYTES; about B > 200 at 8 KV heads on a
+ * 152-SM GPU) is rejected with OPTR_ERR_WORKSPACE before any launch.
+ *
+ * The first call on each device looks up the array's device address with
+ * that device current (cudaGetSymbolAddress); make that first call before
+ * any stream capture.  Nothing in the scratch needs to start at zero.  All
+ * calls on a device share the one array, so calls that overlap on the GPU
+ * (different streams, or different threads without ordering) race and
+ * corrupt each other's results; serialise them.  This call allocates
+ * nothing and never calls cudaMalloc or cudaFree.
+ */
+#define OPTR_NOALLOC_SCRATCH_BYTES (16u << 20)
+optr_status optr_decode_attention_noalloc(const optr_params* p, const void* q,
+                                          const int32_t* block_table,
+                                          const int32_t* seq_lens, int B,
+                                          int max_pages, const uint8_t* pool,
+                                          int num_pages, float* out,
+                                          cudaStream_t stream);
+
 /* Static description of a status code. */
 const char* optr_strerror(optr_status s);
 

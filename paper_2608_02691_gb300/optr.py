@@ -54,6 +54,8 @@ _SIG = {
                                    ctypes.c_size_t, _V]),
     "optr_device_error": (_I, [_V, ctypes.POINTER(ctypes.c_uint32)]),
     "optr_strerror": (ctypes.c_char_p, [_I]),
+    "optr_decode_attention_noalloc": (_I, [_V, _V, _V, _V, _I, _I, _V, _I,
+                                           _V, _V]),
     "optr_profile_enable": (_I, [_V, _I]),
     "optr_profile_last": (_I, [_V, ctypes.POINTER(ctypes.c_float)]),
 }
@@ -191,6 +193,26 @@ def optr_decode_attention(p: Params, q, block_table, seq_lens, pool, out,
         p.handle, _ptr(q), _ptr(block_table), _ptr(seq_lens), B, max_pages,
         _ptr(pool), pool.shape[0], _ptr(out), _ptr(workspace),
         workspace.numel(), _stream(stream)), "optr_decode_attention")
+
+
+NOALLOC_SCRATCH_BYTES = 16 << 20
+
+
+def optr_decode_attention_noalloc(p: Params, q, block_table, seq_lens, pool,
+                                  out, stream=None) -> None:
+    """Decode without a workspace argument: the library uses its own fixed
+    16 MiB device scratch array, so this call allocates nothing.  Calls
+    that overlap on the GPU share that array and must be serialised."""
+    _dev(q, torch.bfloat16, "q")
+    _dev(block_table, torch.int32, "block_table")
+    _dev(seq_lens, torch.int32, "seq_lens")
+    _dev(pool, torch.uint8, "pool")
+    _dev(out, torch.float32, "out")
+    B, max_pages = block_table.shape
+    _check(lib().optr_decode_attention_noalloc(
+        p.handle, _ptr(q), _ptr(block_table), _ptr(seq_lens), B, max_pages,
+        _ptr(pool), pool.shape[0], _ptr(out), _stream(stream)),
+        "optr_decode_attention_noalloc")
 
 
 def optr_device_error(p: Params) -> int:
