@@ -22,7 +22,12 @@ constexpr float kLog2e = 1.4426950408889634f;
 
 // ---------------------------------------------------------------- qrot
 
-__global__ void __launch_bounds__(128)
+// One CTA per (sequence, KV head), 512 threads = 4 slices x 128 channels:
+// slice s sums q[i] R[i][j] over i in [32s, 32s+32) for the 4 query heads of
+// the group, the slices are added in shared memory.
+constexpr int kQrotThreads = 512;
+
+__global__ void __launch_bounds__(kQrotThreads)
 qrot_kernel(const __nv_bfloat16* __restrict__ q, const float* __restrict__ R_k,
             int B, int h_q, int h_kv, float qscale,
             const int32_t* __restrict__ seq_lens, int max_pages,
@@ -30,25 +35,33 @@ qrot_kernel(const __nv_bfloat16* __restrict__ q, const float* __restrict__ R_k,
             uint32_t* __restrict__ frag, float* __restrict__ invs,
             int* __restrict__ pref, int* __restrict__ nzpref, unsigned* err) {
   __shared__ float qsm[4][kD];
+  __shared__ float part[4][4][kD];  // [slice][head][channel]
   __shared__ float qrs[4][kD];
   __shared__ float hmax[4][4];
-  __shared__ int warp_tot[2][4];
-  const int b = blockIdx.x, h = blockIdx.y, j = threadIdx.x;
-  const int warp = j >> 5, lane = j & 31;
-#pragma unroll
-  for (int r = 0; r < 4; ++r)
+  __shared__ int warp_tot[2][kQrotThreads / 32];
+  const int b = blockIdx.x, h = blockIdx.y, tid = threadIdx.x;
+  const int sl = tid >> 7, j = tid & 127;
+  const int warp = tid >> 5, lane = tid & 31;
+  {
+    const int r = tid >> 7;  // 512 threads load the 4 x 128 query values
     qsm[r][j] = __bfloat162float(q[((size_t)b * h_q + 4 * h + r) * kD + j]);
+  }
   __syncthreads();
   float acc[4] = {0.f, 0.f, 0.f, 0.f};
-  const float* R = R_k + (size_t)h * kD * kD;
-  for (int i = 0; i < kD; ++i) {
-    const float rij = __ldg(R + i * kD + j);
+  const float* R = R_k + (size_t)h * kD * kD + (size_t)(32 * sl) * kD + j;
+#pragma unroll 16
+  for (int i = 0; i < 32; ++i) {
+    const float rij = __ldg(R + i * kD);
 #pragma unroll
-    for (int r = 0; r < 4; ++r) acc[r] = fmaf(qsm[r][i], rij, acc[r]);
+    for (int r = 0; r < 4; ++r) acc[r] = fmaf(qsm[r][32 * sl + i], rij, acc[r]);
   }
 #pragma unroll
-  for (int r = 0; r < 4; ++r) {
-    const float x = acc[r] * qscale;
+  for (int r = 0; r < 4; ++r) part[sl][r][j] = acc[r];
+  __syncthreads();
+  if (tid < 4 * kD) {
+    // thread (r, j): the 4 slices of head r, channel j
+    const int r = tid >> 7;
+    const float x = (part[0][r][j] + part[1][r][j] + part[2][r][j] + part[3][r][j]) * qscale;
     const size_t row = (size_t)b * h_q + 4 * h + r;
     qf[row * kD + j] = x;
     qrs[r][j] = x;
@@ -59,49 +72,49 @@ qrot_kernel(const __nv_bfloat16* __restrict__ q, const float* __restrict__ R_k,
       a = fmaxf(a, __shfl_xor_sync(0xffffffffu, a, o));
     }
     if (lane == 0) {
-      qs[row * kGroups + warp] = s;  // warp == group
-      hmax[r][warp] = a;
+      qs[row * kGroups + (j >> 5)] = s;
+      hmax[r][j >> 5] = a;
     }
   }
   __syncthreads();
   // Tensor-core B fragments (see decode_tc.cu): per head a power-of-two
   // prescale 2^e brings max |q'| * 2^e into [2^13, 2^14), so that the fp16
   // hi/lo split stays in the normal range for all but tiny elements.
-  int e[4];
-#pragma unroll
-  for (int r = 0; r < 4; ++r) {
-    const float mx = fmaxf(fmaxf(hmax[r][0], hmax[r][1]), fmaxf(hmax[r][2], hmax[r][3]));
-    e[r] = mx > 0.f ? 13 - ilogbf(mx) : 0;
-    e[r] = max(-100, min(100, e[r]));
-  }
-  if (j < 4) invs[(size_t)b * h_q + 4 * h + j] = ldexpf(1.f, -e[j]);
-  uint32_t* fb = frag + ((size_t)b * h_kv + h) * 512;
-#pragma unroll
-  for (int t = 0; t < 4; ++t) {
-    const int ridx = j + 128 * t;          // 512 fragment registers
+  {
+    const int ridx = tid;  // 512 fragment registers, one per thread
     const int L = ridx >> 4, reg = ridx & 15;
     const int G = reg >> 2, kk = (reg >> 1) & 1, which = reg & 1;
     const int g = L >> 2, c = L & 3;
-    const int head = g >> 1, part = g & 1;
+    const int head = g >> 1, part_hl = g & 1;
+    const float mx = fmaxf(fmaxf(hmax[head][0], hmax[head][1]),
+                           fmaxf(hmax[head][2], hmax[head][3]));
+    const int e = max(-100, min(100, mx > 0.f ? 13 - ilogbf(mx) : 0));
     const int ch = 32 * G + 8 * c + 2 * kk + which;   // low half; +4 high
-    const float sc = ldexpf(1.f, e[head]);
+    const float sc = ldexpf(1.f, e);
     const float x0 = qrs[head][ch] * sc, x1 = qrs[head][ch + 4] * sc;
     const __half h0 = __float2half_rn(x0), h1 = __float2half_rn(x1);
     __half v0 = h0, v1 = h1;
-    if (part) {
+    if (part_hl) {
       v0 = __float2half_rn(x0 - __half2float(h0));
       v1 = __float2half_rn(x1 - __half2float(h1));
     }
-    fb[L * 16 + reg] = (uint32_t)__half_as_ushort(v0) |
-                       ((uint32_t)__half_as_ushort(v1) << 16);
+    frag[((size_t)b * h_kv + h) * 512 + ridx] =
+        (uint32_t)__half_as_ushort(v0) | ((uint32_t)__half_as_ushort(v1) << 16);
+    if (ridx < 4) {
+      const float m2 = fmaxf(fmaxf(hmax[ridx][0], hmax[ridx][1]),
+                             fmaxf(hmax[ridx][2], hmax[ridx][3]));
+      const int e2 = max(-100, min(100, m2 > 0.f ? 13 - ilogbf(m2) : 0));
+      invs[(size_t)b * h_q + 4 * h + ridx] = ldexpf(1.f, -e2);
+    }
   }
 
   if (b != 0 || h != 0) return;
   // Split-K plan: pref[b] = pages of sequences < b, nzpref[b] = non-empty
   // sequences < b.  Invalid lengths count as empty and are flagged.
   int run_p = 0, run_n = 0;
-  for (int base = 0; base < B; base += 128) {
-    const int bb = base + j;
+  constexpr int kW = kQrotThreads / 32;
+  for (int base = 0; base < B; base += kQrotThreads) {
+    const int bb = base + tid;
     int np = 0;
     if (bb < B) {
       const int len = seq_lens[bb];
@@ -123,7 +136,7 @@ qrot_kernel(const __nv_bfloat16* __restrict__ q, const float* __restrict__ R_k,
     for (int w = 0; w < warp; ++w) { op += warp_tot[0][w]; on += warp_tot[1][w]; }
     if (bb < B) { pref[bb + 1] = op + xp; nzpref[bb + 1] = on + xn; }
     if (bb == 0) { pref[0] = 0; nzpref[0] = 0; }
-    for (int w = 0; w < 4; ++w) { run_p += warp_tot[0][w]; run_n += warp_tot[1][w]; }
+    for (int w = 0; w < kW; ++w) { run_p += warp_tot[0][w]; run_n += warp_tot[1][w]; }
     __syncthreads();
   }
 }
@@ -291,43 +304,29 @@ partial_cuda_core_kernel(const uint8_t* __restrict__ pool,
 
 // ------------------------------------------------------------- combine
 
-// One CTA per (sequence b, KV head h, query head r of the group); 1024
-// threads = 8 slices x 128 channels.  Merge weights exp2(m_i - M) / L of the
-// segment partials are computed once into shared memory (W + 1 floats of
-// dynamic shared memory), then every slice sums a strided subset of the
-// partials, and the merged o' is rotated back: out = o' R_v^T.
-constexpr int kCombineThreads = 1024;
-constexpr int kSlices = kCombineThreads / kD;
-
-__device__ __forceinline__ float block_reduce(float v, bool is_max, float* red) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    const float u = __shfl_xor_sync(0xffffffffu, v, o);
-    v = is_max ? fmaxf(v, u) : v + u;
-  }
-  __syncthreads();
-  if (lane == 0) red[warp] = v;
-  __syncthreads();
-  float t = red[0];
-  for (int i = 1; i < kCombineThreads / 32; ++i) t = is_max ? fmaxf(t, red[i]) : t + red[i];
-  return t;
-}
+// One CTA per (sequence b, KV head h), 256 threads, all 4 query heads of
+// the group.  The merge weights exp2(m_i - M) / L of the segment partials
+// are computed once into shared memory (dynamic, (W + 1) x 4 floats); each
+// thread then merges 2 of the 512 outputs o'[head][channel], and the merged
+// o' is rotated back, out = o' R_v^T, with the 128-term sums split over the
+// two halves of the block.
+constexpr int kCombineThreads = 256;
 
 __global__ void __launch_bounds__(kCombineThreads)
 combine_kernel(const float* __restrict__ part, const int* __restrict__ pref,
                const int* __restrict__ nzpref, int B, int h_q, int h_kv, int W,
                const float* __restrict__ R_vT, float* __restrict__ out) {
-  extern __shared__ float wts[];  // [W + 1]
-  __shared__ float red[kCombineThreads / 32];
-  __shared__ float osl[kSlices][kD];
-  __shared__ float orot[kD];
-  const int b = blockIdx.x, h = blockIdx.y, r = blockIdx.z;
-  const int tid = threadIdx.x, sl = tid / kD, j = tid % kD;
+  extern __shared__ float wts[];  // [n][4]
+  __shared__ float red[kCombineThreads / 32][4];
+  __shared__ float ML[2][4];
+  __shared__ float orot[4][kD];
+  __shared__ float half_sum[4][kD];
+  const int b = blockIdx.x, h = blockIdx.y;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int np = __ldg(pref + b + 1) - __ldg(pref + b);
-  float* ob = out + ((size_t)b * h_q + 4 * h + r) * kD;
+  float* ob = out + ((size_t)b * h_q + 4 * h) * kD;
   if (np == 0) {
-    if (tid < kD) ob[tid] = 0.f;
+    for (int i = tid; i < 4 * kD; i += kCombineThreads) ob[i] = 0.f;
     return;
   }
   const long long F = (long long)__ldg(pref + B) * h_kv;
@@ -336,54 +335,82 @@ combine_kernel(const float* __restrict__ part, const int* __restrict__ pref,
   const int n = w1 - w0 + 1;
   const float* pbase = part + ((size_t)__ldg(nzpref + b) * h_kv + h + w0) * kPartFloats;
 
+  // per-head maxima over the partials (thread t: partial t/4, head t%4)
   float mloc = -INFINITY;
-  for (int i = tid; i < n; i += kCombineThreads)
+  for (int t = tid; t < 4 * n; t += kCombineThreads) {
+    const int i = t >> 2, r = t & 3;
     if (!warp_empty(w0 + i, F, W))
       mloc = fmaxf(mloc, __ldg(pbase + (size_t)i * kPartFloats + kPartM + r));
-  const float M = block_reduce(mloc, true, red);
+  }
+  // lanes l and l^4, l^8, l^16 hold the same head (t & 3 == lane & 3)
+#pragma unroll
+  for (int o = 4; o < 32; o <<= 1) mloc = fmaxf(mloc, __shfl_xor_sync(0xffffffffu, mloc, o));
+  if (lane < 4) red[warp][lane] = mloc;
+  __syncthreads();
+  if (tid < 4) {
+    float M = -INFINITY;
+    for (int w = 0; w < kCombineThreads / 32; ++w) M = fmaxf(M, red[w][tid]);
+    ML[0][tid] = M;
+  }
+  __syncthreads();
   float lloc = 0.f;
-  for (int i = tid; i < n; i += kCombineThreads) {
+  for (int t = tid; t < 4 * n; t += kCombineThreads) {
+    const int i = t >> 2, r = t & 3;
     float wgt = 0.f;
     if (!warp_empty(w0 + i, F, W)) {
       const float* pp = pbase + (size_t)i * kPartFloats;
-      wgt = merge_weight(__ldg(pp + kPartM + r), M);
+      wgt = merge_weight(__ldg(pp + kPartM + r), ML[0][r]);
       lloc += __ldg(pp + kPartL + r) * wgt;
     }
-    wts[i] = wgt;
+    wts[t] = wgt;
   }
-  const float L = block_reduce(lloc, false, red);
-  const float invL = L > 0.f ? 1.f / L : 0.f;
+#pragma unroll
+  for (int o = 4; o < 32; o <<= 1) lloc += __shfl_xor_sync(0xffffffffu, lloc, o);
+  __syncthreads();
+  if (lane < 4) red[warp][lane] = lloc;
+  __syncthreads();
+  if (tid < 4) {
+    float L = 0.f;
+    for (int w = 0; w < kCombineThreads / 32; ++w) L += red[w][tid];
+    ML[1][tid] = L > 0.f ? 1.f / L : 0.f;
+  }
+  __syncthreads();
 
-  float o = 0.f;
+  // merge: thread -> channel j, heads hp and hp + 2
+  {
+    const int j = tid & 127, hp = tid >> 7;
+    float o0 = 0.f, o1 = 0.f;
 #pragma unroll 4
-  for (int i = sl; i < n; i += kSlices) {
-    const float wgt = wts[i];
-    if (wgt != 0.f) o = fmaf(__ldg(pbase + (size_t)i * kPartFloats + r * kD + j), wgt, o);
-  }
-  osl[sl][j] = o;
-  __syncthreads();
-  if (tid < kD) {
-    float t = 0.f;
-#pragma unroll
-    for (int k = 0; k < kSlices; ++k) t += osl[k][tid];
-    orot[tid] = t * invL;
+    for (int i = 0; i < n; ++i) {
+      const float* pp = pbase + (size_t)i * kPartFloats;
+      const float w0v = wts[4 * i + hp], w1v = wts[4 * i + hp + 2];
+      if (w0v != 0.f) o0 = fmaf(__ldg(pp + hp * kD + j), w0v, o0);
+      if (w1v != 0.f) o1 = fmaf(__ldg(pp + (hp + 2) * kD + j), w1v, o1);
+    }
+    orot[hp][j] = o0 * ML[1][hp];
+    orot[hp + 2][j] = o1 * ML[1][hp + 2];
   }
   __syncthreads();
-  // out[i] = sum_jj o'[jj] R_v[i][jj] = sum_jj o'[jj] R_vT[jj][i]
-  const float* RT = R_vT + (size_t)h * kD * kD;
-  float acc = 0.f;
-  const int jj0 = sl * (kD / kSlices);
+  // out[r][i] = sum_jj o'[r][jj] R_v[i][jj] = sum_jj o'[r][jj] R_vT[jj][i]
+  {
+    const int i = tid & 127, hf = tid >> 7;
+    const float* RT = R_vT + (size_t)h * kD * kD + (size_t)(64 * hf) * kD + i;
+    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll 16
+    for (int k = 0; k < 64; ++k) {
+      const float rt = __ldg(RT + k * kD);
 #pragma unroll
-  for (int k = 0; k < kD / kSlices; ++k)
-    acc = fmaf(orot[jj0 + k], __ldg(RT + (jj0 + k) * kD + j), acc);
-  __syncthreads();
-  osl[sl][j] = acc;
-  __syncthreads();
-  if (tid < kD) {
-    float t = 0.f;
+      for (int r = 0; r < 4; ++r) acc[r] = fmaf(orot[r][64 * hf + k], rt, acc[r]);
+    }
+    if (hf == 1) {
 #pragma unroll
-    for (int k = 0; k < kSlices; ++k) t += osl[k][tid];
-    ob[tid] = t;
+      for (int r = 0; r < 4; ++r) half_sum[r][i] = acc[r];
+    }
+    __syncthreads();
+    if (hf == 0) {
+#pragma unroll
+      for (int r = 0; r < 4; ++r) ob[r * kD + i] = acc[r] + half_sum[r][i];
+    }
   }
 }
 
@@ -414,7 +441,7 @@ cudaError_t launch_decode(const optr_params* p, int variant,
   const float qscale = kLog2e / sqrtf((float)kD);
 
   prof_mark(p, 2, s);
-  qrot_kernel<<<dim3(B, h_kv), 128, 0, s>>>(q, p->R_k, B, h_q, h_kv, qscale,
+  qrot_kernel<<<dim3(B, h_kv), kQrotThreads, 0, s>>>(q, p->R_k, B, h_q, h_kv, qscale,
                                             seq_lens, max_pages, qf, qs, frag,
                                             invs, pref, nzpref, p->err);
   cudaError_t e = cudaGetLastError();
@@ -431,10 +458,17 @@ cudaError_t launch_decode(const optr_params* p, int variant,
   }
   if (e != cudaSuccess) return e;
   prof_mark(p, 4, s);
-  combine_kernel<<<dim3(B, h_kv, 4), kCombineThreads,
-                   sizeof(float) * (plan.W + 1), s>>>(part, pref, nzpref, B,
-                                                      h_q, h_kv, plan.W,
-                                                      p->R_vT, out);
+  const size_t wts_bytes = sizeof(float) * 4 * (plan.W + 1);
+  if (wts_bytes > 48 * 1024) {
+    e = cudaFuncSetAttribute(combine_kernel,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)wts_bytes);
+    if (e != cudaSuccess) return e;
+  }
+  combine_kernel<<<dim3(B, h_kv), kCombineThreads,
+                   wts_bytes, s>>>(part, pref, nzpref,
+                                                          B, h_q, h_kv, plan.W,
+                                                          p->R_vT, out);
   prof_mark(p, 5, s);
   return cudaGetLastError();
 }
