@@ -181,18 +181,19 @@ append_small_kernel(const __nv_bfloat16* __restrict__ k,
     dst[tid] = off;
     dslot[tid] = slot;
   }
-  __syncthreads();
   const int sl = tid >> 7, j = tid & 127;
   const float* R = (kind ? R_v : R_k) + (size_t)h * kD * kD + (size_t)(32 * sl) * kD + j;
+  float rv[32];
+#pragma unroll
+  for (int i = 0; i < 32; ++i) rv[i] = __ldg(R + i * kD);  // all in flight
+  __syncthreads();
   float acc[T];
 #pragma unroll
   for (int t = 0; t < T; ++t) acc[t] = 0.f;
-#pragma unroll 8
-  for (int i = 0; i < 32; ++i) {
-    const float r = __ldg(R + i * kD);
 #pragma unroll
-    for (int t = 0; t < T; ++t) acc[t] = fmaf(xs[t][32 * sl + i], r, acc[t]);
-  }
+  for (int i = 0; i < 32; ++i)
+#pragma unroll
+    for (int t = 0; t < T; ++t) acc[t] = fmaf(xs[t][32 * sl + i], rv[i], acc[t]);
 #pragma unroll
   for (int t = 0; t < T; ++t) zp[sl][t][j] = acc[t];
   __syncthreads();

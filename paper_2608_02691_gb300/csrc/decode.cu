@@ -46,15 +46,16 @@ qrot_kernel(const __nv_bfloat16* __restrict__ q, const float* __restrict__ R_k,
     const int r = tid >> 7;  // 512 threads load the 4 x 128 query values
     qsm[r][j] = __bfloat162float(q[((size_t)b * h_q + 4 * h + r) * kD + j]);
   }
-  __syncthreads();
   float acc[4] = {0.f, 0.f, 0.f, 0.f};
   const float* R = R_k + (size_t)h * kD * kD + (size_t)(32 * sl) * kD + j;
-#pragma unroll 16
-  for (int i = 0; i < 32; ++i) {
-    const float rij = __ldg(R + i * kD);
+  float rv[32];
 #pragma unroll
-    for (int r = 0; r < 4; ++r) acc[r] = fmaf(qsm[r][32 * sl + i], rij, acc[r]);
-  }
+  for (int i = 0; i < 32; ++i) rv[i] = __ldg(R + i * kD);  // all in flight
+  __syncthreads();
+#pragma unroll
+  for (int i = 0; i < 32; ++i)
+#pragma unroll
+    for (int r = 0; r < 4; ++r) acc[r] = fmaf(qsm[r][32 * sl + i], rv[i], acc[r]);
 #pragma unroll
   for (int r = 0; r < 4; ++r) part[sl][r][j] = acc[r];
   __syncthreads();
@@ -334,15 +335,35 @@ combine_kernel(const float* __restrict__ part, const int* __restrict__ pref,
   const int w0 = warp_of(fs, F, W), w1 = warp_of(fs + np - 1, F, W);
   const int n = w1 - w0 + 1;
   const float* pbase = part + ((size_t)__ldg(nzpref + b) * h_kv + h + w0) * kPartFloats;
-
-  // per-head maxima over the partials (thread t: partial t/4, head t%4)
-  float mloc = -INFINITY;
-  for (int t = tid; t < 4 * n; t += kCombineThreads) {
-    const int i = t >> 2, r = t & 3;
-    if (!warp_empty(w0 + i, F, W))
-      mloc = fmaxf(mloc, __ldg(pbase + (size_t)i * kPartFloats + kPartM + r));
+  {
+    // warm L2 with this head's R_v^T (64 KB = 512 lines) for the last phase
+    const char* rt = reinterpret_cast<const char*>(R_vT + (size_t)h * kD * kD);
+    asm volatile("prefetch.global.L2 [%0];" ::"l"(rt + 128 * tid));
+    asm volatile("prefetch.global.L2 [%0];" ::"l"(rt + 128 * (tid + kCombineThreads)));
   }
-  // lanes l and l^4, l^8, l^16 hold the same head (t & 3 == lane & 3)
+
+  // One pass over the partial headers: thread t owns (partial t/4, head
+  // t%4) for t < 4n (several per thread when n > 64); maxima first, then
+  // weights and sums from the values kept in registers.
+  constexpr int kPer = 4;
+  float mv[kPer], lv[kPer];
+  float mloc = -INFINITY;
+#pragma unroll
+  for (int u = 0; u < kPer; ++u) {
+    const int t = tid + u * kCombineThreads;
+    mv[u] = -INFINITY;
+    lv[u] = 0.f;
+    if (t < 4 * n && !warp_empty(w0 + (t >> 2), F, W)) {
+      const float* pp = pbase + (size_t)(t >> 2) * kPartFloats;
+      mv[u] = __ldg(pp + kPartM + (t & 3));
+      lv[u] = __ldg(pp + kPartL + (t & 3));
+    }
+    mloc = fmaxf(mloc, mv[u]);
+  }
+  for (int t = tid + kPer * kCombineThreads; t < 4 * n; t += kCombineThreads)
+    if (!warp_empty(w0 + (t >> 2), F, W))
+      mloc = fmaxf(mloc, __ldg(pbase + (size_t)(t >> 2) * kPartFloats + kPartM + (t & 3)));
+  // thread t's head is t & 3 == lane & 3: reduce over lanes of equal head
 #pragma unroll
   for (int o = 4; o < 32; o <<= 1) mloc = fmaxf(mloc, __shfl_xor_sync(0xffffffffu, mloc, o));
   if (lane < 4) red[warp][lane] = mloc;
@@ -354,13 +375,22 @@ combine_kernel(const float* __restrict__ part, const int* __restrict__ pref,
   }
   __syncthreads();
   float lloc = 0.f;
-  for (int t = tid; t < 4 * n; t += kCombineThreads) {
-    const int i = t >> 2, r = t & 3;
+  const float Mh = ML[0][lane & 3];
+#pragma unroll
+  for (int u = 0; u < kPer; ++u) {
+    const int t = tid + u * kCombineThreads;
+    if (t < 4 * n) {
+      const float wgt = merge_weight(mv[u], Mh);
+      lloc += lv[u] * wgt;
+      wts[t] = wgt;
+    }
+  }
+  for (int t = tid + kPer * kCombineThreads; t < 4 * n; t += kCombineThreads) {
     float wgt = 0.f;
-    if (!warp_empty(w0 + i, F, W)) {
-      const float* pp = pbase + (size_t)i * kPartFloats;
-      wgt = merge_weight(__ldg(pp + kPartM + r), ML[0][r]);
-      lloc += __ldg(pp + kPartL + r) * wgt;
+    if (!warp_empty(w0 + (t >> 2), F, W)) {
+      const float* pp = pbase + (size_t)(t >> 2) * kPartFloats;
+      wgt = merge_weight(__ldg(pp + kPartM + (t & 3)), Mh);
+      lloc += __ldg(pp + kPartL + (t & 3)) * wgt;
     }
     wts[t] = wgt;
   }
@@ -380,12 +410,15 @@ combine_kernel(const float* __restrict__ part, const int* __restrict__ pref,
   {
     const int j = tid & 127, hp = tid >> 7;
     float o0 = 0.f, o1 = 0.f;
-#pragma unroll 4
+    // empty partials have weight 0; their (never written) slots are read
+    // but multiplied by a select, never accumulated
+#pragma unroll 8
     for (int i = 0; i < n; ++i) {
       const float* pp = pbase + (size_t)i * kPartFloats;
       const float w0v = wts[4 * i + hp], w1v = wts[4 * i + hp + 2];
-      if (w0v != 0.f) o0 = fmaf(__ldg(pp + hp * kD + j), w0v, o0);
-      if (w1v != 0.f) o1 = fmaf(__ldg(pp + (hp + 2) * kD + j), w1v, o1);
+      const float a0 = __ldg(pp + hp * kD + j), a1 = __ldg(pp + (hp + 2) * kD + j);
+      o0 += w0v != 0.f ? a0 * w0v : 0.f;
+      o1 += w1v != 0.f ? a1 * w1v : 0.f;
     }
     orot[hp][j] = o0 * ML[1][hp];
     orot[hp + 2][j] = o1 * ML[1][hp + 2];

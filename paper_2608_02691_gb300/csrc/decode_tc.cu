@@ -25,6 +25,8 @@
 // would show in the output.)  q' and p*scale are split into fp16 hi + lo
 // parts, which fill the 8 MMA columns and keep ~22 bits of the float32
 // operands.
+#include <type_traits>
+
 #include "decode_common.cuh"
 
 namespace optr {
@@ -37,7 +39,10 @@ constexpr float kLazyTau = 8.f;       // log2-domain slack before rescaling
 struct WarpSmemTC {
   alignas(16) uint8_t stage[kStages][kChunk];
   alignas(16) uint32_t pt[kGroups][kPage][4];  // p*scale_v (hi, lo) per head
+  int2 info[kStages];  // per staged page: (segment key b*h_kv+h, valid tokens)
 };
+
+constexpr int kPrefCache = 256;  // sequences whose page prefix sums a CTA caches
 
 __device__ __forceinline__ void mma16816(float* d, uint32_t a0, uint32_t a1,
                                          uint32_t a2, uint32_t a3, uint32_t b0,
@@ -60,10 +65,13 @@ __device__ __forceinline__ void ldsm_x4_trans(uint32_t& r0, uint32_t& r1,
 }
 
 // Two codes (the fields at bit 2r of each 16-bit half of src) as exact
-// fp16 values 0..3.
+// fp16 values 0..3.  exp1024 holds 0x64006400 (the exponent of 1024 in both
+// halves) in a register, so that mask-and-or is a single LOP3.
 template <int r>
-__device__ __forceinline__ uint32_t codes_f16x2(uint32_t src) {
-  const uint32_t x = (src & (0x00030003u << (2 * r))) | 0x64006400u;
+__device__ __forceinline__ uint32_t codes_f16x2(uint32_t src, uint32_t exp1024) {
+  uint32_t x;
+  asm("lop3.b32 %0, %1, %2, %3, 0xEA;"  // (a & b) | c
+      : "=r"(x) : "r"(src), "n"(0x00030003u << (2 * r)), "r"(exp1024));
   const __half2 sc = __float2half2_rn(1.0f / (float)(1 << (2 * r)));
   const __half2 bias = __float2half2_rn(-1024.0f / (float)(1 << (2 * r)));
   const __half2 y = __hfma2(*reinterpret_cast<const __half2*>(&x), sc, bias);
@@ -77,63 +85,71 @@ __device__ __forceinline__ float2 h2f(uint32_t u) {
 // fp16 hi / lo split of x, packed (hi in the low half).
 __device__ __forceinline__ uint32_t split_hilo(float x) {
   const __half hi = __float2half_rn(x);
-  const __half lo = __float2half_rn(x - __half2float(hi));
-  return (uint32_t)__half_as_ushort(hi) | ((uint32_t)__half_as_ushort(lo) << 16);
+  const float lo = x - __half2float(hi);
+  uint32_t r;
+  asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(lo), "f"(x));
+  return r;
 }
 
-// Iterator over a warp's flat page range: yields (b, h, page) in order,
-// seeking the next (sequence, KV head) segment at each boundary.
-struct PageIter {
-  long long f, f1, seg_end;
-  int b, h, page;
-  __device__ void init(long long f0, long long fend, const int* pref, int B,
-                       int h_kv) {
-    f = f0;
-    f1 = fend;
-    seg_end = f0;
-    b = h = page = 0;
-    if (f < f1) seek(pref, B, h_kv);
-  }
-  __device__ void seek(const int* pref, int B, int h_kv) {
-    Segment s = locate_segment(f, f1, pref, B, h_kv);
-    b = s.b;
-    h = s.h;
-    page = s.p0;
-    seg_end = s.f_end;
-  }
-  __device__ bool valid() const { return f < f1; }
-  // true when the step entered a new segment
-  __device__ bool next(const int* pref, int B, int h_kv) {
-    ++f;
-    ++page;
-    if (f < f1 && f == seg_end) {
-      seek(pref, B, h_kv);
-      return true;
-    }
-    return false;
-  }
-};
+// 2^x (the MUFU approximation; relative error ~2^-22).
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
 
-// The issuing side also holds the block-table entries of the next 32 pages
-// of its segment, one per lane, so that a page issue needs no dependent
-// global load.
-struct IssueIter : PageIter {
+// The issuing side of a warp walks its flat page range
+// [f, f1) (sequence-major, then KV head, then page); it keeps the block-table
+// entries of the next 32 pages of its segment one per lane, so that issuing a
+// page needs no dependent global load, and steps from one segment to the
+// next without a search.
+struct Issuer {
+  int f, f1;          // flat page indices still to issue
+  int b, h, page;     // current segment and page
+  int np;             // pages of sequence b
+  int len;            // tokens of sequence b
   int chunk_base;
   int32_t btreg;
-  __device__ void load_chunk(const int32_t* __restrict__ bt, int max_pages,
-                             int lane) {
+  int h_kv, max_pages;
+
+  __device__ void load_chunk(const int32_t* __restrict__ bt, int lane) {
     chunk_base = page;
-    const long long left = seg_end - f;  // pages left in this segment
-    btreg = lane < left ? __ldg(bt + (size_t)b * max_pages + page + lane) : -1;
+    btreg = (page + lane < np) ? __ldg(bt + (size_t)b * max_pages + page + lane) : -1;
   }
-  __device__ int phys(const int32_t* __restrict__ bt, int max_pages, int lane) {
-    if (page - chunk_base >= 32) load_chunk(bt, max_pages, lane);
+  // first segment: f lies in sequence b with pref[b]*h_kv <= f < pref[b+1]*h_kv
+  __device__ void start(int f_begin, int f_end, int bb, const int* __restrict__ pref,
+                        const int32_t* __restrict__ seq_lens,
+                        const int32_t* __restrict__ bt, int lane) {
+    f = f_begin;
+    f1 = f_end;
+    b = bb;
+    np = __ldg(pref + b + 1) - __ldg(pref + b);
+    len = __ldg(seq_lens + b);
+    const int r = f - __ldg(pref + b) * h_kv;
+    h = r / np;
+    page = r - h * np;
+    load_chunk(bt, lane);
+  }
+  __device__ int phys(const int32_t* __restrict__ bt, int lane) {
+    if (page - chunk_base >= 32) load_chunk(bt, lane);
     return __shfl_sync(0xffffffffu, btreg, page - chunk_base);
   }
-  __device__ void advance(const int* pref, int B, int h_kv,
-                          const int32_t* __restrict__ bt, int max_pages,
-                          int lane) {
-    if (next(pref, B, h_kv)) load_chunk(bt, max_pages, lane);
+  __device__ int nvalid() const { return min(kPage, len - page * kPage); }
+  __device__ void advance(const int* __restrict__ pref,
+                          const int32_t* __restrict__ seq_lens,
+                          const int32_t* __restrict__ bt, int lane) {
+    ++f;
+    if (++page < np || f >= f1) return;
+    page = 0;
+    if (++h == h_kv) {  // next non-empty sequence
+      h = 0;
+      do {
+        ++b;
+        np = __ldg(pref + b + 1) - __ldg(pref + b);
+      } while (np == 0);
+      len = __ldg(seq_lens + b);
+    }
+    load_chunk(bt, lane);
   }
 };
 
@@ -149,32 +165,50 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
                       const int* __restrict__ nzpref,
                       float* __restrict__ part, int W, unsigned* err) {
   __shared__ WarpSmemTC smem[kWarps];
+  __shared__ int spref[kPrefCache + 1];
+  uint32_t e1024;
+  asm volatile("mov.b32 %0, 0x64006400;" : "=r"(e1024));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int g = lane >> 2, c = lane & 3;
   WarpSmemTC& S = smem[warp];
   const int w = blockIdx.x * kWarps + warp;
-  const long long F = (long long)__ldg(pref + B) * h_kv;
-  const long long f0 = w * F / W, f1 = (w + 1) * F / W;
-  if (f0 >= f1) return;
+  const int F = __ldg(pref + B) * h_kv;
+  const int f0 = (int)((long long)w * F / W), f1 = (int)((long long)(w + 1) * F / W);
 
-  // issue iterator runs kStages-1 pages ahead of the compute iterator
-  IssueIter is;
-  PageIter cs;
-  is.init(f0, f1, pref, B, h_kv);
-  cs = is;
-  is.load_chunk(bt, max_pages, lane);
-  unsigned okmask = 0;  // bit s: stage s holds a page that was read
-#pragma unroll
-  for (int s = 0; s < kStages - 1; ++s) {
-    if (is.valid()) {
-      if (issue_phys(S.stage[s], pool, is.phys(bt, max_pages, lane),
-                     num_pages, h_kv, is.h, lane, err))
-        okmask |= 1u << s;
-      is.advance(pref, B, h_kv, bt, max_pages, lane);
+  // first segment of this warp: sequence b with pref[b]*h_kv <= f0
+  const bool cached = B <= kPrefCache;
+  if (cached)
+    for (int i = threadIdx.x; i <= B; i += kWarps * 32) spref[i] = __ldg(pref + i);
+  __syncthreads();
+  if (f0 >= f1) return;
+  int b0;
+  {
+    int lo = 0, hi = B;
+    while (hi - lo > 1) {
+      const int mid = (lo + hi) >> 1;
+      const int pm = cached ? spref[mid] : __ldg(pref + mid);
+      if (pm * h_kv <= f0) lo = mid; else hi = mid;
+    }
+    b0 = lo;
+  }
+  Issuer is;
+  is.h_kv = h_kv;
+  is.max_pages = max_pages;
+  is.start(f0, f1, b0, pref, seq_lens, bt, lane);
+
+  // issue one page into stage s; lane 0 records what the stage holds
+  auto issue = [&](int s) {
+    if (is.f < is.f1) {
+      const int ph = is.phys(bt, lane);
+      const bool ok = issue_phys(S.stage[s], pool, ph, num_pages, h_kv, is.h, lane, err);
+      S.info[s] = make_int2(is.b * h_kv + is.h, ok ? is.nvalid() : 0);  // same value from every lane
+      is.advance(pref, seq_lens, bt, lane);
     } else {
       cp_async_commit();
     }
-  }
+  };
+#pragma unroll
+  for (int s = 0; s < kStages - 1; ++s) issue(s);
 
   // per-segment state
   uint32_t bq[kGroups][2][2];  // query B fragments [group][kk][reg]
@@ -183,7 +217,7 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
   float acc_o[kGroups][2][4];  // values: [group][half][c-frag]
   float mv[kGroups];           // sum_tok p * min_v per group (this lane)
   float m_run = -INFINITY, l_lane = 0.f;
-  int cur_b = -1, cur_h = -1, len = 0;
+  int cur_key = -1;
 
   auto flush = [&]() {
     // reduce l and the min-terms over the 8 lanes of head c, then write
@@ -195,7 +229,8 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
 #pragma unroll
       for (int o = 4; o < 32; o <<= 1)
         mv[G] += __shfl_xor_sync(0xffffffffu, mv[G], o);
-    float* slot = part + (size_t)(w + __ldg(nzpref + cur_b) * h_kv + cur_h) * kPartFloats;
+    const int cb = cur_key / h_kv, ch = cur_key - cb * h_kv;
+    float* slot = part + (size_t)(w + __ldg(nzpref + cb) * h_kv + ch) * kPartFloats;
     float* dst = slot + c * kD;
 #pragma unroll
     for (int G = 0; G < kGroups; ++G) {
@@ -214,61 +249,45 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
     }
   };
 
-  for (int i = 0; cs.valid(); ++i) {
-    // keep kStages-1 pages in flight
-    const int slot_issue = (i + kStages - 1) % kStages;
-    okmask &= ~(1u << slot_issue);
-    if (is.valid()) {
-      if (issue_phys(S.stage[slot_issue], pool, is.phys(bt, max_pages, lane),
-                     num_pages, h_kv, is.h, lane, err))
-        okmask |= 1u << slot_issue;
-      is.advance(pref, B, h_kv, bt, max_pages, lane);
-    } else {
-      cp_async_commit();
+  auto begin_segment = [&](int key) {
+    cur_key = key;
+    const int cb = key / h_kv, ch = key - cb * h_kv;
+    const uint4* fq = reinterpret_cast<const uint4*>(
+        frag + (((size_t)cb * h_kv + ch) * 32 + lane) * 16);
+#pragma unroll
+    for (int G = 0; G < kGroups; ++G) {
+      const uint4 v = __ldg(fq + G);
+      bq[G][0][0] = v.x;
+      bq[G][0][1] = v.y;
+      bq[G][1][0] = v.z;
+      bq[G][1][1] = v.w;
     }
-    cp_async_wait<kStages - 1>();
-    __syncwarp();
-
-    if (cs.b != cur_b || cs.h != cur_h) {
-      if (cur_b >= 0) flush();
-      cur_b = cs.b;
-      cur_h = cs.h;
-      len = __ldg(seq_lens + cur_b);
-      const uint4* fq = reinterpret_cast<const uint4*>(
-          frag + (((size_t)cur_b * h_kv + cur_h) * 32 + lane) * 16);
+    const size_t row = (size_t)cb * h_q + 4 * ch + c;
+    const float4 q4 = __ldg(reinterpret_cast<const float4*>(qs + row * kGroups));
+    qsum[0] = q4.x;
+    qsum[1] = q4.y;
+    qsum[2] = q4.z;
+    qsum[3] = q4.w;
+    inv_s = __ldg(invs + row);
 #pragma unroll
-      for (int G = 0; G < kGroups; ++G) {
-        const uint4 v = __ldg(fq + G);
-        bq[G][0][0] = v.x;
-        bq[G][0][1] = v.y;
-        bq[G][1][0] = v.z;
-        bq[G][1][1] = v.w;
-      }
-      const size_t row = (size_t)cur_b * h_q + 4 * cur_h + c;
-      const float4 q4 = __ldg(reinterpret_cast<const float4*>(qs + row * kGroups));
-      qsum[0] = q4.x;
-      qsum[1] = q4.y;
-      qsum[2] = q4.z;
-      qsum[3] = q4.w;
-      inv_s = __ldg(invs + row);
+    for (int G = 0; G < kGroups; ++G) {
+      mv[G] = 0.f;
 #pragma unroll
-      for (int G = 0; G < kGroups; ++G) {
-        mv[G] = 0.f;
+      for (int hf = 0; hf < 2; ++hf)
 #pragma unroll
-        for (int hf = 0; hf < 2; ++hf)
-#pragma unroll
-          for (int k = 0; k < 4; ++k) acc_o[G][hf][k] = 0.f;
-      }
-      m_run = -INFINITY;
-      l_lane = 0.f;
+        for (int k = 0; k < 4; ++k) acc_o[G][hf][k] = 0.f;
     }
+    m_run = -INFINITY;
+    l_lane = 0.f;
+  };
 
-    const uint8_t* st = S.stage[i % kStages];
-    const bool ok = (okmask >> (i % kStages)) & 1u;
-    const int nvalid = ok ? min(kPage, len - cs.page * kPage) : 0;
-
-    // ---------------------------------------------------------- logits
-    float sc[2];
+  // One page of the stage st: logits, online softmax, values.  FULL = all
+  // 16 tokens valid (no masking code).
+  auto page = [&](const uint8_t* st, int nvalid, auto full_tag) {
+    constexpr bool FULL = decltype(full_tag)::value;
+    const bool v0 = FULL || g < nvalid, v1 = FULL || g + 8 < nvalid;
+    // ------------------------------------------------------------ logits
+    float sc0, sc1;
     {
       const uint2 k0 = *reinterpret_cast<const uint2*>(st + OPTR_K_CODES_OFFSET + g * 32 + 8 * c);
       const uint2 k1 = *reinterpret_cast<const uint2*>(st + OPTR_K_CODES_OFFSET + (g + 8) * 32 + 8 * c);
@@ -284,11 +303,11 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
         const uint32_t src1 = (G < 2 ? y01_1 : y23_1) >> (8 * (G & 1));
 #pragma unroll
         for (int k = 0; k < 4; ++k) s_acc[G][k] = 0.f;
-        mma16816(s_acc[G], codes_f16x2<0>(src0), codes_f16x2<0>(src1),
-                 codes_f16x2<1>(src0), codes_f16x2<1>(src1), bq[G][0][0],
+        mma16816(s_acc[G], codes_f16x2<0>(src0, e1024), codes_f16x2<0>(src1, e1024),
+                 codes_f16x2<1>(src0, e1024), codes_f16x2<1>(src1, e1024), bq[G][0][0],
                  bq[G][0][1]);
-        mma16816(s_acc[G], codes_f16x2<2>(src0), codes_f16x2<2>(src1),
-                 codes_f16x2<3>(src0), codes_f16x2<3>(src1), bq[G][1][0],
+        mma16816(s_acc[G], codes_f16x2<2>(src0, e1024), codes_f16x2<2>(src1, e1024),
+                 codes_f16x2<3>(src0, e1024), codes_f16x2<3>(src1, e1024), bq[G][1][0],
                  bq[G][1][1]);
       }
       const uint4 km0 = *reinterpret_cast<const uint4*>(st + OPTR_K_META_OFFSET + g * 16);
@@ -298,43 +317,53 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
       float t0 = 0.f, t1 = 0.f, u0 = 0.f, u1 = 0.f;
 #pragma unroll
       for (int G = 0; G < kGroups; ++G) {
-        const float2 a = h2f(kmv0[G]);  // (scale, min) of token g
-        const float2 bb = h2f(kmv1[G]); // token g+8
+        const float2 a = h2f(kmv0[G]);   // (scale, min) of token g
+        const float2 bb = h2f(kmv1[G]);  // token g+8
         t0 = fmaf(a.x, s_acc[G][0] + s_acc[G][1], t0);
         t1 = fmaf(bb.x, s_acc[G][2] + s_acc[G][3], t1);
         u0 = fmaf(a.y, qsum[G], u0);
         u1 = fmaf(bb.y, qsum[G], u1);
       }
-      sc[0] = g < nvalid ? fmaf(inv_s, t0, u0) : -INFINITY;
-      sc[1] = g + 8 < nvalid ? fmaf(inv_s, t1, u1) : -INFINITY;
-    }
-
-    // ------------------------------------------------ online softmax
-    float tmax = fmaxf(sc[0], sc[1]);
-#pragma unroll
-    for (int o = 4; o < 32; o <<= 1) tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, o));
-    const bool need = tmax > m_run + kLazyTau;
-    if (__any_sync(0xffffffffu, need)) {
-      const float m_new = need ? tmax : m_run;
-      const float alpha = (m_run == -INFINITY) ? 0.f : exp2f(m_run - m_new);
-      if (need) {
-        l_lane *= alpha;
-#pragma unroll
-        for (int G = 0; G < kGroups; ++G) {
-          mv[G] *= alpha;
-#pragma unroll
-          for (int hf = 0; hf < 2; ++hf)
-#pragma unroll
-            for (int k = 0; k < 4; ++k) acc_o[G][hf][k] *= alpha;
-        }
-        m_run = m_new;
+      sc0 = fmaf(inv_s, t0, u0);
+      sc1 = fmaf(inv_s, t1, u1);
+      if (!FULL) {
+        sc0 = v0 ? sc0 : -INFINITY;
+        sc1 = v1 ? sc1 : -INFINITY;
       }
     }
-    const float p0 = sc[0] == -INFINITY ? 0.f : exp2f(sc[0] - m_run);
-    const float p1 = sc[1] == -INFINITY ? 0.f : exp2f(sc[1] - m_run);
+    // ---------------------------------------------------- online softmax
+    // Lazy rescaling: the running reference m_run of head c only moves when
+    // some logit exceeds it by more than kLazyTau (log2 units), so p <= 2^8.
+    // Each lane tests its own logits; only then is the head maximum reduced
+    // over the 8 lanes of the head and the accumulators rescaled.
+    {
+      const float lmax = fmaxf(sc0, sc1);
+      if (__any_sync(0xffffffffu, lmax > m_run + kLazyTau)) {
+        float tmax = lmax;
+#pragma unroll
+        for (int o = 4; o < 32; o <<= 1) tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, o));
+        if (tmax > m_run + kLazyTau) {  // uniform over the lanes of head c
+          const float alpha = (m_run == -INFINITY) ? 0.f : ex2(m_run - tmax);
+          l_lane *= alpha;
+#pragma unroll
+          for (int G = 0; G < kGroups; ++G) {
+            mv[G] *= alpha;
+#pragma unroll
+            for (int hf = 0; hf < 2; ++hf)
+#pragma unroll
+              for (int k = 0; k < 4; ++k) acc_o[G][hf][k] *= alpha;
+          }
+          m_run = tmax;
+        }
+      }
+    }
+    float p0 = ex2(sc0 - m_run), p1 = ex2(sc1 - m_run);  // ex2(-inf) = 0
+    if (!FULL) {  // a fully masked page before any finite max: -inf - -inf
+      p0 = v0 ? p0 : 0.f;
+      p1 = v1 ? p1 : 0.f;
+    }
     l_lane += p0 + p1;
-
-    // ----------------------------------------------------------- values
+    // ------------------------------------------------------------ values
     {
       const uint4 vm0 = *reinterpret_cast<const uint4*>(st + OPTR_V_META_OFFSET + g * 16);
       const uint4 vm1 = *reinterpret_cast<const uint4*>(st + OPTR_V_META_OFFSET + (g + 8) * 16);
@@ -342,16 +371,17 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
       const uint32_t vmv1[4] = {vm1.x, vm1.y, vm1.z, vm1.w};
 #pragma unroll
       for (int G = 0; G < kGroups; ++G) {
-        const float2 a = h2f(vmv0[G]);
-        const float2 bb = h2f(vmv1[G]);
-        // masked tokens: p = 0, and their (possibly garbage) metadata is
-        // never multiplied in
-        const float pt0 = g < nvalid ? p0 * a.x : 0.f;
-        const float pt1 = g + 8 < nvalid ? p1 * bb.x : 0.f;
-        if (g < nvalid) mv[G] = fmaf(p0, a.y, mv[G]);
-        if (g + 8 < nvalid) mv[G] = fmaf(p1, bb.y, mv[G]);
-        S.pt[G][g][c] = split_hilo(pt0);
-        S.pt[G][g + 8][c] = split_hilo(pt1);
+        float2 a = h2f(vmv0[G]);
+        float2 bb = h2f(vmv1[G]);
+        if (!FULL) {
+          // masked tokens have p = 0; their (possibly garbage) metadata is
+          // never multiplied in
+          a = v0 ? a : make_float2(0.f, 0.f);
+          bb = v1 ? bb : make_float2(0.f, 0.f);
+        }
+        mv[G] = fmaf(p0, a.y, fmaf(p1, bb.y, mv[G]));
+        S.pt[G][g][c] = split_hilo(p0 * a.x);
+        S.pt[G][g + 8][c] = split_hilo(p1 * bb.x);
       }
     }
     __syncwarp();
@@ -375,14 +405,37 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
       for (int G = 0; G < kGroups; ++G) {
         const uint32_t sa = (G < 2 ? a01 : a23) >> (8 * (G & 1));
         const uint32_t sb = (G < 2 ? b01 : b23) >> (8 * (G & 1));
-        mma16816(acc_o[G][0], codes_f16x2<0>(sa), codes_f16x2<1>(sa),
-                 codes_f16x2<0>(sb), codes_f16x2<1>(sb), bv[G][0], bv[G][1]);
-        mma16816(acc_o[G][1], codes_f16x2<2>(sa), codes_f16x2<3>(sa),
-                 codes_f16x2<2>(sb), codes_f16x2<3>(sb), bv[G][0], bv[G][1]);
+        mma16816(acc_o[G][0], codes_f16x2<0>(sa, e1024), codes_f16x2<1>(sa, e1024),
+                 codes_f16x2<0>(sb, e1024), codes_f16x2<1>(sb, e1024), bv[G][0], bv[G][1]);
+        mma16816(acc_o[G][1], codes_f16x2<2>(sa, e1024), codes_f16x2<3>(sa, e1024),
+                 codes_f16x2<2>(sb, e1024), codes_f16x2<3>(sb, e1024), bv[G][0], bv[G][1]);
       }
     }
-    __syncwarp();
-    cs.next(pref, B, h_kv);
+  };
+
+  const int total = f1 - f0;
+  int done = 0;
+  while (done < total) {
+#pragma unroll
+    for (int s = 0; s < kStages; ++s) {
+      if (done < total) {
+        issue((s + kStages - 1) % kStages);
+        cp_async_wait<kStages - 1>();
+        __syncwarp();
+        const int2 inf = S.info[s];
+        const int nvalid = inf.y;
+        if (inf.x != cur_key) {
+          if (cur_key >= 0) flush();
+          begin_segment(inf.x);
+        }
+        if (nvalid == kPage)
+          page(S.stage[s], nvalid, std::true_type{});
+        else
+          page(S.stage[s], nvalid, std::false_type{});
+        __syncwarp();
+        ++done;
+      }
+    }
   }
   flush();
 }

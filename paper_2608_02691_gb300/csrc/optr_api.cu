@@ -201,6 +201,9 @@ optr_status optr_decode_attention(const optr_params* p, const void* q,
     return OPTR_ERR_INVALID_ARG;
   if ((long long)max_pages * kPage > (1LL << 30) || B > (1 << 24))
     return OPTR_ERR_OUT_OF_RANGE;
+  // the split-K plan indexes (sequence, KV head, page) units with 32 bits
+  if ((long long)B * max_pages * p->cfg.h_kv >= (1LL << 31))
+    return OPTR_ERR_OUT_OF_RANGE;
   DecodePlan plan = decode_plan(p, B, max_pages);
   if (!workspace || ws_bytes < plan.total || !aligned(workspace, 256))
     return OPTR_ERR_WORKSPACE;
