@@ -98,60 +98,52 @@ __device__ __forceinline__ float ex2(float x) {
   return y;
 }
 
-// The issuing side of a warp walks its flat page range
-// [f, f1) (sequence-major, then KV head, then page); it keeps the block-table
-// entries of the next 32 pages of its segment one per lane, so that issuing a
-// page needs no dependent global load, and steps from one segment to the
-// next without a search.
-struct Issuer {
-  int f, f1;          // flat page indices still to issue
-  int b, h, page;     // current segment and page
-  int np;             // pages of sequence b
-  int len;            // tokens of sequence b
-  int chunk_base;
-  int32_t btreg;
-  int h_kv, max_pages;
-
-  __device__ void load_chunk(const int32_t* __restrict__ bt, int lane) {
-    chunk_base = page;
-    btreg = (page + lane < np) ? __ldg(bt + (size_t)b * max_pages + page + lane) : -1;
-  }
-  // first segment: f lies in sequence b with pref[b]*h_kv <= f < pref[b+1]*h_kv
-  __device__ void start(int f_begin, int f_end, int bb, const int* __restrict__ pref,
-                        const int32_t* __restrict__ seq_lens,
-                        const int32_t* __restrict__ bt, int lane) {
-    f = f_begin;
-    f1 = f_end;
-    b = bb;
-    np = __ldg(pref + b + 1) - __ldg(pref + b);
-    len = __ldg(seq_lens + b);
-    const int r = f - __ldg(pref + b) * h_kv;
-    h = r / np;
-    page = r - h * np;
-    load_chunk(bt, lane);
-  }
-  __device__ int phys(const int32_t* __restrict__ bt, int lane) {
-    if (page - chunk_base >= 32) load_chunk(bt, lane);
-    return __shfl_sync(0xffffffffu, btreg, page - chunk_base);
-  }
-  __device__ int nvalid() const { return min(kPage, len - page * kPage); }
-  __device__ void advance(const int* __restrict__ pref,
-                          const int32_t* __restrict__ seq_lens,
-                          const int32_t* __restrict__ bt, int lane) {
-    ++f;
-    if (++page < np || f >= f1) return;
-    page = 0;
-    if (++h == h_kv) {  // next non-empty sequence
-      h = 0;
-      do {
-        ++b;
-        np = __ldg(pref + b + 1) - __ldg(pref + b);
-      } while (np == 0);
-      len = __ldg(seq_lens + b);
-    }
-    load_chunk(bt, lane);
-  }
+// The issuing side of a warp describes its flat page range
+// (sequence-major, then KV head, then page) 32 pages at a time: lane l of a
+// chunk resolves flat page base + l to its physical page, segment key
+// (b * h_kv + h) and valid token count, so that issuing a page is a shuffle
+// and an address computation with no dependent global load.
+struct PageChunk {
+  int base;        // first flat page of the chunk
+  int unit;        // this lane's page: physical page * h_kv + h, or -1
+  int key, nvalid; // segment key b * h_kv + h and valid tokens
 };
+
+__device__ __forceinline__ void load_chunk(PageChunk& ch, int base, int f1,
+                                           const int* __restrict__ pref,
+                                           const int* spref, bool cached,
+                                           const int32_t* __restrict__ seq_lens,
+                                           const int32_t* __restrict__ bt,
+                                           int B, int h_kv, int max_pages,
+                                           int num_pages, unsigned* err,
+                                           int lane) {
+  ch.base = base;
+  ch.unit = -1;
+  ch.key = -1;
+  ch.nvalid = 0;
+  const int f = base + lane;
+  if (f < f1) {
+    int lo = 0, hi = B;  // largest b with pref[b] * h_kv <= f
+    while (hi - lo > 1) {
+      const int mid = (lo + hi) >> 1;
+      const int pm = cached ? spref[mid] : __ldg(pref + mid);
+      if (pm * h_kv <= f) lo = mid; else hi = mid;
+    }
+    const int p0 = cached ? spref[lo] : __ldg(pref + lo);
+    const int np = (cached ? spref[lo + 1] : __ldg(pref + lo + 1)) - p0;
+    const int r = f - p0 * h_kv;
+    const int h = r / np;
+    const int page = r - h * np;
+    const int phys = __ldg(bt + (size_t)lo * max_pages + page);
+    ch.key = lo * h_kv + h;
+    if (phys >= 0 && phys < num_pages) {
+      ch.unit = phys * h_kv + h;
+      ch.nvalid = min(kPage, __ldg(seq_lens + lo) - page * kPage);
+    } else {
+      atomicOr(err, OPTR_DEVERR_PAGE_ID);  // skipped: its tokens count as masked
+    }
+  }
+}
 
 __global__ void __launch_bounds__(kWarps * 32, 4)
 partial_tensor_kernel(const uint8_t* __restrict__ pool,
@@ -181,28 +173,31 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
     for (int i = threadIdx.x; i <= B; i += kWarps * 32) spref[i] = __ldg(pref + i);
   __syncthreads();
   if (f0 >= f1) return;
-  int b0;
-  {
-    int lo = 0, hi = B;
-    while (hi - lo > 1) {
-      const int mid = (lo + hi) >> 1;
-      const int pm = cached ? spref[mid] : __ldg(pref + mid);
-      if (pm * h_kv <= f0) lo = mid; else hi = mid;
-    }
-    b0 = lo;
-  }
-  Issuer is;
-  is.h_kv = h_kv;
-  is.max_pages = max_pages;
-  is.start(f0, f1, b0, pref, seq_lens, bt, lane);
+  PageChunk chk;
+  int f_issue = f0;
+  load_chunk(chk, f0, f1, pref, spref, cached, seq_lens, bt, B, h_kv,
+             max_pages, num_pages, err, lane);
 
-  // issue one page into stage s; lane 0 records what the stage holds
+  // issue one page into stage s; every lane records what the stage holds
   auto issue = [&](int s) {
-    if (is.f < is.f1) {
-      const int ph = is.phys(bt, lane);
-      const bool ok = issue_phys(S.stage[s], pool, ph, num_pages, h_kv, is.h, lane, err);
-      S.info[s] = make_int2(is.b * h_kv + is.h, ok ? is.nvalid() : 0);  // same value from every lane
-      is.advance(pref, seq_lens, bt, lane);
+    if (f_issue < f1) {
+      if (f_issue - chk.base == 32)
+        load_chunk(chk, f_issue, f1, pref, spref, cached, seq_lens, bt, B, h_kv,
+                   max_pages, num_pages, err, lane);
+      const int j = f_issue - chk.base;
+      const int unit = __shfl_sync(0xffffffffu, chk.unit, j);
+      const int key = __shfl_sync(0xffffffffu, chk.key, j);
+      const int nv = __shfl_sync(0xffffffffu, chk.nvalid, j);
+      if (unit >= 0) {
+        const uint8_t* src = pool + (size_t)unit * kChunk + lane * 16;
+        uint8_t* dst = S.stage[s] + lane * 16;
+        cp_async16(dst, src);
+        cp_async16(dst + 512, src + 512);
+        cp_async16(dst + 1024, src + 1024);
+      }
+      cp_async_commit();
+      S.info[s] = make_int2(key, nv);  // same value from every lane
+      ++f_issue;
     } else {
       cp_async_commit();
     }
