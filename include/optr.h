@@ -133,6 +133,7 @@ typedef enum {
 #define OPTR_DEVERR_POSITION 2u  /* append position >= max_pages * 16 or <0 */
 #define OPTR_DEVERR_SEQ_LEN 4u   /* seq_lens[b] < 0 or > max_pages * 16     */
 #define OPTR_DEVERR_CU_NEW 8u    /* cu_new not non-decreasing within n_tok  */
+#define OPTR_DEVERR_FP16_RANGE 16u /* tensor-core append: |k| or |v| >= 65504 */
 
 /* Kernel variants (for measurement; 0 picks the library default). */
 #define OPTR_VARIANT_DEFAULT 0
@@ -189,7 +190,10 @@ size_t optr_page_bytes(const optr_params* p);
  *   block_table device int32 [B][max_pages]: logical page -> physical page.
  *   pool        device bytes [num_pages][h_kv][1536], written in place.
  * Each written slot's codes and metadata are replaced entirely.  Two appends
- * that target the same slot concurrently race.  Out-of-range table entries
+ * that target the same slot concurrently race.  The tensor-core variant
+ * (default for more than 256 new tokens) converts k and v to fp16: values of
+ * magnitude 65504 or more set OPTR_DEVERR_FP16_RANGE (use the CUDA-core
+ * variant for such inputs).  Out-of-range table entries
  * or positions skip that token and set a device error bit.
  */
 optr_status optr_kv_append(const optr_params* p, const void* k, const void* v,

@@ -4,48 +4,10 @@
 // mu R_K precomputed, subtracted right after the rotation).
 #include "optr_internal.cuh"
 #include "quant.cuh"
+#include "append_common.cuh"
 
 namespace optr {
 namespace {
-
-// Sequence of new token t: the largest b with cu_new[b] <= t.
-__device__ __forceinline__ int find_seq(const int32_t* __restrict__ cu_new,
-                                        int B, int t) {
-  int lo = 0, hi = B;
-  while (hi - lo > 1) {
-    int mid = (lo + hi) >> 1;
-    if (__ldg(cu_new + mid) <= t) lo = mid; else hi = mid;
-  }
-  return lo;
-}
-
-// Byte offset in the pool of the chunk (page, h) and the slot of new token
-// `tok`, or -1 (after flagging the device error word) when a table entry,
-// position or cu_new entry is out of range.
-__device__ long long resolve_slot(int tok, int h, const int32_t* __restrict__ cu_new,
-                                  const int32_t* __restrict__ pos0,
-                                  const int32_t* __restrict__ bt, int B,
-                                  int max_pages, int num_pages, int h_kv,
-                                  int* slot, unsigned* err) {
-  int b = find_seq(cu_new, B, tok);
-  int c0 = __ldg(cu_new + b), c1 = __ldg(cu_new + b + 1);
-  if (!(c0 <= tok && tok < c1)) {
-    atomicOr(err, OPTR_DEVERR_CU_NEW);
-    return -1;
-  }
-  long long pos = (long long)__ldg(pos0 + b) + (tok - c0);
-  if (pos < 0 || pos >= (long long)max_pages * kPage) {
-    atomicOr(err, OPTR_DEVERR_POSITION);
-    return -1;
-  }
-  int page = __ldg(bt + (size_t)b * max_pages + pos / kPage);
-  if (page < 0 || page >= num_pages) {
-    atomicOr(err, OPTR_DEVERR_PAGE_ID);
-    return -1;
-  }
-  *slot = (int)(pos % kPage);
-  return ((long long)page * h_kv + h) * kChunk;
-}
 
 // CUDA-core variant.  Block = 256 threads: warp w < 4 computes key group w,
 // warp w >= 4 value group w-4; lane = channel within the group.  Each block

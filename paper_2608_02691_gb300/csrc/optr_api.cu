@@ -122,6 +122,21 @@ optr_status optr_params_create(const optr_config* cfg, const float* R_k,
   if (e == cudaSuccess) e = cudaMalloc(&p->R_vT, sizeof(float) * H * mat);
   if (e == cudaSuccess) e = cudaMalloc(&p->muR, sizeof(float) * H * kD);
   if (e == cudaSuccess) e = cudaMalloc(&p->err, sizeof(unsigned));
+  std::vector<uint32_t> frags((size_t)H * kRFragWords);
+  if (e == cudaSuccess) e = cudaMalloc(&p->Rk_tc, sizeof(uint32_t) * frags.size());
+  if (e == cudaSuccess) e = cudaMalloc(&p->Rv_tc, sizeof(uint32_t) * frags.size());
+  if (e == cudaSuccess) {
+    for (int h = 0; h < H; ++h)
+      build_rotation_fragments(R_k + h * mat, frags.data() + (size_t)h * kRFragWords);
+    e = cudaMemcpy(p->Rk_tc, frags.data(), sizeof(uint32_t) * frags.size(),
+                   cudaMemcpyHostToDevice);
+  }
+  if (e == cudaSuccess) {
+    for (int h = 0; h < H; ++h)
+      build_rotation_fragments(R_v + h * mat, frags.data() + (size_t)h * kRFragWords);
+    e = cudaMemcpy(p->Rv_tc, frags.data(), sizeof(uint32_t) * frags.size(),
+                   cudaMemcpyHostToDevice);
+  }
   if (e == cudaSuccess)
     e = cudaMemcpy(p->R_k, R_k, sizeof(float) * H * mat, cudaMemcpyHostToDevice);
   if (e == cudaSuccess)
@@ -171,12 +186,22 @@ optr_status optr_kv_append(const optr_params* p, const void* k, const void* v,
   if (!aligned(pool, 16) || !aligned(k, 16) || !aligned(v, 16))
     return OPTR_ERR_INVALID_ARG;
   if ((long long)max_pages * kPage > (1LL << 30)) return OPTR_ERR_OUT_OF_RANGE;
-  int variant = p->cfg.append_variant;
-  (void)variant;
+  const int variant = p->cfg.append_variant;
   prof_mark(p, 0, stream);
-  cudaError_t e = launch_append_cuda_core(
-      p, (const __nv_bfloat16*)k, (const __nv_bfloat16*)v, n_tok, cu_new, pos0,
-      block_table, B, max_pages, pool, num_pages, stream);
+  cudaError_t e;
+  // decode-step sized appends (<= 256 tokens) use the slice-parallel
+  // CUDA-core kernel under every variant; larger ones the tensor-core kernel
+  // unless the CUDA-core variant is requested
+  if (variant == OPTR_VARIANT_CUDA_CORE || n_tok <= 256)
+    e = launch_append_cuda_core(p, (const __nv_bfloat16*)k,
+                                (const __nv_bfloat16*)v, n_tok, cu_new, pos0,
+                                block_table, B, max_pages, pool, num_pages,
+                                stream);
+  else
+    e = launch_append_tensor(p, (const __nv_bfloat16*)k,
+                             (const __nv_bfloat16*)v, n_tok, cu_new, pos0,
+                             block_table, B, max_pages, pool, num_pages,
+                             stream);
   prof_mark(p, 1, stream);
   if (p->prof) const_cast<optr_params*>(p)->ran[0] = 1;
   return cuda_status(e);
