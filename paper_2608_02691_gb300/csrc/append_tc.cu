@@ -235,13 +235,9 @@ cudaError_t launch_append_tensor(const optr_params* p, const __nv_bfloat16* k,
                                  const int32_t* bt, int B, int max_pages,
                                  uint8_t* pool, int num_pages, cudaStream_t s) {
   const int smem = kRFragWords * 4;  // 64 KB of B fragments
-  static bool attr_set = false;      // per process; the attribute is per function
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(
-        append_tensor_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    if (e != cudaSuccess) return e;
-    attr_set = true;
-  }
+  cudaError_t e = ensure_dynamic_smem(
+      reinterpret_cast<const void*>(&append_tensor_kernel), smem);
+  if (e != cudaSuccess) return e;
   const int h_kv = p->cfg.h_kv;
   const int tiles = (n_tok + kTile - 1) / kTile;
   int per_hk = max(1, (2 * p->num_sms) / (2 * h_kv));

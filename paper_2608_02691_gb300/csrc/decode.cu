@@ -32,13 +32,15 @@ qrot_kernel(const __nv_bfloat16* __restrict__ q, const float* __restrict__ R_k,
             int B, int h_q, int h_kv, float qscale,
             const int32_t* __restrict__ seq_lens, int max_pages,
             float* __restrict__ qf, float* __restrict__ qs,
-            uint32_t* __restrict__ frag, float* __restrict__ invs,
-            int* __restrict__ pref, int* __restrict__ nzpref, unsigned* err) {
+            uint32_t* __restrict__ frag, float* __restrict__ koff,
+            float* __restrict__ invs, int* __restrict__ pref,
+            int* __restrict__ nzpref, unsigned* err) {
   __shared__ float qsm[4][kD];
   __shared__ float part[4][4][kD];  // [slice][head][channel]
   __shared__ float qrs[4][kD];
   __shared__ float hmax[4][4];
   __shared__ int warp_tot[2][kQrotThreads / 32];
+  __shared__ double koff_part[kQrotThreads / 32][kGroups];
   const int b = blockIdx.x, h = blockIdx.y, tid = threadIdx.x;
   const int sl = tid >> 7, j = tid & 127;
   const int warp = tid >> 5, lane = tid & 31;
@@ -80,7 +82,12 @@ qrot_kernel(const __nv_bfloat16* __restrict__ q, const float* __restrict__ R_k,
   __syncthreads();
   // Tensor-core B fragments (see decode_tc.cu): per head a power-of-two
   // prescale 2^e brings max |q'| * 2^e into [2^13, 2^14), so that the fp16
-  // hi/lo split stays in the normal range for all but tiny elements.
+  // hi/lo split stays in the normal range for all but tiny elements.  The
+  // key codes enter the MMA as 1024 + code * 2^pos (pos = kCodePos[G&1][r]),
+  // so the fragment of channel 32G + 4w + r also carries 2^-pos, and koff
+  // holds the offset sum 1024 * sum over the group of the fragment values,
+  // per (query head, group, hi/lo column), which the MMA starts from
+  // (negated) so that the accumulator sums code * q' exactly as before.
   {
     const int ridx = tid;  // 512 fragment registers, one per thread
     const int L = ridx >> 4, reg = ridx & 15;
@@ -90,8 +97,9 @@ qrot_kernel(const __nv_bfloat16* __restrict__ q, const float* __restrict__ R_k,
     const float mx = fmaxf(fmaxf(hmax[head][0], hmax[head][1]),
                            fmaxf(hmax[head][2], hmax[head][3]));
     const int e = max(-100, min(100, mx > 0.f ? 13 - ilogbf(mx) : 0));
-    const int ch = 32 * G + 8 * c + 2 * kk + which;   // low half; +4 high
-    const float sc = ldexpf(1.f, e);
+    const int r = 2 * kk + which;
+    const int ch = 32 * G + 8 * c + r;   // low half; +4 high
+    const float sc = ldexpf(1.f, e - code_pos(G, r));
     const float x0 = qrs[head][ch] * sc, x1 = qrs[head][ch + 4] * sc;
     const __half h0 = __float2half_rn(x0), h1 = __float2half_rn(x1);
     __half v0 = h0, v1 = h1;
@@ -101,6 +109,20 @@ qrot_kernel(const __nv_bfloat16* __restrict__ q, const float* __restrict__ R_k,
     }
     frag[((size_t)b * h_kv + h) * 512 + ridx] =
         (uint32_t)__half_as_ushort(v0) | ((uint32_t)__half_as_ushort(v1) << 16);
+    // offset sum over the 32 channels of group G for column g: reduce over
+    // (kk, which) = lane bits 0-1, c bit 0 = lane bit 4, c bit 1 = warp bit 0
+    double t = (double)__half2float(v0) + (double)__half2float(v1);
+    t += __shfl_xor_sync(0xffffffffu, t, 1);
+    t += __shfl_xor_sync(0xffffffffu, t, 2);
+    t += __shfl_xor_sync(0xffffffffu, t, 16);
+    if ((lane & 15) % 4 == 0) koff_part[warp][G] = t;
+    __syncthreads();
+    if (tid < 32) {  // tid = (g, G): koff[head][G][hl] for column g
+      const int gg = tid >> 2, GG = tid & 3;
+      const double tot = koff_part[2 * gg][GG] + koff_part[2 * gg + 1][GG];
+      koff[((size_t)b * h_kv + h) * 32 + (gg >> 1) * 8 + GG * 2 + (gg & 1)] =
+          (float)(1024.0 * tot);
+    }
     if (ridx < 4) {
       const float m2 = fmaxf(fmaxf(hmax[ridx][0], hmax[ridx][1]),
                              fmaxf(hmax[ridx][2], hmax[ridx][3]));
@@ -452,10 +474,10 @@ combine_kernel(const float* __restrict__ part, const int* __restrict__ pref,
 cudaError_t launch_partial_tensor(const optr_params* p, const uint8_t* pool,
                                   const int32_t* bt, const int32_t* seq_lens,
                                   int B, int max_pages, int num_pages,
-                                  const uint32_t* frag, const float* invs,
-                                  const float* qs, const int* pref,
-                                  const int* nzpref, float* part, int W,
-                                  cudaStream_t s);
+                                  const uint32_t* frag, const float* koff,
+                                  const float* invs, const float* qs,
+                                  const int* pref, const int* nzpref,
+                                  float* part, int W, cudaStream_t s);
 
 cudaError_t launch_decode(const optr_params* p, int variant,
                           const __nv_bfloat16* q, const int32_t* bt,
@@ -466,6 +488,7 @@ cudaError_t launch_decode(const optr_params* p, int variant,
   float* qf = reinterpret_cast<float*>(w + plan.off_qf);
   float* qs = reinterpret_cast<float*>(w + plan.off_qs);
   uint32_t* frag = reinterpret_cast<uint32_t*>(w + plan.off_frag);
+  float* koff = reinterpret_cast<float*>(w + plan.off_koff);
   float* invs = reinterpret_cast<float*>(w + plan.off_invs);
   int* pref = reinterpret_cast<int*>(w + plan.off_pref);
   int* nzpref = pref + (B + 1);
@@ -476,13 +499,14 @@ cudaError_t launch_decode(const optr_params* p, int variant,
   prof_mark(p, 2, s);
   qrot_kernel<<<dim3(B, h_kv), kQrotThreads, 0, s>>>(q, p->R_k, B, h_q, h_kv, qscale,
                                             seq_lens, max_pages, qf, qs, frag,
-                                            invs, pref, nzpref, p->err);
+                                            koff, invs, pref, nzpref, p->err);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   prof_mark(p, 3, s);
   if (variant != OPTR_VARIANT_CUDA_CORE) {
     e = launch_partial_tensor(p, pool, bt, seq_lens, B, max_pages, num_pages,
-                              frag, invs, qs, pref, nzpref, part, plan.W, s);
+                              frag, koff, invs, qs, pref, nzpref, part, plan.W,
+                              s);
   } else {
     partial_cuda_core_kernel<<<plan.W / 4, 128, 0, s>>>(
         pool, bt, seq_lens, B, max_pages, num_pages, h_q, h_kv, qf, qs, pref,
@@ -492,12 +516,9 @@ cudaError_t launch_decode(const optr_params* p, int variant,
   if (e != cudaSuccess) return e;
   prof_mark(p, 4, s);
   const size_t wts_bytes = sizeof(float) * 4 * (plan.W + 1);
-  if (wts_bytes > 48 * 1024) {
-    e = cudaFuncSetAttribute(combine_kernel,
-                             cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)wts_bytes);
-    if (e != cudaSuccess) return e;
-  }
+  e = ensure_dynamic_smem(reinterpret_cast<const void*>(&combine_kernel),
+                          wts_bytes);
+  if (e != cudaSuccess) return e;
   combine_kernel<<<dim3(B, h_kv), kCombineThreads,
                    wts_bytes, s>>>(part, pref, nzpref,
                                                           B, h_q, h_kv, plan.W,

@@ -37,6 +37,17 @@ __device__ __forceinline__ Segment locate_segment(long long f, long long f1,
   return s;
 }
 
+// Key-side code position for the tensor-core decode.  Within a 16-bit half
+// holding the code bytes of groups (2j, 2j+1) of one word w (low byte group
+// 2j), code r of the even group sits at bit 2r and of the odd group at bit
+// 8 + 2r.  The tensor kernel moves every field, with at most one shift of
+// the 32-bit word (left by 4 or right by 6), to bit 4, 6 or 8 of its half:
+// even group r = 0, 1 from (word << 4), r = 2, 3 in place; odd group r = 0 in
+// place, r = 1, 2, 3 from (word >> 6).  This is that final bit position.
+__host__ __device__ constexpr int code_pos(int G, int r) {
+  return (G & 1) ? (r == 0 ? 8 : 2 + 2 * r) : 4 + 2 * (r & 1);
+}
+
 // Warp w owns flat indices [floor(w*F/W), floor((w+1)*F/W)).  The warp that
 // owns index f (0 <= f < F) is floor(((f+1)*W - 1) / F).
 __device__ __forceinline__ int warp_of(long long f, long long F, int W) {

@@ -12,19 +12,27 @@
 //            per 32-channel group, then l = sum_g scale_g * S_g
 //            + sum_g min_g * sum(q' over group g)      (Sec. 3 Eq. 1 on the
 //            dequantized rotated key, Appendix "Rotated-query implementation")
-//   values   O[ch][n] += code[ch][tok] * (p[tok] * scale_g[tok])_{hi,lo}, plus
-//            sum_tok p * min_g[tok] per group              (Sec. 3 Eq. 2)
+//   values   O[ch][n] += (code[ch][tok] - 1.5) * (p[tok] * scale_g[tok])_{hi,lo},
+//            plus sum_tok p * (min_g + 1.5 scale_g)[tok] per group
+//                                                          (Sec. 3 Eq. 2)
 //
-// The 2-bit codes enter the MMA as exact normal fp16 integers 0..3: one LOP3
-// masks the code field at bit 2r of each 16-bit half and ORs in the exponent
-// of 1024, giving the half 1024 + code * 4^r, and one HFMA2 maps it to
-// (x - 1024) * 4^-r = code exactly.  (Raw masked fields would be fp16
-// subnormals; the MMA keeps only ~17 bits below its largest product for
-// subnormal A operands, against ~21 for normal ones, and the value-side sum
-// sum_tok p*scale*code nearly cancels against sum_tok p*min, so that loss
-// would show in the output.)  q' and p*scale are split into fp16 hi + lo
-// parts, which fill the 8 MMA columns and keep ~22 bits of the float32
-// operands.
+// The 2-bit codes enter the MMA as normal fp16 values.  One LOP3 masks a
+// code field and ORs in the exponent of 1024, giving 1024 + code * 2^pos;
+// every field is first moved to bit pos = 4, 6 or 8 of its 16-bit half by at
+// most one shift of the 32-bit word (code_pos), so that the offset 1024 is at
+// most 64x the code's weight.  Raw masked fields would be fp16 subnormals,
+// and the MMA keeps only ~17 bits below its largest product for subnormal A
+// operands, against ~21 for normal ones.
+//   keys    the LOP3 result goes to the MMA as is: the query fragment of that
+//           channel carries 2^-pos, and the MMA starts from minus the group's
+//           offset sum 1024 * sum(fragment), leaving sum code * q'.
+//   values  one HFMA2 maps it to the exact centered code - 1.5, and the min
+//           term carries min + 1.5 * scale.  Centering keeps the tensor-core
+//           accumulator o' a random walk over the pages instead of a sum that
+//           grows with the context and cancels against the min term, so its
+//           rounding error grows far more slowly with the pages per warp.
+// q' and p*scale are split into fp16 hi + lo parts, which fill the 8 MMA
+// columns and keep ~22 bits of the float32 operands.
 #include <type_traits>
 
 #include "decode_common.cuh"
@@ -54,6 +62,18 @@ __device__ __forceinline__ void mma16816(float* d, uint32_t a0, uint32_t a1,
       : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
 
+// d = a * b + (c0, c1, c0, c1): the first MMA of a chain, started from a
+// per-column value instead of the accumulator.
+__device__ __forceinline__ void mma16816_c(float* d, uint32_t a0, uint32_t a1,
+                                           uint32_t a2, uint32_t a3, uint32_t b0,
+                                           uint32_t b1, float c0, float c1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 "
+      "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%10,%11,%10,%11};\n"
+      : "=f"(d[0]), "=f"(d[1]), "=f"(d[2]), "=f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1), "f"(c0), "f"(c1));
+}
+
 __device__ __forceinline__ void ldsm_x4_trans(uint32_t& r0, uint32_t& r1,
                                               uint32_t& r2, uint32_t& r3,
                                               const void* smem_row) {
@@ -64,16 +84,40 @@ __device__ __forceinline__ void ldsm_x4_trans(uint32_t& r0, uint32_t& r1,
       : "r"(a));
 }
 
-// Two codes (the fields at bit 2r of each 16-bit half of src) as exact
-// fp16 values 0..3.  exp1024 holds 0x64006400 (the exponent of 1024 in both
-// halves) in a register, so that mask-and-or is a single LOP3.
-template <int r>
-__device__ __forceinline__ uint32_t codes_f16x2(uint32_t src, uint32_t exp1024) {
+// The two code fields at bit pos of each 16-bit half of src as fp16
+// 1024 + code * 2^pos (pos <= 8 keeps the field inside the mantissa).
+template <int pos>
+__device__ __forceinline__ uint32_t field_f16x2(uint32_t src, uint32_t exp1024) {
   uint32_t x;
   asm("lop3.b32 %0, %1, %2, %3, 0xEA;"  // (a & b) | c
-      : "=r"(x) : "r"(src), "n"(0x00030003u << (2 * r)), "r"(exp1024));
-  const __half2 sc = __float2half2_rn(1.0f / (float)(1 << (2 * r)));
-  const __half2 bias = __float2half2_rn(-1024.0f / (float)(1 << (2 * r)));
+      : "=r"(x) : "r"(src), "n"(0x00030003u << pos), "r"(exp1024));
+  return x;
+}
+
+// The 16 code fields of a word y whose 16-bit halves each hold one byte of
+// group 2j (low byte) and one of group 2j+1 (high byte), as MMA A registers
+// out[parity][r] = fp16 1024 + code * 2^pos, pos = code_pos(parity, r).
+__device__ __forceinline__ void code_fields(uint32_t y, uint32_t e1024,
+                                           uint32_t (&out)[2][4]) {
+  const uint32_t yl = y << 4, yr = y >> 6;
+  out[0][0] = field_f16x2<code_pos(0, 0)>(yl, e1024);
+  out[0][1] = field_f16x2<code_pos(0, 1)>(yl, e1024);
+  out[0][2] = field_f16x2<code_pos(0, 2)>(y, e1024);
+  out[0][3] = field_f16x2<code_pos(0, 3)>(y, e1024);
+  out[1][0] = field_f16x2<code_pos(1, 0)>(y, e1024);
+  out[1][1] = field_f16x2<code_pos(1, 1)>(yr, e1024);
+  out[1][2] = field_f16x2<code_pos(1, 2)>(yr, e1024);
+  out[1][3] = field_f16x2<code_pos(1, 3)>(yr, e1024);
+}
+
+// A field from code_fields() of group parity par and code index r
+// (1024 + code * 2^pos) mapped by one HFMA2 to the exact centered code
+// code - 1.5 in {-1.5, -0.5, 0.5, 1.5}: x * 2^-pos - (1024 * 2^-pos + 1.5).
+// Both constants are exact fp16 values for pos = 4, 6, 8.
+__device__ __forceinline__ uint32_t centered(uint32_t x, int par, int r) {
+  const int pos = code_pos(par, r);
+  const __half2 sc = __float2half2_rn(1.0f / (float)(1 << pos));
+  const __half2 bias = __float2half2_rn(-1024.0f / (float)(1 << pos) - 1.5f);
   const __half2 y = __hfma2(*reinterpret_cast<const __half2*>(&x), sc, bias);
   return *reinterpret_cast<const uint32_t*>(&y);
 }
@@ -151,6 +195,7 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
                       const int32_t* __restrict__ seq_lens, int B,
                       int max_pages, int num_pages, int h_q, int h_kv,
                       const uint32_t* __restrict__ frag,
+                      const float* __restrict__ koff,
                       const float* __restrict__ invs,
                       const float* __restrict__ qs,
                       const int* __restrict__ pref,
@@ -207,6 +252,7 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
 
   // per-segment state
   uint32_t bq[kGroups][2][2];  // query B fragments [group][kk][reg]
+  float kneg[kGroups][2];      // minus the key-code offset sums, head c
   float qsum[kGroups];         // sum of q' over each group, head c
   float inv_s = 0.f;           // 1 / prescale of head c
   float acc_o[kGroups][2][4];  // values: [group][half][c-frag]
@@ -257,6 +303,15 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
       bq[G][1][0] = v.z;
       bq[G][1][1] = v.w;
     }
+    {
+      const float4* ko = reinterpret_cast<const float4*>(
+          koff + ((size_t)cb * h_kv + ch) * 32 + c * 8);
+      const float4 k01 = __ldg(ko), k23 = __ldg(ko + 1);
+      kneg[0][0] = -k01.x; kneg[0][1] = -k01.y;
+      kneg[1][0] = -k01.z; kneg[1][1] = -k01.w;
+      kneg[2][0] = -k23.x; kneg[2][1] = -k23.y;
+      kneg[3][0] = -k23.z; kneg[3][1] = -k23.w;
+    }
     const size_t row = (size_t)cb * h_q + 4 * ch + c;
     const float4 q4 = __ldg(reinterpret_cast<const float4*>(qs + row * kGroups));
     qsum[0] = q4.x;
@@ -293,17 +348,18 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
       const uint32_t y23_1 = __byte_perm(k1.x, k1.y, 0x7632);
       float s_acc[kGroups][4];
 #pragma unroll
-      for (int G = 0; G < kGroups; ++G) {
-        const uint32_t src0 = (G < 2 ? y01_0 : y23_0) >> (8 * (G & 1));
-        const uint32_t src1 = (G < 2 ? y01_1 : y23_1) >> (8 * (G & 1));
+      for (int j = 0; j < 2; ++j) {  // groups 2j, 2j+1
+        uint32_t f0[2][4], f1[2][4];  // token rows g, g+8
+        code_fields(j ? y23_0 : y01_0, e1024, f0);
+        code_fields(j ? y23_1 : y01_1, e1024, f1);
 #pragma unroll
-        for (int k = 0; k < 4; ++k) s_acc[G][k] = 0.f;
-        mma16816(s_acc[G], codes_f16x2<0>(src0, e1024), codes_f16x2<0>(src1, e1024),
-                 codes_f16x2<1>(src0, e1024), codes_f16x2<1>(src1, e1024), bq[G][0][0],
-                 bq[G][0][1]);
-        mma16816(s_acc[G], codes_f16x2<2>(src0, e1024), codes_f16x2<2>(src1, e1024),
-                 codes_f16x2<3>(src0, e1024), codes_f16x2<3>(src1, e1024), bq[G][1][0],
-                 bq[G][1][1]);
+        for (int par = 0; par < 2; ++par) {
+          const int G = 2 * j + par;
+          mma16816_c(s_acc[G], f0[par][0], f1[par][0], f0[par][1], f1[par][1],
+                     bq[G][0][0], bq[G][0][1], kneg[G][0], kneg[G][1]);
+          mma16816(s_acc[G], f0[par][2], f1[par][2], f0[par][3], f1[par][3],
+                   bq[G][1][0], bq[G][1][1]);
+        }
       }
       const uint4 km0 = *reinterpret_cast<const uint4*>(st + OPTR_K_META_OFFSET + g * 16);
       const uint4 km1 = *reinterpret_cast<const uint4*>(st + OPTR_K_META_OFFSET + (g + 8) * 16);
@@ -374,9 +430,12 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
           a = v0 ? a : make_float2(0.f, 0.f);
           bb = v1 ? bb : make_float2(0.f, 0.f);
         }
-        mv[G] = fmaf(p0, a.y, fmaf(p1, bb.y, mv[G]));
-        S.pt[G][g][c] = split_hilo(p0 * a.x);
-        S.pt[G][g + 8][c] = split_hilo(p1 * bb.x);
+        // the MMA sees centered codes (code - 1.5): the min term carries
+        // min + 1.5 * scale
+        const float ps0 = p0 * a.x, ps1 = p1 * bb.x;
+        mv[G] = fmaf(1.5f, ps0, fmaf(p0, a.y, fmaf(1.5f, ps1, fmaf(p1, bb.y, mv[G]))));
+        S.pt[G][g][c] = split_hilo(ps0);
+        S.pt[G][g + 8][c] = split_hilo(ps1);
       }
     }
     __syncwarp();
@@ -397,13 +456,20 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
       const uint32_t a01 = __byte_perm(x0, x1, 0x5410), a23 = __byte_perm(x0, x1, 0x7632);
       const uint32_t b01 = __byte_perm(x2, x3, 0x5410), b23 = __byte_perm(x2, x3, 0x7632);
 #pragma unroll
-      for (int G = 0; G < kGroups; ++G) {
-        const uint32_t sa = (G < 2 ? a01 : a23) >> (8 * (G & 1));
-        const uint32_t sb = (G < 2 ? b01 : b23) >> (8 * (G & 1));
-        mma16816(acc_o[G][0], codes_f16x2<0>(sa, e1024), codes_f16x2<1>(sa, e1024),
-                 codes_f16x2<0>(sb, e1024), codes_f16x2<1>(sb, e1024), bv[G][0], bv[G][1]);
-        mma16816(acc_o[G][1], codes_f16x2<2>(sa, e1024), codes_f16x2<3>(sa, e1024),
-                 codes_f16x2<2>(sb, e1024), codes_f16x2<3>(sb, e1024), bv[G][0], bv[G][1]);
+      for (int j = 0; j < 2; ++j) {  // groups 2j, 2j+1
+        uint32_t fa[2][4], fb[2][4];  // tokens (2c, 2c+1), (2c+8, 2c+9)
+        code_fields(j ? a23 : a01, e1024, fa);
+        code_fields(j ? b23 : b01, e1024, fb);
+#pragma unroll
+        for (int par = 0; par < 2; ++par) {
+          const int G = 2 * j + par;
+          mma16816(acc_o[G][0], centered(fa[par][0], par, 0), centered(fa[par][1], par, 1),
+                   centered(fb[par][0], par, 0), centered(fb[par][1], par, 1),
+                   bv[G][0], bv[G][1]);
+          mma16816(acc_o[G][1], centered(fa[par][2], par, 2), centered(fa[par][3], par, 3),
+                   centered(fb[par][2], par, 2), centered(fb[par][3], par, 3),
+                   bv[G][0], bv[G][1]);
+        }
       }
     }
   };
@@ -411,7 +477,7 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
   const int total = f1 - f0;
   int done = 0;
   while (done < total) {
-#pragma unroll
+#pragma unroll 1
     for (int s = 0; s < kStages; ++s) {
       if (done < total) {
         issue((s + kStages - 1) % kStages);
@@ -440,13 +506,13 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
 cudaError_t launch_partial_tensor(const optr_params* p, const uint8_t* pool,
                                   const int32_t* bt, const int32_t* seq_lens,
                                   int B, int max_pages, int num_pages,
-                                  const uint32_t* frag, const float* invs,
-                                  const float* qs, const int* pref,
-                                  const int* nzpref, float* part, int W,
-                                  cudaStream_t s) {
+                                  const uint32_t* frag, const float* koff,
+                                  const float* invs, const float* qs,
+                                  const int* pref, const int* nzpref,
+                                  float* part, int W, cudaStream_t s) {
   partial_tensor_kernel<<<W / kWarps, kWarps * 32, 0, s>>>(
       pool, bt, seq_lens, B, max_pages, num_pages, p->cfg.h_q, p->cfg.h_kv,
-      frag, invs, qs, pref, nzpref, part, W, p->err);
+      frag, koff, invs, qs, pref, nzpref, part, W, p->err);
   return cudaGetLastError();
 }
 

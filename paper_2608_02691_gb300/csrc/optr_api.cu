@@ -6,6 +6,7 @@
 #include <stdlib.h>
 #include <string.h>
 
+#include <mutex>
 #include <vector>
 
 #include "optr_internal.cuh"
@@ -28,10 +29,38 @@ size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 namespace optr {
 
+cudaError_t ensure_dynamic_smem(const void* kernel, size_t bytes) {
+  struct Entry {
+    const void* kernel;
+    int device;
+    size_t bytes;
+  };
+  static std::mutex mu;
+  static std::vector<Entry> done;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  std::lock_guard<std::mutex> lock(mu);
+  Entry* hit = nullptr;
+  for (Entry& x : done)
+    if (x.kernel == kernel && x.device == dev) hit = &x;
+  if (hit && hit->bytes >= bytes) return cudaSuccess;
+  e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           (int)bytes);
+  if (e != cudaSuccess) return e;
+  if (hit)
+    hit->bytes = bytes;
+  else
+    done.push_back(Entry{kernel, dev, bytes});
+  return cudaSuccess;
+}
+
 // Workspace of one decode call (all offsets 256-byte aligned):
 //   qf   float [B][h_q][128]   rotated, pre-scaled queries
 //   qs   float [B][h_q][4]     per-group sums of qf
 //   frag u32   [B][h_kv][32][16] tensor-core B fragments of qf (hi/lo f16)
+//   koff float [B][h_kv][4][4][2] code-offset sums of the fragments
+//                               [query head][group][hi/lo] (decode_tc.cu)
 //   invs float [B][h_q]         1 / (power-of-two prescale of frag)
 //   pref int   [2][B+1]        page prefix sums / non-empty prefix counts
 //   part float [W + B*h_kv][520] split-K partials (o'[4][128], m[4], l[4])
@@ -49,6 +78,8 @@ DecodePlan decode_plan(const optr_params* p, int B, int max_pages) {
   o = round_up(o + sizeof(float) * (size_t)B * d.h_q * kGroups, 256);
   d.off_frag = o;
   o = round_up(o + sizeof(uint32_t) * (size_t)B * d.h_kv * 32 * 16, 256);
+  d.off_koff = o;
+  o = round_up(o + sizeof(float) * (size_t)B * d.h_kv * 32, 256);
   d.off_invs = o;
   o = round_up(o + sizeof(float) * (size_t)B * d.h_q, 256);
   d.off_pref = o;

@@ -44,6 +44,12 @@ struct optr_params {
 };
 
 namespace optr {
+// Raise a kernel's dynamic shared memory limit on the current device to at
+// least `bytes` (static plus dynamic shared memory may exceed 48 KB only
+// after this opt-in).  Cached per (kernel, device) under a lock, so the
+// runtime call is made once per new maximum.
+cudaError_t ensure_dynamic_smem(const void* kernel, size_t bytes);
+
 // Record stage event i on stream s when profiling is on.
 inline void prof_mark(const optr_params* p, int i, cudaStream_t s) {
   if (p->prof) cudaEventRecord(p->ev[i], s);
@@ -55,7 +61,7 @@ namespace optr {
 // Byte offsets of the decode workspace for a batch shape.
 struct DecodePlan {
   int B, h_q, h_kv, max_pages, W;  // W = partial-kernel warps
-  size_t off_qf, off_qs, off_frag, off_invs, off_pref, off_part, total;
+  size_t off_qf, off_qs, off_frag, off_koff, off_invs, off_pref, off_part, total;
 };
 DecodePlan decode_plan(const optr_params* p, int B, int max_pages);
 
