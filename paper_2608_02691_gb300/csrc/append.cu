@@ -32,6 +32,8 @@ append_cuda_core_kernel(const __nv_bfloat16* __restrict__ k,
   const int h = blockIdx.y;
   const int t0 = blockIdx.x * T;
   const int tid = threadIdx.x;
+  pdl_wait();
+  pdl_trigger();
 
   for (int idx = tid; idx < 2 * T * kD; idx += blockDim.x) {
     int kind = idx / (T * kD);
@@ -107,6 +109,7 @@ append_cuda_core_kernel(const __nv_bfloat16* __restrict__ k,
 // tokens; the slices are added in shared memory, then warp t quantizes and
 // packs token t group by group.
 constexpr int kSmallTok = 16;
+constexpr int kSmallCuCache = 512;   // sequences whose cu_new / pos0 a CTA caches
 
 __global__ void __launch_bounds__(512)
 append_small_kernel(const __nv_bfloat16* __restrict__ k,
@@ -124,30 +127,49 @@ append_small_kernel(const __nv_bfloat16* __restrict__ k,
   __shared__ float zp[4][T][kD];
   __shared__ long long dst[T];
   __shared__ int dslot[T];
+  __shared__ int s_cu[kSmallCuCache + 1];
+  __shared__ int s_p0[kSmallCuCache];
   const int h = blockIdx.y, kind = blockIdx.z;
   const int t0 = blockIdx.x * T;
   const int tid = threadIdx.x;
+  const int sl = tid >> 7, j = tid & 127;
+  // rotation column first (independent of everything else): all in flight
+  const float* R = (kind ? R_v : R_k) + (size_t)h * kD * kD + (size_t)(32 * sl) * kD + j;
+  float rv[32];
+#pragma unroll
+  for (int i = 0; i < 32; ++i) rv[i] = __ldg(R + i * kD);
+  float musub[kGroups];  // mu R_k of this lane's channel in each group (keys)
+#pragma unroll
+  for (int g = 0; g < kGroups; ++g)
+    musub[g] = kind ? 0.f : __ldg(muR + h * kD + 32 * g + (tid & 31));
+  pdl_wait();  // inputs and the pool may come from earlier kernels
+  pdl_trigger();
   const __nv_bfloat16* src = kind ? v : k;
   for (int idx = tid; idx < T * kD; idx += 512) {
     const int t = idx >> 7, i = idx & 127;
     const int tok = t0 + t;
     xs[t][i] = tok < n_tok ? __bfloat162float(src[((size_t)tok * h_kv + h) * kD + i]) : 0.f;
   }
+  const bool cached = B <= kSmallCuCache;
+  if (cached) {
+    for (int i = tid; i <= B; i += 512) {
+      s_cu[i] = __ldg(cu_new + i);
+      if (i < B) s_p0[i] = __ldg(pos0 + i);
+    }
+    __syncthreads();
+  }
   if (tid < T) {
     const int tok = t0 + tid;
     int slot = 0;
     long long off = -1;
     if (tok < n_tok)
-      off = resolve_slot(tok, h, cu_new, pos0, bt, B, max_pages, num_pages,
-                         h_kv, &slot, err);
+      off = cached ? resolve_slot_cached(tok, h, s_cu, s_p0, bt, B, max_pages,
+                                         num_pages, h_kv, &slot, err)
+                   : resolve_slot(tok, h, cu_new, pos0, bt, B, max_pages,
+                                  num_pages, h_kv, &slot, err);
     dst[tid] = off;
     dslot[tid] = slot;
   }
-  const int sl = tid >> 7, j = tid & 127;
-  const float* R = (kind ? R_v : R_k) + (size_t)h * kD * kD + (size_t)(32 * sl) * kD + j;
-  float rv[32];
-#pragma unroll
-  for (int i = 0; i < 32; ++i) rv[i] = __ldg(R + i * kD);  // all in flight
   __syncthreads();
   float acc[T];
 #pragma unroll
@@ -172,7 +194,7 @@ append_small_kernel(const __nv_bfloat16* __restrict__ k,
   for (int g = 0; g < kGroups; ++g) {
     const int jj = 32 * g + lane;
     const float zsum = ((zp[0][warp][jj] + zp[1][warp][jj]) + zp[2][warp][jj]) + zp[3][warp][jj];
-    const float z = __fsub_rn(zsum, kind ? 0.f : __ldg(muR + h * kD + jj));
+    const float z = __fsub_rn(zsum, musub[g]);
     float lo = z, hi = z;
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
@@ -203,19 +225,18 @@ cudaError_t launch_append_cuda_core(const optr_params* p,
   // few tokens (decode steps): slice-parallel rotation
   if (n_tok <= 256) {
     dim3 grid((n_tok + kSmallTok - 1) / kSmallTok, p->cfg.h_kv, 2);
-    append_small_kernel<<<grid, 512, 0, s>>>(
-        k, v, n_tok, cu_new, pos0, bt, B, max_pages, pool, num_pages,
-        p->cfg.h_kv, p->R_k, p->R_v, p->muR, p->cfg.clip_k, p->cfg.clip_v,
-        p->err);
+    return launch_pdl(append_small_kernel, grid, dim3(512), 0, s, k, v, n_tok,
+                      cu_new, pos0, bt, B, max_pages, pool, num_pages,
+                      p->cfg.h_kv, p->R_k, p->R_v, p->muR, p->cfg.clip_k,
+                      p->cfg.clip_v, p->err);
   } else {
     constexpr int T = 32;
     dim3 grid((n_tok + T - 1) / T, p->cfg.h_kv);
-    append_cuda_core_kernel<T><<<grid, 256, 0, s>>>(
-        k, v, n_tok, cu_new, pos0, bt, B, max_pages, pool, num_pages,
-        p->cfg.h_kv, p->R_k, p->R_v, p->muR, p->cfg.clip_k, p->cfg.clip_v,
-        p->err);
+    return launch_pdl(append_cuda_core_kernel<T>, grid, dim3(256), 0, s, k, v,
+                      n_tok, cu_new, pos0, bt, B, max_pages, pool, num_pages,
+                      p->cfg.h_kv, p->R_k, p->R_v, p->muR, p->cfg.clip_k,
+                      p->cfg.clip_v, p->err);
   }
-  return cudaGetLastError();
 }
 
 }  // namespace optr

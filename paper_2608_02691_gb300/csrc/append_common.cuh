@@ -44,4 +44,36 @@ __device__ __forceinline__ long long resolve_slot(int tok, int h, const int32_t*
   return ((long long)page * h_kv + h) * kChunk;
 }
 
+// resolve_slot() with cu_new[0..B] and pos0[0..B-1] already in shared
+// memory (cu and p0 point there); only the block-table entry is read from
+// global memory.
+__device__ __forceinline__ long long resolve_slot_cached(
+    int tok, int h, const int* cu, const int* p0,
+    const int32_t* __restrict__ bt, int B, int max_pages, int num_pages,
+    int h_kv, int* slot, unsigned* err) {
+  int lo = 0, hi = B;
+  while (hi - lo > 1) {
+    const int mid = (lo + hi) >> 1;
+    if (cu[mid] <= tok) lo = mid; else hi = mid;
+  }
+  const int b = lo;
+  const int c0 = cu[b], c1 = cu[b + 1];
+  if (!(c0 <= tok && tok < c1)) {
+    atomicOr(err, OPTR_DEVERR_CU_NEW);
+    return -1;
+  }
+  const long long pos = (long long)p0[b] + (tok - c0);
+  if (pos < 0 || pos >= (long long)max_pages * kPage) {
+    atomicOr(err, OPTR_DEVERR_POSITION);
+    return -1;
+  }
+  const int page = __ldg(bt + (size_t)b * max_pages + pos / kPage);
+  if (page < 0 || page >= num_pages) {
+    atomicOr(err, OPTR_DEVERR_PAGE_ID);
+    return -1;
+  }
+  *slot = (int)(pos % kPage);
+  return ((long long)page * h_kv + h) * kChunk;
+}
+
 }  // namespace optr

@@ -129,6 +129,8 @@ append_tensor_kernel(const __nv_bfloat16* __restrict__ k,
       cp_async16_zfill(&bfrag[i], &src[i], true);
     cp_async_commit();
     smu[tid] = kind ? 0.f : __ldg(muR + h * kD + tid);
+    pdl_wait();  // inputs and the pool may come from earlier kernels
+    pdl_trigger();
     cp_async_wait<0>();
     __syncthreads();
   }
@@ -243,10 +245,10 @@ cudaError_t launch_append_tensor(const optr_params* p, const __nv_bfloat16* k,
   int per_hk = max(1, (2 * p->num_sms) / (2 * h_kv));
   per_hk = min(per_hk, (tiles + kAppendWarps - 1) / kAppendWarps);
   dim3 grid(per_hk, h_kv, 2);
-  append_tensor_kernel<<<grid, kAppendWarps * 32, smem, s>>>(
-      k, v, n_tok, cu_new, pos0, bt, B, max_pages, pool, num_pages, h_kv,
-      p->Rk_tc, p->Rv_tc, p->muR, p->cfg.clip_k, p->cfg.clip_v, p->err);
-  return cudaGetLastError();
+  return launch_pdl(append_tensor_kernel, grid, dim3(kAppendWarps * 32),
+                    (size_t)smem, s, k, v, n_tok, cu_new, pos0, bt, B,
+                    max_pages, pool, num_pages, h_kv, p->Rk_tc, p->Rv_tc,
+                    p->muR, p->cfg.clip_k, p->cfg.clip_v, p->err);
 }
 
 }  // namespace optr

@@ -34,7 +34,8 @@ qrot_kernel(const __nv_bfloat16* __restrict__ q, const float* __restrict__ R_k,
             float* __restrict__ qf, float* __restrict__ qs,
             uint32_t* __restrict__ frag, float* __restrict__ koff,
             float* __restrict__ invs, int* __restrict__ pref,
-            int* __restrict__ nzpref, unsigned* err) {
+            int* __restrict__ nzpref, int* __restrict__ cnt_ws,
+            unsigned* err) {
   __shared__ float qsm[4][kD];
   __shared__ float part[4][4][kD];  // [slice][head][channel]
   __shared__ float qrs[4][kD];
@@ -44,15 +45,18 @@ qrot_kernel(const __nv_bfloat16* __restrict__ q, const float* __restrict__ R_k,
   const int b = blockIdx.x, h = blockIdx.y, tid = threadIdx.x;
   const int sl = tid >> 7, j = tid & 127;
   const int warp = tid >> 5, lane = tid & 31;
-  {
-    const int r = tid >> 7;  // 512 threads load the 4 x 128 query values
-    qsm[r][j] = __bfloat162float(q[((size_t)b * h_q + 4 * h + r) * kD + j]);
-  }
   float acc[4] = {0.f, 0.f, 0.f, 0.f};
   const float* R = R_k + (size_t)h * kD * kD + (size_t)(32 * sl) * kD + j;
   float rv[32];
 #pragma unroll
   for (int i = 0; i < 32; ++i) rv[i] = __ldg(R + i * kD);  // all in flight
+  pdl_wait();  // the query, lengths and workspace may belong to earlier kernels
+  pdl_trigger();
+  if (tid == 0) cnt_ws[(size_t)b * h_kv + h] = 0;  // combine arrivals
+  {
+    const int r = tid >> 7;  // 512 threads load the 4 x 128 query values
+    qsm[r][j] = __bfloat162float(q[((size_t)b * h_q + 4 * h + r) * kD + j]);
+  }
   __syncthreads();
 #pragma unroll
   for (int i = 0; i < 32; ++i)
@@ -184,10 +188,12 @@ partial_cuda_core_kernel(const uint8_t* __restrict__ pool,
                          const int* __restrict__ nzpref,
                          float* __restrict__ part, int W, unsigned* err) {
   __shared__ WarpSmemCC smem[4];
+  pdl_wait();
+  pdl_trigger();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   WarpSmemCC& S = smem[warp];
   const int w = blockIdx.x * 4 + warp;
-  const long long F = (long long)__ldg(pref + B) * h_kv;
+  const long long F = (long long)__ldcg(pref + B) * h_kv;
   long long f = w * F / W;
   const long long f1 = (w + 1) * F / W;
 
@@ -197,9 +203,9 @@ partial_cuda_core_kernel(const uint8_t* __restrict__ pool,
     const int len = __ldg(seq_lens + b);
     // rotated queries of the GQA group
     for (int i = lane; i < 4 * kD; i += 32)
-      S.qv[i / kD][i % kD] = __ldg(qf + ((size_t)b * h_q + 4 * h) * kD + i);
+      S.qv[i / kD][i % kD] = __ldcg(qf + ((size_t)b * h_q + 4 * h) * kD + i);
     if (lane < 16)
-      S.qsum[lane / 4][lane % 4] = __ldg(qs + ((size_t)b * h_q + 4 * h) * kGroups + lane);
+      S.qsum[lane / 4][lane % 4] = __ldcg(qs + ((size_t)b * h_q + 4 * h) * kGroups + lane);
     float m[4], l[4], acc[4][4];
 #pragma unroll
     for (int r = 0; r < 4; ++r) {
@@ -327,145 +333,226 @@ partial_cuda_core_kernel(const uint8_t* __restrict__ pool,
 
 // ------------------------------------------------------------- combine
 
-// One CTA per (sequence b, KV head h), 256 threads, all 4 query heads of
-// the group.  The merge weights exp2(m_i - M) / L of the segment partials
-// are computed once into shared memory (dynamic, (W + 1) x 4 floats); each
-// thread then merges 2 of the 512 outputs o'[head][channel], and the merged
-// o' is rotated back, out = o' R_v^T, with the 128-term sums split over the
-// two halves of the block.
-constexpr int kCombineThreads = 256;
+// Grid (B, h_kv, S), 512 threads.  CTA (b, h, s) merges chunk s of the
+// segment partials of (b, h) (log-sum-exp merge, Sec. 3 Eq. 1-2 split over
+// the context); with S = 1 it also normalises and rotates back,
+// out = o' R_v^T.  With S > 1 each CTA writes its chunk's (m, l, o') to
+// the workspace, and the last CTA of (b, h) to arrive (atomic counter,
+// zeroed by qrot) merges the S chunk results and rotates.  Before waiting
+// for the partial kernel every CTA copies this head's R_v^T (64 KB,
+// library-owned) into shared memory, so the rotation never waits on global
+// memory.  Partials are read 32 at a time: the headers and the o' float4s
+// of a batch are all requested before any is used.
+constexpr int kCombineThreads = 512;
+constexpr int kCombineBatch = 32;
+
+struct CombineState {
+  float M[4], L[4];      // running maxima / sums per query head
+  float alpha[4];        // rescale of the accumulators for the batch
+  float w[kCombineBatch][4];
+  float red[kCombineThreads / 32][4];
+};
+
+// Merge cnt (<= kCombineBatch) partials at base + i * kPartFloats into the
+// running state st and the thread's float4 accumulator acc (float4 v of
+// o'[4][128] over the partials i = ph (mod 4)).  first_w >= 0 marks partial
+// slots of warps first_w + i, which may be empty (never written) when
+// sparse; their weight is 0 and their values are never accumulated.
+__device__ __forceinline__ void combine_batch(const float* base, int cnt,
+                                              int first_w, bool sparse,
+                                              long long F, int W,
+                                              CombineState& st, float4& acc) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int v = tid & 127, ph = tid >> 7, hd = v >> 5;
+  // issue every load of the batch first
+  float m = -INFINITY, l = 0.f;
+  bool hv = false;
+  if (tid < 4 * cnt) {
+    hv = !(sparse && first_w >= 0 && warp_empty(first_w + (tid >> 2), F, W));
+    if (hv) {
+      const float* pp = base + (size_t)(tid >> 2) * kPartFloats;
+      m = __ldcg(pp + kPartM + (tid & 3));
+      l = __ldcg(pp + kPartL + (tid & 3));
+    }
+  }
+  float4 a[kCombineBatch / 4];
+#pragma unroll
+  for (int j = 0; j < kCombineBatch / 4; ++j) {
+    const int i = ph + 4 * j;
+    a[j] = i < cnt ? __ldcg(reinterpret_cast<const float4*>(base + (size_t)i * kPartFloats) + v)
+                   : make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+  // batch maximum per head (thread t's head is t & 3 == lane & 3)
+  float mx = m;
+#pragma unroll
+  for (int o = 4; o < 32; o <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+  if (lane < 4) st.red[warp][lane] = mx;
+  __syncthreads();
+  if (tid < 4) {
+    float bm = -INFINITY;
+    for (int w = 0; w < kCombineThreads / 32; ++w) bm = fmaxf(bm, st.red[w][tid]);
+    const float Mn = fmaxf(st.M[tid], bm);
+    st.alpha[tid] = merge_weight(st.M[tid], Mn);
+    st.M[tid] = Mn;
+  }
+  __syncthreads();
+  const float Mh = st.M[lane & 3];
+  float wl = 0.f;
+  if (tid < 4 * cnt) {
+    const float wgt = hv ? merge_weight(m, Mh) : 0.f;
+    st.w[tid >> 2][tid & 3] = wgt;
+    wl = l * wgt;
+  }
+#pragma unroll
+  for (int o = 4; o < 32; o <<= 1) wl += __shfl_xor_sync(0xffffffffu, wl, o);
+  if (lane < 4) st.red[warp][lane] = wl;
+  __syncthreads();
+  if (tid < 4) {
+    float sl = 0.f;
+    for (int w = 0; w < kCombineThreads / 32; ++w) sl += st.red[w][tid];
+    st.L[tid] = st.L[tid] * st.alpha[tid] + sl;
+  }
+  const float al = st.alpha[hd];
+  acc.x *= al;
+  acc.y *= al;
+  acc.z *= al;
+  acc.w *= al;
+#pragma unroll
+  for (int j = 0; j < kCombineBatch / 4; ++j) {
+    const int i = ph + 4 * j;
+    const float wv = i < cnt ? st.w[i][hd] : 0.f;
+    if (wv != 0.f) {
+      acc.x = fmaf(a[j].x, wv, acc.x);
+      acc.y = fmaf(a[j].y, wv, acc.y);
+      acc.z = fmaf(a[j].z, wv, acc.z);
+      acc.w = fmaf(a[j].w, wv, acc.w);
+    }
+  }
+  __syncthreads();  // st.w / st.red are reused by the next batch
+}
 
 __global__ void __launch_bounds__(kCombineThreads)
 combine_kernel(const float* __restrict__ part, const int* __restrict__ pref,
                const int* __restrict__ nzpref, int B, int h_q, int h_kv, int W,
-               const float* __restrict__ R_vT, float* __restrict__ out) {
-  extern __shared__ float wts[];  // [n][4]
-  __shared__ float red[kCombineThreads / 32][4];
-  __shared__ float ML[2][4];
+               const float* __restrict__ R_vT, float* __restrict__ cpart,
+               int* __restrict__ cnt_ws, float* __restrict__ out) {
+  extern __shared__ float4 dsm[];
+  float* rts = reinterpret_cast<float*>(dsm);  // [128][128] R_v^T[h]
+  __shared__ float4 msum[4][kD];               // [phase][float4 of o']
   __shared__ float orot[4][kD];
-  __shared__ float half_sum[4][kD];
-  const int b = blockIdx.x, h = blockIdx.y;
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int np = __ldg(pref + b + 1) - __ldg(pref + b);
+  __shared__ CombineState st;
+  __shared__ int last;
+  const int b = blockIdx.x, h = blockIdx.y, sp = blockIdx.z, S = gridDim.z;
+  const int tid = threadIdx.x;
+  {
+    const float4* src = reinterpret_cast<const float4*>(R_vT + (size_t)h * kD * kD);
+#pragma unroll
+    for (int u = 0; u < kD * kD / 4 / kCombineThreads; ++u)
+      cp_async16(&dsm[tid + u * kCombineThreads], src + tid + u * kCombineThreads);
+    cp_async_commit();
+  }
+  if (tid < 4) {
+    st.M[tid] = -INFINITY;
+    st.L[tid] = 0.f;
+  }
+  // The page prefix sums were written by qrot, two kernels back: the
+  // partial kernel only lets this grid launch after its own pdl_wait(),
+  // i.e. after qrot completed with its writes visible, so they are read
+  // (through L2) before waiting for the partials themselves.
+  const int np = __ldcg(pref + b + 1) - __ldcg(pref + b);
+  const long long F = (long long)__ldcg(pref + B) * h_kv;
+  const long long fs = (long long)__ldcg(pref + b) * h_kv + (long long)h * np;
+  const int nzb = __ldcg(nzpref + b);
+  int w0 = 0, n = 0;
+  if (np > 0) {
+    w0 = warp_of(fs, F, W);
+    n = warp_of(fs + np - 1, F, W) - w0 + 1;
+  }
+  const bool sparse = F < W;
+  const float* pbase = part + ((size_t)nzb * h_kv + h + w0) * kPartFloats;
+  const int i0 = sp * n / S, i1 = (sp + 1) * n / S;  // n <= W: no overflow
+  pdl_wait();
+  pdl_trigger();
   float* ob = out + ((size_t)b * h_q + 4 * h) * kD;
   if (np == 0) {
-    for (int i = tid; i < 4 * kD; i += kCombineThreads) ob[i] = 0.f;
+    if (sp == 0) ob[tid] = 0.f;
+    cp_async_wait<0>();
     return;
   }
-  const long long F = (long long)__ldg(pref + B) * h_kv;
-  const long long fs = (long long)__ldg(pref + b) * h_kv + (long long)h * np;
-  const int w0 = warp_of(fs, F, W), w1 = warp_of(fs + np - 1, F, W);
-  const int n = w1 - w0 + 1;
-  const float* pbase = part + ((size_t)__ldg(nzpref + b) * h_kv + h + w0) * kPartFloats;
-  {
-    // warm L2 with this head's R_v^T (64 KB = 512 lines) for the last phase
-    const char* rt = reinterpret_cast<const char*>(R_vT + (size_t)h * kD * kD);
-    asm volatile("prefetch.global.L2 [%0];" ::"l"(rt + 128 * tid));
-    asm volatile("prefetch.global.L2 [%0];" ::"l"(rt + 128 * (tid + kCombineThreads)));
-  }
-
-  // One pass over the partial headers: thread t owns (partial t/4, head
-  // t%4) for t < 4n (several per thread when n > 64); maxima first, then
-  // weights and sums from the values kept in registers.
-  constexpr int kPer = 4;
-  float mv[kPer], lv[kPer];
-  float mloc = -INFINITY;
-#pragma unroll
-  for (int u = 0; u < kPer; ++u) {
-    const int t = tid + u * kCombineThreads;
-    mv[u] = -INFINITY;
-    lv[u] = 0.f;
-    if (t < 4 * n && !warp_empty(w0 + (t >> 2), F, W)) {
-      const float* pp = pbase + (size_t)(t >> 2) * kPartFloats;
-      mv[u] = __ldg(pp + kPartM + (t & 3));
-      lv[u] = __ldg(pp + kPartL + (t & 3));
-    }
-    mloc = fmaxf(mloc, mv[u]);
-  }
-  for (int t = tid + kPer * kCombineThreads; t < 4 * n; t += kCombineThreads)
-    if (!warp_empty(w0 + (t >> 2), F, W))
-      mloc = fmaxf(mloc, __ldg(pbase + (size_t)(t >> 2) * kPartFloats + kPartM + (t & 3)));
-  // thread t's head is t & 3 == lane & 3: reduce over lanes of equal head
-#pragma unroll
-  for (int o = 4; o < 32; o <<= 1) mloc = fmaxf(mloc, __shfl_xor_sync(0xffffffffu, mloc, o));
-  if (lane < 4) red[warp][lane] = mloc;
+  __syncthreads();  // st initialised
+  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+  for (int i = i0; i < i1; i += kCombineBatch)
+    combine_batch(pbase + (size_t)i * kPartFloats, min(kCombineBatch, i1 - i),
+                  w0 + i, sparse, F, W, st, acc);
+  const int v = tid & 127, ph = tid >> 7;
+  msum[ph][v] = acc;
   __syncthreads();
-  if (tid < 4) {
-    float M = -INFINITY;
-    for (int w = 0; w < kCombineThreads / 32; ++w) M = fmaxf(M, red[w][tid]);
-    ML[0][tid] = M;
-  }
-  __syncthreads();
-  float lloc = 0.f;
-  const float Mh = ML[0][lane & 3];
-#pragma unroll
-  for (int u = 0; u < kPer; ++u) {
-    const int t = tid + u * kCombineThreads;
-    if (t < 4 * n) {
-      const float wgt = merge_weight(mv[u], Mh);
-      lloc += lv[u] * wgt;
-      wts[t] = wgt;
+  if (S > 1) {
+    // publish this chunk: o'[4][128], M[4], L[4] in the partial format
+    const size_t seg = (size_t)b * h_kv + h;
+    float* cp = cpart + (seg * S + sp) * kPartFloats;
+    if (tid < kD) {
+      const float4 a = msum[0][tid], b1 = msum[1][tid], c = msum[2][tid], d = msum[3][tid];
+      reinterpret_cast<float4*>(cp)[tid] =
+          make_float4((a.x + b1.x) + (c.x + d.x), (a.y + b1.y) + (c.y + d.y),
+                      (a.z + b1.z) + (c.z + d.z), (a.w + b1.w) + (c.w + d.w));
+    } else if (tid < kD + 4) {
+      cp[kPartM + tid - kD] = st.M[tid - kD];
+      cp[kPartL + tid - kD] = st.L[tid - kD];
     }
-  }
-  for (int t = tid + kPer * kCombineThreads; t < 4 * n; t += kCombineThreads) {
-    float wgt = 0.f;
-    if (!warp_empty(w0 + (t >> 2), F, W)) {
-      const float* pp = pbase + (size_t)(t >> 2) * kPartFloats;
-      wgt = merge_weight(__ldg(pp + kPartM + (t & 3)), Mh);
-      lloc += __ldg(pp + kPartL + (t & 3)) * wgt;
-    }
-    wts[t] = wgt;
-  }
-#pragma unroll
-  for (int o = 4; o < 32; o <<= 1) lloc += __shfl_xor_sync(0xffffffffu, lloc, o);
-  __syncthreads();
-  if (lane < 4) red[warp][lane] = lloc;
-  __syncthreads();
-  if (tid < 4) {
-    float L = 0.f;
-    for (int w = 0; w < kCombineThreads / 32; ++w) L += red[w][tid];
-    ML[1][tid] = L > 0.f ? 1.f / L : 0.f;
-  }
-  __syncthreads();
-
-  // merge: thread -> channel j, heads hp and hp + 2
-  {
-    const int j = tid & 127, hp = tid >> 7;
-    float o0 = 0.f, o1 = 0.f;
-    // empty partials have weight 0; their (never written) slots are read
-    // but multiplied by a select, never accumulated
-#pragma unroll 8
-    for (int i = 0; i < n; ++i) {
-      const float* pp = pbase + (size_t)i * kPartFloats;
-      const float w0v = wts[4 * i + hp], w1v = wts[4 * i + hp + 2];
-      const float a0 = __ldg(pp + hp * kD + j), a1 = __ldg(pp + (hp + 2) * kD + j);
-      o0 += w0v != 0.f ? a0 * w0v : 0.f;
-      o1 += w1v != 0.f ? a1 * w1v : 0.f;
-    }
-    orot[hp][j] = o0 * ML[1][hp];
-    orot[hp + 2][j] = o1 * ML[1][hp + 2];
-  }
-  __syncthreads();
-  // out[r][i] = sum_jj o'[r][jj] R_v[i][jj] = sum_jj o'[r][jj] R_vT[jj][i]
-  {
-    const int i = tid & 127, hf = tid >> 7;
-    const float* RT = R_vT + (size_t)h * kD * kD + (size_t)(64 * hf) * kD + i;
-    float acc[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll 16
-    for (int k = 0; k < 64; ++k) {
-      const float rt = __ldg(RT + k * kD);
-#pragma unroll
-      for (int r = 0; r < 4; ++r) acc[r] = fmaf(orot[r][64 * hf + k], rt, acc[r]);
-    }
-    if (hf == 1) {
-#pragma unroll
-      for (int r = 0; r < 4; ++r) half_sum[r][i] = acc[r];
-    }
+    __threadfence();
     __syncthreads();
-    if (hf == 0) {
-#pragma unroll
-      for (int r = 0; r < 4; ++r) ob[r * kD + i] = acc[r] + half_sum[r][i];
+    if (tid == 0) last = atomicAdd(cnt_ws + seg, 1) == S - 1;
+    __syncthreads();
+    if (!last) {
+      cp_async_wait<0>();
+      return;
     }
+    __threadfence();
+    if (tid < 4) {
+      st.M[tid] = -INFINITY;
+      st.L[tid] = 0.f;
+    }
+    if (tid == 0) cnt_ws[seg] = 0;
+    __syncthreads();
+    acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int i = 0; i < S; i += kCombineBatch)
+      combine_batch(cpart + (seg * S + i) * kPartFloats, min(kCombineBatch, S - i),
+                    -1, false, F, W, st, acc);
+    msum[ph][v] = acc;
+    __syncthreads();
+  }
+  if (tid < kD) {
+    const float4 a = msum[0][tid], b1 = msum[1][tid], c = msum[2][tid], d = msum[3][tid];
+    const int hd = tid >> 5, ch = (tid & 31) * 4;
+    const float L = st.L[hd];
+    const float il = L > 0.f ? 1.f / L : 0.f;
+    orot[hd][ch + 0] = ((a.x + b1.x) + (c.x + d.x)) * il;
+    orot[hd][ch + 1] = ((a.y + b1.y) + (c.y + d.y)) * il;
+    orot[hd][ch + 2] = ((a.z + b1.z) + (c.z + d.z)) * il;
+    orot[hd][ch + 3] = ((a.w + b1.w) + (c.w + d.w)) * il;
+  }
+  cp_async_wait<0>();
+  __syncthreads();
+  // out[r][i] = sum_k o'[r][k] R_v[i][k] = sum_k o'[r][k] R_vT[k][i]:
+  // thread (i, q) sums k in [32q, 32q + 32) for the 4 heads, reading each
+  // R_v^T element once; the 4 quarters are added through shared memory.
+  {
+    const int i = tid & 127, q = tid >> 7;
+    float acc4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll 8
+    for (int k = 32 * q; k < 32 * q + 32; ++k) {
+      const float rt = rts[k * kD + i];
+#pragma unroll
+      for (int r = 0; r < 4; ++r) acc4[r] = fmaf(orot[r][k], rt, acc4[r]);
+    }
+    float* qs4 = reinterpret_cast<float*>(msum);  // reuse: [4 quarters][4][128]
+#pragma unroll
+    for (int r = 0; r < 4; ++r) qs4[(q * 4 + r) * kD + i] = acc4[r];
+    __syncthreads();
+    const int r = tid >> 7;
+    ob[r * kD + i] = (qs4[(0 * 4 + r) * kD + i] + qs4[(1 * 4 + r) * kD + i]) +
+                     (qs4[(2 * 4 + r) * kD + i] + qs4[(3 * 4 + r) * kD + i]);
   }
 }
 
@@ -497,10 +584,10 @@ cudaError_t launch_decode(const optr_params* p, int variant,
   const float qscale = kLog2e / sqrtf((float)kD);
 
   prof_mark(p, 2, s);
-  qrot_kernel<<<dim3(B, h_kv), kQrotThreads, 0, s>>>(q, p->R_k, B, h_q, h_kv, qscale,
-                                            seq_lens, max_pages, qf, qs, frag,
-                                            koff, invs, pref, nzpref, p->err);
-  cudaError_t e = cudaGetLastError();
+  cudaError_t e = launch_pdl(qrot_kernel, dim3(B, h_kv), dim3(kQrotThreads), 0,
+                             s, q, p->R_k, B, h_q, h_kv, qscale, seq_lens,
+                             max_pages, qf, qs, frag, koff, invs, pref, nzpref,
+                             reinterpret_cast<int*>(w + plan.off_cnt), p->err);
   if (e != cudaSuccess) return e;
   prof_mark(p, 3, s);
   if (variant != OPTR_VARIANT_CUDA_CORE) {
@@ -508,23 +595,24 @@ cudaError_t launch_decode(const optr_params* p, int variant,
                               frag, koff, invs, qs, pref, nzpref, part, plan.W,
                               s);
   } else {
-    partial_cuda_core_kernel<<<plan.W / 4, 128, 0, s>>>(
-        pool, bt, seq_lens, B, max_pages, num_pages, h_q, h_kv, qf, qs, pref,
-        nzpref, part, plan.W, p->err);
-    e = cudaGetLastError();
+    e = launch_pdl(partial_cuda_core_kernel, dim3(plan.W / 4), dim3(128), 0, s,
+                   pool, bt, seq_lens, B, max_pages, num_pages, h_q, h_kv, qf,
+                   qs, pref, nzpref, part, plan.W, p->err);
   }
   if (e != cudaSuccess) return e;
   prof_mark(p, 4, s);
-  const size_t wts_bytes = sizeof(float) * 4 * (plan.W + 1);
+  const size_t cmb_bytes = sizeof(float) * kD * kD;
   e = ensure_dynamic_smem(reinterpret_cast<const void*>(&combine_kernel),
-                          wts_bytes);
+                          cmb_bytes);
   if (e != cudaSuccess) return e;
-  combine_kernel<<<dim3(B, h_kv), kCombineThreads,
-                   wts_bytes, s>>>(part, pref, nzpref,
-                                                          B, h_q, h_kv, plan.W,
-                                                          p->R_vT, out);
+  e = launch_pdl(combine_kernel, dim3(B, h_kv, plan.S), dim3(kCombineThreads),
+                 cmb_bytes, s, (const float*)part, (const int*)pref,
+                 (const int*)nzpref, B, h_q, h_kv, plan.W, (const float*)p->R_vT,
+                 reinterpret_cast<float*>(w + plan.off_cpart),
+                 reinterpret_cast<int*>(w + plan.off_cnt), out);
+  if (e != cudaSuccess) return e;
   prof_mark(p, 5, s);
-  return cudaGetLastError();
+  return cudaSuccess;
 }
 
 }  // namespace optr

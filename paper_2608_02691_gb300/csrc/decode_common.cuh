@@ -22,12 +22,12 @@ __device__ __forceinline__ Segment locate_segment(long long f, long long f1,
                        // construction because f < pref[B]*h_kv)
   while (hi - lo > 1) {
     const int mid = (lo + hi) >> 1;
-    if ((long long)__ldg(pref + mid) * h_kv <= f) lo = mid; else hi = mid;
+    if ((long long)__ldcg(pref + mid) * h_kv <= f) lo = mid; else hi = mid;
   }
   Segment s;
   s.b = lo;
-  const int np = __ldg(pref + lo + 1) - __ldg(pref + lo);
-  const long long base = (long long)__ldg(pref + lo) * h_kv;
+  const int np = __ldcg(pref + lo + 1) - __ldcg(pref + lo);
+  const long long base = (long long)__ldcg(pref + lo) * h_kv;
   const long long r = f - base;
   s.h = (int)(r / np);
   s.p0 = (int)(r - (long long)s.h * np);

@@ -170,11 +170,11 @@ __device__ __forceinline__ void load_chunk(PageChunk& ch, int base, int f1,
     int lo = 0, hi = B;  // largest b with pref[b] * h_kv <= f
     while (hi - lo > 1) {
       const int mid = (lo + hi) >> 1;
-      const int pm = cached ? spref[mid] : __ldg(pref + mid);
+      const int pm = cached ? spref[mid] : __ldcg(pref + mid);
       if (pm * h_kv <= f) lo = mid; else hi = mid;
     }
-    const int p0 = cached ? spref[lo] : __ldg(pref + lo);
-    const int np = (cached ? spref[lo + 1] : __ldg(pref + lo + 1)) - p0;
+    const int p0 = cached ? spref[lo] : __ldcg(pref + lo);
+    const int np = (cached ? spref[lo + 1] : __ldcg(pref + lo + 1)) - p0;
     const int r = f - p0 * h_kv;
     const int h = r / np;
     const int page = r - h * np;
@@ -203,19 +203,21 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
                       float* __restrict__ part, int W, unsigned* err) {
   __shared__ WarpSmemTC smem[kWarps];
   __shared__ int spref[kPrefCache + 1];
+  pdl_wait();
+  pdl_trigger();
   uint32_t e1024;
   asm volatile("mov.b32 %0, 0x64006400;" : "=r"(e1024));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int g = lane >> 2, c = lane & 3;
   WarpSmemTC& S = smem[warp];
   const int w = blockIdx.x * kWarps + warp;
-  const int F = __ldg(pref + B) * h_kv;
+  const int F = __ldcg(pref + B) * h_kv;
   const int f0 = (int)((long long)w * F / W), f1 = (int)((long long)(w + 1) * F / W);
 
   // first segment of this warp: sequence b with pref[b]*h_kv <= f0
   const bool cached = B <= kPrefCache;
   if (cached)
-    for (int i = threadIdx.x; i <= B; i += kWarps * 32) spref[i] = __ldg(pref + i);
+    for (int i = threadIdx.x; i <= B; i += kWarps * 32) spref[i] = __ldcg(pref + i);
   __syncthreads();
   if (f0 >= f1) return;
   PageChunk chk;
@@ -271,7 +273,7 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
       for (int o = 4; o < 32; o <<= 1)
         mv[G] += __shfl_xor_sync(0xffffffffu, mv[G], o);
     const int cb = cur_key / h_kv, ch = cur_key - cb * h_kv;
-    float* slot = part + (size_t)(w + __ldg(nzpref + cb) * h_kv + ch) * kPartFloats;
+    float* slot = part + (size_t)(w + __ldcg(nzpref + cb) * h_kv + ch) * kPartFloats;
     float* dst = slot + c * kD;
 #pragma unroll
     for (int G = 0; G < kGroups; ++G) {
@@ -297,7 +299,7 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
         frag + (((size_t)cb * h_kv + ch) * 32 + lane) * 16);
 #pragma unroll
     for (int G = 0; G < kGroups; ++G) {
-      const uint4 v = __ldg(fq + G);
+      const uint4 v = __ldcg(fq + G);
       bq[G][0][0] = v.x;
       bq[G][0][1] = v.y;
       bq[G][1][0] = v.z;
@@ -306,19 +308,19 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
     {
       const float4* ko = reinterpret_cast<const float4*>(
           koff + ((size_t)cb * h_kv + ch) * 32 + c * 8);
-      const float4 k01 = __ldg(ko), k23 = __ldg(ko + 1);
+      const float4 k01 = __ldcg(ko), k23 = __ldcg(ko + 1);
       kneg[0][0] = -k01.x; kneg[0][1] = -k01.y;
       kneg[1][0] = -k01.z; kneg[1][1] = -k01.w;
       kneg[2][0] = -k23.x; kneg[2][1] = -k23.y;
       kneg[3][0] = -k23.z; kneg[3][1] = -k23.w;
     }
     const size_t row = (size_t)cb * h_q + 4 * ch + c;
-    const float4 q4 = __ldg(reinterpret_cast<const float4*>(qs + row * kGroups));
+    const float4 q4 = __ldcg(reinterpret_cast<const float4*>(qs + row * kGroups));
     qsum[0] = q4.x;
     qsum[1] = q4.y;
     qsum[2] = q4.z;
     qsum[3] = q4.w;
-    inv_s = __ldg(invs + row);
+    inv_s = __ldcg(invs + row);
 #pragma unroll
     for (int G = 0; G < kGroups; ++G) {
       mv[G] = 0.f;
@@ -510,10 +512,10 @@ cudaError_t launch_partial_tensor(const optr_params* p, const uint8_t* pool,
                                   const float* invs, const float* qs,
                                   const int* pref, const int* nzpref,
                                   float* part, int W, cudaStream_t s) {
-  partial_tensor_kernel<<<W / kWarps, kWarps * 32, 0, s>>>(
-      pool, bt, seq_lens, B, max_pages, num_pages, p->cfg.h_q, p->cfg.h_kv,
-      frag, koff, invs, qs, pref, nzpref, part, W, p->err);
-  return cudaGetLastError();
+  return launch_pdl(partial_tensor_kernel, dim3(W / kWarps), dim3(kWarps * 32),
+                    0, s, pool, bt, seq_lens, B, max_pages, num_pages,
+                    p->cfg.h_q, p->cfg.h_kv, frag, koff, invs, qs, pref, nzpref,
+                    part, W, p->err);
 }
 
 }  // namespace optr

@@ -6,6 +6,7 @@
 #include <stdlib.h>
 #include <string.h>
 
+#include <algorithm>
 #include <mutex>
 #include <vector>
 
@@ -63,7 +64,12 @@ cudaError_t ensure_dynamic_smem(const void* kernel, size_t bytes) {
 //                               [query head][group][hi/lo] (decode_tc.cu)
 //   invs float [B][h_q]         1 / (power-of-two prescale of frag)
 //   pref int   [2][B+1]        page prefix sums / non-empty prefix counts
+//   cnt  int   [B*h_kv]        combine arrival counters (zeroed by qrot)
 //   part float [W + B*h_kv][520] split-K partials (o'[4][128], m[4], l[4])
+//   cpart float [B*h_kv*S][520] combine chunk results (only when S > 1)
+// S, the combine CTAs per (sequence, KV head), is sized for ~32 partials
+// each when every sequence is max_pages long: a segment then overlaps about
+// W / (B*h_kv) + 2 warp ranges.
 DecodePlan decode_plan(const optr_params* p, int B, int max_pages) {
   DecodePlan d;
   d.B = B;
@@ -84,9 +90,20 @@ DecodePlan decode_plan(const optr_params* p, int B, int max_pages) {
   o = round_up(o + sizeof(float) * (size_t)B * d.h_q, 256);
   d.off_pref = o;
   o = round_up(o + sizeof(int) * 2 * (size_t)(B + 1), 256);
+  d.off_cnt = o;
+  o = round_up(o + sizeof(int) * (size_t)B * d.h_kv, 256);
   d.off_part = o;
   o = round_up(o + sizeof(float) * kPartFloats *
                        ((size_t)d.W + (size_t)B * d.h_kv), 256);
+  {
+    const long long segs = (long long)B * d.h_kv;
+    const long long n_est = d.W / segs + 2;
+    d.S = (int)std::min<long long>(kCombineMaxSplit,
+                                   std::max<long long>(1, (n_est + 31) / 32));
+  }
+  d.off_cpart = o;
+  if (d.S > 1)
+    o = round_up(o + sizeof(float) * kPartFloats * (size_t)B * d.h_kv * d.S, 256);
   d.total = o;
   return d;
 }

@@ -21,6 +21,7 @@ constexpr int kMaxRatio = 8;             // largest supported h_q / h_kv
 // partial kernel; the workspace holds one partial slot per warp plus one per
 // (sequence, KV head), see DecodePlan.
 constexpr int kDecodeWarpsPerSm = 16;
+constexpr int kCombineMaxSplit = 16;  // combine CTAs per (sequence, KV head)
 
 }  // namespace optr
 
@@ -50,6 +51,39 @@ namespace optr {
 // runtime call is made once per new maximum.
 cudaError_t ensure_dynamic_smem(const void* kernel, size_t bytes);
 
+// Programmatic dependent launch.  Every kernel of the library is launched
+// with launch_pdl(), so the GPU may schedule it while the previous kernel in
+// the stream is still draining.  Each kernel calls pdl_wait() before it
+// touches any memory that an earlier kernel in the stream may write (or
+// read): only the library-owned rotation state in optr_params may be read
+// before it.  pdl_wait() returns once the previous grid has completed and
+// its writes are visible; since every kernel waits before it completes, the
+// order of the whole stream is kept.  pdl_trigger() (right after the wait)
+// lets the next kernel's blocks be scheduled.  Data written by the previous
+// kernel is read with ld.global.cg (__ldcg), never the non-coherent path.
+__device__ __forceinline__ void pdl_wait() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+__device__ __forceinline__ void pdl_trigger() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block,
+                       size_t smem, cudaStream_t s, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
+
 // Record stage event i on stream s when profiling is on.
 inline void prof_mark(const optr_params* p, int i, cudaStream_t s) {
   if (p->prof) cudaEventRecord(p->ev[i], s);
@@ -61,7 +95,9 @@ namespace optr {
 // Byte offsets of the decode workspace for a batch shape.
 struct DecodePlan {
   int B, h_q, h_kv, max_pages, W;  // W = partial-kernel warps
-  size_t off_qf, off_qs, off_frag, off_koff, off_invs, off_pref, off_part, total;
+  int S;                           // combine CTAs per (sequence, KV head)
+  size_t off_qf, off_qs, off_frag, off_koff, off_invs, off_pref, off_cnt,
+      off_part, off_cpart, total;
 };
 DecodePlan decode_plan(const optr_params* p, int B, int max_pages);
 
