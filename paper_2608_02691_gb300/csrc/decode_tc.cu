@@ -126,12 +126,14 @@ __device__ __forceinline__ float2 h2f(uint32_t u) {
   return __half22float2(*reinterpret_cast<const __half2*>(&u));
 }
 
-// fp16 hi / lo split of x, packed (hi in the low half).
+// fp16 hi / lo split of x, packed (hi in the low half): hi is x with its
+// mantissa cut to 11 significant bits (exact in fp16 when |x| is in fp16's
+// normal range), lo = x - hi exactly, rounded to fp16.
 __device__ __forceinline__ uint32_t split_hilo(float x) {
-  const __half hi = __float2half_rn(x);
-  const float lo = x - __half2float(hi);
+  const float hi = __uint_as_float(__float_as_uint(x) & 0xffffe000u);
+  const float lo = x - hi;
   uint32_t r;
-  asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(lo), "f"(x));
+  asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(lo), "f"(hi));
   return r;
 }
 
@@ -255,11 +257,14 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
   // per-segment state
   uint32_t bq[kGroups][2][2];  // query B fragments [group][kk][reg]
   float kneg[kGroups][2];      // minus the key-code offset sums, head c
-  float qsum[kGroups];         // sum of q' over each group, head c
+  uint32_t bmin = 0;           // key min-term B fragment (sum q' per group)
   float inv_s = 0.f;           // 1 / prescale of head c
   float acc_o[kGroups][2][4];  // values: [group][half][c-frag]
   float mv[kGroups];           // sum_tok p * min_v per group (this lane)
-  float m_run = -INFINITY, l_lane = 0.f;
+  float m_ref = -INFINITY, l_lane = 0.f;
+  float m_lazy = -INFINITY;    // kLazyTau above the running maximum logit
+  int k_s = -30;               // 2^k_s bounds the value scales seen
+  float s_cap = 0x1p-30f;      // 2^k_s
   int cur_key = -1;
 
   auto flush = [&]() {
@@ -287,7 +292,7 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
       *reinterpret_cast<float4*>(dst + 32 * G + 4 * g) = o4;
     }
     if (g == 0) {
-      slot[kPartM + c] = m_run;
+      slot[kPartM + c] = m_ref;
       slot[kPartL + c] = l;
     }
   };
@@ -315,11 +320,13 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
       kneg[3][0] = -k23.z; kneg[3][1] = -k23.w;
     }
     const size_t row = (size_t)cb * h_q + 4 * ch + c;
-    const float4 q4 = __ldcg(reinterpret_cast<const float4*>(qs + row * kGroups));
-    qsum[0] = q4.x;
-    qsum[1] = q4.y;
-    qsum[2] = q4.z;
-    qsum[3] = q4.w;
+    {
+      // column g of the min-term MMA: head g/2, fp16 limb g%2 of the
+      // group-c sum of q'; rows k = 2c (scale entries) are 0
+      const float qg = __ldcg(qs + ((size_t)cb * h_q + 4 * ch + (g >> 1)) * kGroups + c);
+      const uint32_t hl = split_hilo(qg);
+      bmin = (g & 1) ? (hl & 0xffff0000u) : (hl << 16);
+    }
     inv_s = __ldcg(invs + row);
 #pragma unroll
     for (int G = 0; G < kGroups; ++G) {
@@ -329,7 +336,10 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
 #pragma unroll
         for (int k = 0; k < 4; ++k) acc_o[G][hf][k] = 0.f;
     }
-    m_run = -INFINITY;
+    m_ref = -INFINITY;
+    m_lazy = -INFINITY;
+    k_s = -30;
+    s_cap = 0x1p-30f;
     l_lane = 0.f;
   };
 
@@ -367,36 +377,75 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
       const uint4 km1 = *reinterpret_cast<const uint4*>(st + OPTR_K_META_OFFSET + (g + 8) * 16);
       const uint32_t kmv0[4] = {km0.x, km0.y, km0.z, km0.w};
       const uint32_t kmv1[4] = {km1.x, km1.y, km1.z, km1.w};
-      float t0 = 0.f, t1 = 0.f, u0 = 0.f, u1 = 0.f;
+      // sum_g min_g * sum(q' over g) on the tensor core: A row t = the 8
+      // (scale, min) halves of token t, B = (0, Q_g) per (scale, min) pair
+      float u[4] = {0.f, 0.f, 0.f, 0.f};
+      {
+        const uint32_t w0 = *reinterpret_cast<const uint32_t*>(st + OPTR_K_META_OFFSET + g * 16 + 4 * c);
+        const uint32_t w1 = *reinterpret_cast<const uint32_t*>(st + OPTR_K_META_OFFSET + (g + 8) * 16 + 4 * c);
+        mma16816(u, w0, w1, 0u, 0u, bmin, 0u);
+      }
+      float t0 = 0.f, t1 = 0.f;
 #pragma unroll
       for (int G = 0; G < kGroups; ++G) {
-        const float2 a = h2f(kmv0[G]);   // (scale, min) of token g
-        const float2 bb = h2f(kmv1[G]);  // token g+8
-        t0 = fmaf(a.x, s_acc[G][0] + s_acc[G][1], t0);
-        t1 = fmaf(bb.x, s_acc[G][2] + s_acc[G][3], t1);
-        u0 = fmaf(a.y, qsum[G], u0);
-        u1 = fmaf(bb.y, qsum[G], u1);
+        const float a = __low2float(*reinterpret_cast<const __half2*>(&kmv0[G]));   // scale, token g
+        const float bb = __low2float(*reinterpret_cast<const __half2*>(&kmv1[G]));  // token g+8
+        t0 = fmaf(a, s_acc[G][0] + s_acc[G][1], t0);
+        t1 = fmaf(bb, s_acc[G][2] + s_acc[G][3], t1);
       }
-      sc0 = fmaf(inv_s, t0, u0);
-      sc1 = fmaf(inv_s, t1, u1);
+      sc0 = fmaf(inv_s, t0, u[0] + u[1]);
+      sc1 = fmaf(inv_s, t1, u[2] + u[3]);
       if (!FULL) {
         sc0 = v0 ? sc0 : -INFINITY;
         sc1 = v1 ? sc1 : -INFINITY;
       }
     }
-    // ---------------------------------------------------- online softmax
-    // Lazy rescaling: the running reference m_run of head c only moves when
-    // some logit exceeds it by more than kLazyTau (log2 units), so p <= 2^8.
-    // Each lane tests its own logits; only then is the head maximum reduced
-    // over the 8 lanes of the head and the accumulators rescaled.
+    // ------------------------------------------- value metadata, softmax
+    const uint4 vm0 = *reinterpret_cast<const uint4*>(st + OPTR_V_META_OFFSET + g * 16);
+    const uint4 vm1 = *reinterpret_cast<const uint4*>(st + OPTR_V_META_OFFSET + (g + 8) * 16);
+    const uint32_t vmv0[4] = {vm0.x, vm0.y, vm0.z, vm0.w};
+    const uint32_t vmv1[4] = {vm1.x, vm1.y, vm1.z, vm1.w};
+    float2 va[kGroups], vb[kGroups];  // (scale, min) of tokens g, g+8
+    float smax = 0.f;
+#pragma unroll
+    for (int G = 0; G < kGroups; ++G) {
+      va[G] = h2f(vmv0[G]);
+      vb[G] = h2f(vmv1[G]);
+      if (!FULL) {
+        // masked tokens have p = 0; their (possibly garbage) metadata is
+        // never multiplied in
+        va[G] = v0 ? va[G] : make_float2(0.f, 0.f);
+        vb[G] = v1 ? vb[G] : make_float2(0.f, 0.f);
+      }
+      smax = fmaxf(smax, fmaxf(va[G].x, vb[G].x));
+    }
+    // Lazy reference: p = 2^(l - m_ref) with m_ref = m_lazy + k_s - 15,
+    // where m_lazy lies kLazyTau (log2 units) above the head's running
+    // maximum logit and 2^k_s bounds every value scale seen.  Then
+    // p * scale <= 2^15 always fits fp16, and the largest products sit near
+    // 2^15, so their fp16 lo parts stay normal whatever the magnitude of the
+    // values.  m_lazy and k_s move only when a logit exceeds m_lazy or a
+    // scale exceeds 2^k_s; each lane tests its own tokens, and only then are
+    // the head maxima reduced over the 8 lanes of the head and the
+    // accumulators rescaled.
     {
       const float lmax = fmaxf(sc0, sc1);
-      if (__any_sync(0xffffffffu, lmax > m_run + kLazyTau)) {
-        float tmax = lmax;
+      if (__any_sync(0xffffffffu, lmax > m_lazy || smax > s_cap)) {
+        float tmax = lmax, smx = smax;
 #pragma unroll
-        for (int o = 4; o < 32; o <<= 1) tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, o));
-        if (tmax > m_run + kLazyTau) {  // uniform over the lanes of head c
-          const float alpha = (m_run == -INFINITY) ? 0.f : ex2(m_run - tmax);
+        for (int o = 4; o < 32; o <<= 1) {
+          tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, o));
+          smx = fmaxf(smx, __shfl_xor_sync(0xffffffffu, smx, o));
+        }
+        // uniform over the lanes of head c
+        if (tmax > m_lazy) m_lazy = tmax + kLazyTau;
+        if (smx > s_cap) {
+          k_s = ilogbf(smx) + 1;  // smx < 2^k_s
+          s_cap = ldexpf(1.f, k_s);
+        }
+        const float m_new = m_lazy + (float)(k_s - 15);
+        if (m_new != m_ref) {
+          const float alpha = (m_ref == -INFINITY) ? 0.f : ex2(m_ref - m_new);
           l_lane *= alpha;
 #pragma unroll
           for (int G = 0; G < kGroups; ++G) {
@@ -406,39 +455,25 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
 #pragma unroll
               for (int k = 0; k < 4; ++k) acc_o[G][hf][k] *= alpha;
           }
-          m_run = tmax;
+          m_ref = m_new;
         }
       }
     }
-    float p0 = ex2(sc0 - m_run), p1 = ex2(sc1 - m_run);  // ex2(-inf) = 0
+    float p0 = ex2(sc0 - m_ref), p1 = ex2(sc1 - m_ref);  // ex2(-inf) = 0
     if (!FULL) {  // a fully masked page before any finite max: -inf - -inf
       p0 = v0 ? p0 : 0.f;
       p1 = v1 ? p1 : 0.f;
     }
     l_lane += p0 + p1;
     // ------------------------------------------------------------ values
-    {
-      const uint4 vm0 = *reinterpret_cast<const uint4*>(st + OPTR_V_META_OFFSET + g * 16);
-      const uint4 vm1 = *reinterpret_cast<const uint4*>(st + OPTR_V_META_OFFSET + (g + 8) * 16);
-      const uint32_t vmv0[4] = {vm0.x, vm0.y, vm0.z, vm0.w};
-      const uint32_t vmv1[4] = {vm1.x, vm1.y, vm1.z, vm1.w};
 #pragma unroll
-      for (int G = 0; G < kGroups; ++G) {
-        float2 a = h2f(vmv0[G]);
-        float2 bb = h2f(vmv1[G]);
-        if (!FULL) {
-          // masked tokens have p = 0; their (possibly garbage) metadata is
-          // never multiplied in
-          a = v0 ? a : make_float2(0.f, 0.f);
-          bb = v1 ? bb : make_float2(0.f, 0.f);
-        }
-        // the MMA sees centered codes (code - 1.5): the min term carries
-        // min + 1.5 * scale
-        const float ps0 = p0 * a.x, ps1 = p1 * bb.x;
-        mv[G] = fmaf(1.5f, ps0, fmaf(p0, a.y, fmaf(1.5f, ps1, fmaf(p1, bb.y, mv[G]))));
-        S.pt[G][g][c] = split_hilo(ps0);
-        S.pt[G][g + 8][c] = split_hilo(ps1);
-      }
+    for (int G = 0; G < kGroups; ++G) {
+      // the MMA sees centered codes (code - 1.5): the min term carries
+      // min + 1.5 * scale
+      const float ps0 = p0 * va[G].x, ps1 = p1 * vb[G].x;
+      mv[G] = fmaf(1.5f, ps0, fmaf(p0, va[G].y, fmaf(1.5f, ps1, fmaf(p1, vb[G].y, mv[G]))));
+      S.pt[G][g][c] = split_hilo(ps0);
+      S.pt[G][g + 8][c] = split_hilo(ps1);
     }
     __syncwarp();
     uint32_t bv[kGroups][2];

@@ -230,3 +230,22 @@ def test_workspace_too_small_is_rejected():
         optr.optr_decode_attention(p, c["q"].cuda(), c["block_table"].cuda(),
                                    c["seq_lens"].cuda(), pool, out, ws)
     assert e.value.status == -4
+
+
+@pytest.mark.parametrize("variant", VARIANTS)
+@pytest.mark.parametrize("kscale,vscale", [(1.0, 1024.0), (1 / 64, 1 / 4096), (8.0, 1.0)])
+def test_decode_value_magnitudes(variant, kscale, vscale):
+    """Keys and values far from unit magnitude (large value scales, where
+    p * scale would leave fp16's range without the softmax reference's
+    headroom; tiny ones near fp16's subnormal range; sharp logits).  Powers
+    of two keep the bf16 inputs exact."""
+    c = synth.build_case(synth.workload("decode8k", 1, 1 / 32), 1)
+    for kk, f in (("k_ctx", kscale), ("k_new", kscale), ("v_ctx", vscale),
+                  ("v_new", vscale)):
+        c[kk] = (c[kk].float() * f).to(torch.bfloat16)
+    c["mu"] = c["mu"] * kscale
+    pool_ref, _, _ = ph.oracle_case(c)
+    got = ph.gpu_decode(c, pool_ref, variant=variant)
+    ref = ph.oracle_decode(c, pool_ref)
+    r = ph.assert_decode_close(got, ref, f"k x{kscale} v x{vscale}")
+    print(f"k x{kscale} v x{vscale} variant {variant}: err/rms {r:.2e}")
