@@ -260,7 +260,7 @@ optr_status optr_profile_last(const optr_params* p, float ms[4]);
  * OPTR_NOALLOC_SCRATCH_BYTES (16 MiB) in the library's device image; every
  * GPU that loads the library holds it until the process exits.  A batch
  * whose workspace would exceed it (optr_decode_workspace_size(p, B,
- * max_pages) > OPTR_NOALLOC_SCRATCH_BYTES; about B > 200 at 8 KV heads on a
+ * max_pages) > OPTR_NOALLOC_SCRATCH_BYTES; about B > 230 at 8 KV heads on a
  * 152-SM GPU) is rejected with OPTR_ERR_WORKSPACE before any launch.
  *
  * The first call on each device looks up the array's device address with
