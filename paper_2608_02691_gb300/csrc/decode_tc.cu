@@ -41,7 +41,7 @@ namespace optr {
 namespace {
 
 constexpr int kStages = 4;            // cp.async pages in flight per warp
-constexpr int kWarps = 4;             // warps per CTA
+constexpr int kWarps = 16;            // warps per CTA: one CTA per SM
 constexpr float kLazyTau = 8.f;       // log2-domain slack before rescaling
 
 struct WarpSmemTC {
@@ -191,7 +191,7 @@ __device__ __forceinline__ void load_chunk(PageChunk& ch, int base, int f1,
   }
 }
 
-__global__ void __launch_bounds__(kWarps * 32, 4)
+__global__ void __launch_bounds__(kWarps * 32, 1)
 partial_tensor_kernel(const uint8_t* __restrict__ pool,
                       const int32_t* __restrict__ bt,
                       const int32_t* __restrict__ seq_lens, int B,
@@ -203,7 +203,11 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
                       const int* __restrict__ pref,
                       const int* __restrict__ nzpref,
                       float* __restrict__ part, int W, unsigned* err) {
-  __shared__ WarpSmemTC smem[kWarps];
+  // One 16-warp CTA per SM: the warp schedulers favour the CTAs that
+  // arrived first on an SM, and with four 4-warp CTAs per SM the last CTA
+  // finished ~20% after the first; within one CTA the warps keep pace.
+  extern __shared__ __align__(16) unsigned char dsm_[];
+  WarpSmemTC* smem = reinterpret_cast<WarpSmemTC*>(dsm_);  // [kWarps]
   __shared__ int spref[kPrefCache + 1];
   pdl_wait();
   pdl_trigger();
@@ -547,8 +551,12 @@ cudaError_t launch_partial_tensor(const optr_params* p, const uint8_t* pool,
                                   const float* invs, const float* qs,
                                   const int* pref, const int* nzpref,
                                   float* part, int W, cudaStream_t s) {
+  const size_t dsmem = sizeof(WarpSmemTC) * kWarps;
+  cudaError_t e =
+      ensure_dynamic_smem(reinterpret_cast<const void*>(&partial_tensor_kernel), dsmem);
+  if (e != cudaSuccess) return e;
   return launch_pdl(partial_tensor_kernel, dim3(W / kWarps), dim3(kWarps * 32),
-                    0, s, pool, bt, seq_lens, B, max_pages, num_pages,
+                    dsmem, s, pool, bt, seq_lens, B, max_pages, num_pages,
                     p->cfg.h_q, p->cfg.h_kv, frag, koff, invs, qs, pref, nzpref,
                     part, W, p->err);
 }
