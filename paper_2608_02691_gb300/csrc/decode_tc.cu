@@ -241,13 +241,13 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
       const int unit = __shfl_sync(0xffffffffu, chk.unit, j);
       const int key = __shfl_sync(0xffffffffu, chk.key, j);
       const int nv = __shfl_sync(0xffffffffu, chk.nvalid, j);
-      if (unit >= 0) {
-        const uint8_t* src = pool + (size_t)unit * kChunk + lane * 16;
-        uint8_t* dst = S.stage[s] + lane * 16;
-        cp_async16(dst, src);
-        cp_async16(dst + 512, src + 512);
-        cp_async16(dst + 1024, src + 1024);
-      }
+      // an invalid page (flagged, all tokens masked) is filled with zeros
+      const bool ok = unit >= 0;
+      const uint8_t* src = pool + (size_t)(ok ? unit : 0) * kChunk + lane * 16;
+      uint8_t* dst = S.stage[s] + lane * 16;
+      cp_async16_zfill(dst, src, ok);
+      cp_async16_zfill(dst + 512, src + 512, ok);
+      cp_async16_zfill(dst + 1024, src + 1024, ok);
       cp_async_commit();
       S.info[s] = make_int2(key, nv);  // same value from every lane
       ++f_issue;
@@ -515,29 +515,25 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
     }
   };
 
+  static_assert((kStages & (kStages - 1)) == 0, "kStages: a power of two");
   const int total = f1 - f0;
-  int done = 0;
-  while (done < total) {
 #pragma unroll 1
-    for (int s = 0; s < kStages; ++s) {
-      if (done < total) {
-        issue((s + kStages - 1) % kStages);
-        cp_async_wait<kStages - 1>();
-        __syncwarp();
-        const int2 inf = S.info[s];
-        const int nvalid = inf.y;
-        if (inf.x != cur_key) {
-          if (cur_key >= 0) flush();
-          begin_segment(inf.x);
-        }
-        if (nvalid == kPage)
-          page(S.stage[s], nvalid, std::true_type{});
-        else
-          page(S.stage[s], nvalid, std::false_type{});
-        __syncwarp();
-        ++done;
-      }
+  for (int done = 0; done < total; ++done) {
+    const int s = done & (kStages - 1);
+    issue((s + kStages - 1) & (kStages - 1));
+    cp_async_wait<kStages - 1>();
+    __syncwarp();
+    const int2 inf = S.info[s];
+    const int nvalid = inf.y;
+    if (inf.x != cur_key) {
+      if (cur_key >= 0) flush();
+      begin_segment(inf.x);
     }
+    if (nvalid == kPage)
+      page(S.stage[s], nvalid, std::true_type{});
+    else
+      page(S.stage[s], nvalid, std::false_type{});
+    __syncwarp();
   }
   flush();
 }
