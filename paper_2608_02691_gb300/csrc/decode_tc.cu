@@ -46,7 +46,7 @@ constexpr float kLazyTau = 8.f;       // log2-domain slack before rescaling
 
 struct WarpSmemTC {
   alignas(16) uint8_t stage[kStages][kChunk];
-  alignas(16) uint32_t pt[kGroups][kPage][4];  // p*scale_v (hi, lo) per head
+  alignas(16) uint32_t pt[2][kGroups][kPage][4];  // p*scale_v (hi, lo) per head, 2 pages
   int2 info[kStages];  // per staged page: (segment key b*h_kv+h, valid tokens)
 };
 
@@ -231,7 +231,8 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
   load_chunk(chk, f0, f1, pref, spref, cached, seq_lens, bt, B, h_kv,
              max_pages, num_pages, err, lane);
 
-  // issue one page into stage s; every lane records what the stage holds
+  // issue one page into stage s (no commit); every lane records what the
+  // stage holds
   auto issue = [&](int s) {
     if (f_issue < f1) {
       if (f_issue - chk.base == 32)
@@ -248,15 +249,17 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
       cp_async16_zfill(dst, src, ok);
       cp_async16_zfill(dst + 512, src + 512, ok);
       cp_async16_zfill(dst + 1024, src + 1024, ok);
-      cp_async_commit();
       S.info[s] = make_int2(key, nv);  // same value from every lane
       ++f_issue;
-    } else {
-      cp_async_commit();
     }
   };
-#pragma unroll
-  for (int s = 0; s < kStages - 1; ++s) issue(s);
+  // the next two pages into stages 2q, 2q+1, one cp.async group
+  auto issue_pair = [&](int q) {
+    issue(2 * q);
+    issue(2 * q + 1);
+    cp_async_commit();
+  };
+  issue_pair(0);
 
   // per-segment state
   uint32_t bq[kGroups][2][2];  // query B fragments [group][kk][reg]
@@ -347,193 +350,248 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
     l_lane = 0.f;
   };
 
-  // One page of the stage st: logits, online softmax, values.  FULL = all
-  // 16 tokens valid (no masking code).
+  // ------------------------------------------------ parts of one page
+  // logits of tokens g and g+8 (head c) of the page staged at st
+  auto logits = [&](const uint8_t* st, float& sc0, float& sc1) {
+    const uint2 k0 = *reinterpret_cast<const uint2*>(st + OPTR_K_CODES_OFFSET + g * 32 + 8 * c);
+    const uint2 k1 = *reinterpret_cast<const uint2*>(st + OPTR_K_CODES_OFFSET + (g + 8) * 32 + 8 * c);
+    // bytes [G0 w2c, G1 w2c, G0 w2c+1, G1 w2c+1] and the same for G2/G3
+    const uint32_t y01_0 = __byte_perm(k0.x, k0.y, 0x5410);
+    const uint32_t y23_0 = __byte_perm(k0.x, k0.y, 0x7632);
+    const uint32_t y01_1 = __byte_perm(k1.x, k1.y, 0x5410);
+    const uint32_t y23_1 = __byte_perm(k1.x, k1.y, 0x7632);
+    float s_acc[kGroups][4];
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {  // groups 2j, 2j+1
+      uint32_t f0[2][4], f1[2][4];  // token rows g, g+8
+      code_fields(j ? y23_0 : y01_0, e1024, f0);
+      code_fields(j ? y23_1 : y01_1, e1024, f1);
+#pragma unroll
+      for (int par = 0; par < 2; ++par) {
+        const int G = 2 * j + par;
+        mma16816_c(s_acc[G], f0[par][0], f1[par][0], f0[par][1], f1[par][1],
+                   bq[G][0][0], bq[G][0][1], kneg[G][0], kneg[G][1]);
+        mma16816(s_acc[G], f0[par][2], f1[par][2], f0[par][3], f1[par][3],
+                 bq[G][1][0], bq[G][1][1]);
+      }
+    }
+    const uint4 km0 = *reinterpret_cast<const uint4*>(st + OPTR_K_META_OFFSET + g * 16);
+    const uint4 km1 = *reinterpret_cast<const uint4*>(st + OPTR_K_META_OFFSET + (g + 8) * 16);
+    const uint32_t kmv0[4] = {km0.x, km0.y, km0.z, km0.w};
+    const uint32_t kmv1[4] = {km1.x, km1.y, km1.z, km1.w};
+    // sum_g min_g * sum(q' over g) on the tensor core: A row t = the 8
+    // (scale, min) halves of token t, B = (0, Q_g) per (scale, min) pair
+    float u[4] = {0.f, 0.f, 0.f, 0.f};
+    {
+      const uint32_t w0 = *reinterpret_cast<const uint32_t*>(st + OPTR_K_META_OFFSET + g * 16 + 4 * c);
+      const uint32_t w1 = *reinterpret_cast<const uint32_t*>(st + OPTR_K_META_OFFSET + (g + 8) * 16 + 4 * c);
+      mma16816(u, w0, w1, 0u, 0u, bmin, 0u);
+    }
+    float t0 = 0.f, t1 = 0.f;
+#pragma unroll
+    for (int G = 0; G < kGroups; ++G) {
+      const float a = __low2float(*reinterpret_cast<const __half2*>(&kmv0[G]));   // scale, token g
+      const float bb = __low2float(*reinterpret_cast<const __half2*>(&kmv1[G]));  // token g+8
+      t0 = fmaf(a, s_acc[G][0] + s_acc[G][1], t0);
+      t1 = fmaf(bb, s_acc[G][2] + s_acc[G][3], t1);
+    }
+    sc0 = fmaf(inv_s, t0, u[0] + u[1]);
+    sc1 = fmaf(inv_s, t1, u[2] + u[3]);
+  };
+
+  // value (scale, min) halves of tokens g (vm[0..3]) and g+8 (vm[4..7])
+  // per group, kept packed; returns their largest scale
+  auto vmeta = [&](const uint8_t* st, uint32_t (&vm)[2 * kGroups]) {
+    const uint4 m0 = *reinterpret_cast<const uint4*>(st + OPTR_V_META_OFFSET + g * 16);
+    const uint4 m1 = *reinterpret_cast<const uint4*>(st + OPTR_V_META_OFFSET + (g + 8) * 16);
+    vm[0] = m0.x; vm[1] = m0.y; vm[2] = m0.z; vm[3] = m0.w;
+    vm[4] = m1.x; vm[5] = m1.y; vm[6] = m1.z; vm[7] = m1.w;
+    __half2 mx = *reinterpret_cast<const __half2*>(&vm[0]);
+#pragma unroll
+    for (int i = 1; i < 2 * kGroups; ++i) mx = __hmax2(mx, *reinterpret_cast<const __half2*>(&vm[i]));
+    return __low2float(mx);  // scales are >= 0 (fp16 max ignores a NaN min half)
+  };
+
+  // Lazy reference: p = 2^(l - m_ref) with m_ref = m_lazy + k_s - 15,
+  // where m_lazy lies kLazyTau (log2 units) above the head's running
+  // maximum logit and 2^k_s bounds every value scale seen.  Then
+  // p * scale <= 2^15 always fits fp16, and the largest products sit near
+  // 2^15, so their fp16 lo parts stay normal whatever the magnitude of the
+  // values.  m_lazy and k_s move only when a logit exceeds m_lazy or a
+  // scale exceeds 2^k_s; each lane tests its own tokens, and only then are
+  // the head maxima reduced over the 8 lanes of the head and the
+  // accumulators rescaled.
+  auto reference = [&](float lmax, float smax) {
+    if (__any_sync(0xffffffffu, lmax > m_lazy || smax > s_cap)) {
+      float tmax = lmax, smx = smax;
+#pragma unroll
+      for (int o = 4; o < 32; o <<= 1) {
+        tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, o));
+        smx = fmaxf(smx, __shfl_xor_sync(0xffffffffu, smx, o));
+      }
+      // uniform over the lanes of head c
+      if (tmax > m_lazy) m_lazy = tmax + kLazyTau;
+      if (smx > s_cap) {
+        k_s = ilogbf(smx) + 1;  // smx < 2^k_s
+        s_cap = ldexpf(1.f, k_s);
+      }
+      const float m_new = m_lazy + (float)(k_s - 15);
+      if (m_new != m_ref) {
+        const float alpha = (m_ref == -INFINITY) ? 0.f : ex2(m_ref - m_new);
+        l_lane *= alpha;
+#pragma unroll
+        for (int G = 0; G < kGroups; ++G) {
+          mv[G] *= alpha;
+#pragma unroll
+          for (int hf = 0; hf < 2; ++hf)
+#pragma unroll
+            for (int k = 0; k < 4; ++k) acc_o[G][hf][k] *= alpha;
+        }
+        m_ref = m_new;
+      }
+    }
+  };
+
+  // value-side B operands p * scale (hi, lo) into pt, min terms into mv
+  auto vprod = [&](float p0, float p1, const uint32_t (&vm)[2 * kGroups],
+                   uint32_t (&pt)[kGroups][kPage][4]) {
+#pragma unroll
+    for (int G = 0; G < kGroups; ++G) {
+      const float2 va = h2f(vm[G]), vb = h2f(vm[kGroups + G]);  // tokens g, g+8
+      // the MMA sees centered codes (code - 1.5): the min term carries
+      // min + 1.5 * scale
+      const float ps0 = p0 * va.x, ps1 = p1 * vb.x;
+      mv[G] = fmaf(1.5f, ps0, fmaf(p0, va.y, fmaf(1.5f, ps1, fmaf(p1, vb.y, mv[G]))));
+      pt[G][g][c] = split_hilo(ps0);
+      pt[G][g + 8][c] = split_hilo(ps1);
+    }
+  };
+
+  // P.V of the page at st with the B operands in pt (after a __syncwarp)
+  auto vcodes = [&](const uint8_t* st, uint32_t (&pt)[kGroups][kPage][4]) {
+    uint32_t bv[kGroups][2];
+    {
+      // lanes 0-7 address rows 0-7 of group G, 8-15 rows 8-15, 16-31 the
+      // same for group G+1
+      const int r = lane & 15, gsel = lane >> 4;
+      ldsm_x4_trans(bv[0][0], bv[0][1], bv[1][0], bv[1][1], &pt[gsel][r][0]);
+      ldsm_x4_trans(bv[2][0], bv[2][1], bv[3][0], bv[3][1], &pt[2 + gsel][r][0]);
+    }
+    const uint8_t* vc = st + OPTR_V_CODES_OFFSET + 4 * g;
+    const uint32_t x0 = *reinterpret_cast<const uint32_t*>(vc + (2 * c) * 32);
+    const uint32_t x1 = *reinterpret_cast<const uint32_t*>(vc + (2 * c + 1) * 32);
+    const uint32_t x2 = *reinterpret_cast<const uint32_t*>(vc + (2 * c + 8) * 32);
+    const uint32_t x3 = *reinterpret_cast<const uint32_t*>(vc + (2 * c + 9) * 32);
+    const uint32_t a01 = __byte_perm(x0, x1, 0x5410), a23 = __byte_perm(x0, x1, 0x7632);
+    const uint32_t b01 = __byte_perm(x2, x3, 0x5410), b23 = __byte_perm(x2, x3, 0x7632);
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {  // groups 2j, 2j+1
+      uint32_t fa[2][4], fb[2][4];  // tokens (2c, 2c+1), (2c+8, 2c+9)
+      code_fields(j ? a23 : a01, e1024, fa);
+      code_fields(j ? b23 : b01, e1024, fb);
+#pragma unroll
+      for (int par = 0; par < 2; ++par) {
+        const int G = 2 * j + par;
+        mma16816(acc_o[G][0], centered(fa[par][0], par, 0), centered(fa[par][1], par, 1),
+                 centered(fb[par][0], par, 0), centered(fb[par][1], par, 1),
+                 bv[G][0], bv[G][1]);
+        mma16816(acc_o[G][1], centered(fa[par][2], par, 2), centered(fa[par][3], par, 3),
+                 centered(fb[par][2], par, 2), centered(fb[par][3], par, 3),
+                 bv[G][0], bv[G][1]);
+      }
+    }
+  };
+
+  // One page on its own (segment starts, partial pages).  FULL = all 16
+  // tokens valid (no masking code).
   auto page = [&](const uint8_t* st, int nvalid, auto full_tag) {
     constexpr bool FULL = decltype(full_tag)::value;
     const bool v0 = FULL || g < nvalid, v1 = FULL || g + 8 < nvalid;
-    // ------------------------------------------------------------ logits
     float sc0, sc1;
-    {
-      const uint2 k0 = *reinterpret_cast<const uint2*>(st + OPTR_K_CODES_OFFSET + g * 32 + 8 * c);
-      const uint2 k1 = *reinterpret_cast<const uint2*>(st + OPTR_K_CODES_OFFSET + (g + 8) * 32 + 8 * c);
-      // bytes [G0 w2c, G1 w2c, G0 w2c+1, G1 w2c+1] and the same for G2/G3
-      const uint32_t y01_0 = __byte_perm(k0.x, k0.y, 0x5410);
-      const uint32_t y23_0 = __byte_perm(k0.x, k0.y, 0x7632);
-      const uint32_t y01_1 = __byte_perm(k1.x, k1.y, 0x5410);
-      const uint32_t y23_1 = __byte_perm(k1.x, k1.y, 0x7632);
-      float s_acc[kGroups][4];
-#pragma unroll
-      for (int j = 0; j < 2; ++j) {  // groups 2j, 2j+1
-        uint32_t f0[2][4], f1[2][4];  // token rows g, g+8
-        code_fields(j ? y23_0 : y01_0, e1024, f0);
-        code_fields(j ? y23_1 : y01_1, e1024, f1);
-#pragma unroll
-        for (int par = 0; par < 2; ++par) {
-          const int G = 2 * j + par;
-          mma16816_c(s_acc[G], f0[par][0], f1[par][0], f0[par][1], f1[par][1],
-                     bq[G][0][0], bq[G][0][1], kneg[G][0], kneg[G][1]);
-          mma16816(s_acc[G], f0[par][2], f1[par][2], f0[par][3], f1[par][3],
-                   bq[G][1][0], bq[G][1][1]);
-        }
-      }
-      const uint4 km0 = *reinterpret_cast<const uint4*>(st + OPTR_K_META_OFFSET + g * 16);
-      const uint4 km1 = *reinterpret_cast<const uint4*>(st + OPTR_K_META_OFFSET + (g + 8) * 16);
-      const uint32_t kmv0[4] = {km0.x, km0.y, km0.z, km0.w};
-      const uint32_t kmv1[4] = {km1.x, km1.y, km1.z, km1.w};
-      // sum_g min_g * sum(q' over g) on the tensor core: A row t = the 8
-      // (scale, min) halves of token t, B = (0, Q_g) per (scale, min) pair
-      float u[4] = {0.f, 0.f, 0.f, 0.f};
-      {
-        const uint32_t w0 = *reinterpret_cast<const uint32_t*>(st + OPTR_K_META_OFFSET + g * 16 + 4 * c);
-        const uint32_t w1 = *reinterpret_cast<const uint32_t*>(st + OPTR_K_META_OFFSET + (g + 8) * 16 + 4 * c);
-        mma16816(u, w0, w1, 0u, 0u, bmin, 0u);
-      }
-      float t0 = 0.f, t1 = 0.f;
+    logits(st, sc0, sc1);
+    uint32_t vm[2 * kGroups];
+    if (!FULL) {
+      // masked tokens have p = 0 and their (possibly garbage) metadata is
+      // zeroed before it is read, so it is never multiplied in
+      sc0 = v0 ? sc0 : -INFINITY;
+      sc1 = v1 ? sc1 : -INFINITY;
+    }
+    float smax = vmeta(st, vm);
+    if (!FULL) {
 #pragma unroll
       for (int G = 0; G < kGroups; ++G) {
-        const float a = __low2float(*reinterpret_cast<const __half2*>(&kmv0[G]));   // scale, token g
-        const float bb = __low2float(*reinterpret_cast<const __half2*>(&kmv1[G]));  // token g+8
-        t0 = fmaf(a, s_acc[G][0] + s_acc[G][1], t0);
-        t1 = fmaf(bb, s_acc[G][2] + s_acc[G][3], t1);
+        vm[G] = v0 ? vm[G] : 0u;
+        vm[kGroups + G] = v1 ? vm[kGroups + G] : 0u;
       }
-      sc0 = fmaf(inv_s, t0, u[0] + u[1]);
-      sc1 = fmaf(inv_s, t1, u[2] + u[3]);
-      if (!FULL) {
-        sc0 = v0 ? sc0 : -INFINITY;
-        sc1 = v1 ? sc1 : -INFINITY;
-      }
+      __half2 mx = *reinterpret_cast<const __half2*>(&vm[0]);
+#pragma unroll
+      for (int i = 1; i < 2 * kGroups; ++i) mx = __hmax2(mx, *reinterpret_cast<const __half2*>(&vm[i]));
+      smax = __low2float(mx);
     }
-    // ------------------------------------------- value metadata, softmax
-    const uint4 vm0 = *reinterpret_cast<const uint4*>(st + OPTR_V_META_OFFSET + g * 16);
-    const uint4 vm1 = *reinterpret_cast<const uint4*>(st + OPTR_V_META_OFFSET + (g + 8) * 16);
-    const uint32_t vmv0[4] = {vm0.x, vm0.y, vm0.z, vm0.w};
-    const uint32_t vmv1[4] = {vm1.x, vm1.y, vm1.z, vm1.w};
-    float2 va[kGroups], vb[kGroups];  // (scale, min) of tokens g, g+8
-    float smax = 0.f;
-#pragma unroll
-    for (int G = 0; G < kGroups; ++G) {
-      va[G] = h2f(vmv0[G]);
-      vb[G] = h2f(vmv1[G]);
-      if (!FULL) {
-        // masked tokens have p = 0; their (possibly garbage) metadata is
-        // never multiplied in
-        va[G] = v0 ? va[G] : make_float2(0.f, 0.f);
-        vb[G] = v1 ? vb[G] : make_float2(0.f, 0.f);
-      }
-      smax = fmaxf(smax, fmaxf(va[G].x, vb[G].x));
-    }
-    // Lazy reference: p = 2^(l - m_ref) with m_ref = m_lazy + k_s - 15,
-    // where m_lazy lies kLazyTau (log2 units) above the head's running
-    // maximum logit and 2^k_s bounds every value scale seen.  Then
-    // p * scale <= 2^15 always fits fp16, and the largest products sit near
-    // 2^15, so their fp16 lo parts stay normal whatever the magnitude of the
-    // values.  m_lazy and k_s move only when a logit exceeds m_lazy or a
-    // scale exceeds 2^k_s; each lane tests its own tokens, and only then are
-    // the head maxima reduced over the 8 lanes of the head and the
-    // accumulators rescaled.
-    {
-      const float lmax = fmaxf(sc0, sc1);
-      if (__any_sync(0xffffffffu, lmax > m_lazy || smax > s_cap)) {
-        float tmax = lmax, smx = smax;
-#pragma unroll
-        for (int o = 4; o < 32; o <<= 1) {
-          tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, o));
-          smx = fmaxf(smx, __shfl_xor_sync(0xffffffffu, smx, o));
-        }
-        // uniform over the lanes of head c
-        if (tmax > m_lazy) m_lazy = tmax + kLazyTau;
-        if (smx > s_cap) {
-          k_s = ilogbf(smx) + 1;  // smx < 2^k_s
-          s_cap = ldexpf(1.f, k_s);
-        }
-        const float m_new = m_lazy + (float)(k_s - 15);
-        if (m_new != m_ref) {
-          const float alpha = (m_ref == -INFINITY) ? 0.f : ex2(m_ref - m_new);
-          l_lane *= alpha;
-#pragma unroll
-          for (int G = 0; G < kGroups; ++G) {
-            mv[G] *= alpha;
-#pragma unroll
-            for (int hf = 0; hf < 2; ++hf)
-#pragma unroll
-              for (int k = 0; k < 4; ++k) acc_o[G][hf][k] *= alpha;
-          }
-          m_ref = m_new;
-        }
-      }
-    }
+    reference(fmaxf(sc0, sc1), smax);
     float p0 = ex2(sc0 - m_ref), p1 = ex2(sc1 - m_ref);  // ex2(-inf) = 0
     if (!FULL) {  // a fully masked page before any finite max: -inf - -inf
       p0 = v0 ? p0 : 0.f;
       p1 = v1 ? p1 : 0.f;
     }
     l_lane += p0 + p1;
-    // ------------------------------------------------------------ values
-#pragma unroll
-    for (int G = 0; G < kGroups; ++G) {
-      // the MMA sees centered codes (code - 1.5): the min term carries
-      // min + 1.5 * scale
-      const float ps0 = p0 * va[G].x, ps1 = p1 * vb[G].x;
-      mv[G] = fmaf(1.5f, ps0, fmaf(p0, va[G].y, fmaf(1.5f, ps1, fmaf(p1, vb[G].y, mv[G]))));
-      S.pt[G][g][c] = split_hilo(ps0);
-      S.pt[G][g + 8][c] = split_hilo(ps1);
-    }
+    vprod(p0, p1, vm, S.pt[0]);
     __syncwarp();
-    uint32_t bv[kGroups][2];
-    {
-      // lanes 0-7 address rows 0-7 of group G, 8-15 rows 8-15, 16-31 the
-      // same for group G+1
-      const int r = lane & 15, gsel = lane >> 4;
-      ldsm_x4_trans(bv[0][0], bv[0][1], bv[1][0], bv[1][1], &S.pt[gsel][r][0]);
-      ldsm_x4_trans(bv[2][0], bv[2][1], bv[3][0], bv[3][1], &S.pt[2 + gsel][r][0]);
-    }
-    {
-      const uint8_t* vc = st + OPTR_V_CODES_OFFSET + 4 * g;
-      const uint32_t x0 = *reinterpret_cast<const uint32_t*>(vc + (2 * c) * 32);
-      const uint32_t x1 = *reinterpret_cast<const uint32_t*>(vc + (2 * c + 1) * 32);
-      const uint32_t x2 = *reinterpret_cast<const uint32_t*>(vc + (2 * c + 8) * 32);
-      const uint32_t x3 = *reinterpret_cast<const uint32_t*>(vc + (2 * c + 9) * 32);
-      const uint32_t a01 = __byte_perm(x0, x1, 0x5410), a23 = __byte_perm(x0, x1, 0x7632);
-      const uint32_t b01 = __byte_perm(x2, x3, 0x5410), b23 = __byte_perm(x2, x3, 0x7632);
-#pragma unroll
-      for (int j = 0; j < 2; ++j) {  // groups 2j, 2j+1
-        uint32_t fa[2][4], fb[2][4];  // tokens (2c, 2c+1), (2c+8, 2c+9)
-        code_fields(j ? a23 : a01, e1024, fa);
-        code_fields(j ? b23 : b01, e1024, fb);
-#pragma unroll
-        for (int par = 0; par < 2; ++par) {
-          const int G = 2 * j + par;
-          mma16816(acc_o[G][0], centered(fa[par][0], par, 0), centered(fa[par][1], par, 1),
-                   centered(fb[par][0], par, 0), centered(fb[par][1], par, 1),
-                   bv[G][0], bv[G][1]);
-          mma16816(acc_o[G][1], centered(fa[par][2], par, 2), centered(fa[par][3], par, 3),
-                   centered(fb[par][2], par, 2), centered(fb[par][3], par, 3),
-                   bv[G][0], bv[G][1]);
-        }
-      }
-    }
+    vcodes(st, S.pt[0]);
   };
 
-  static_assert((kStages & (kStages - 1)) == 0, "kStages: a power of two");
-  const int total = f1 - f0;
-#pragma unroll 1
-  for (int done = 0; done < total; ++done) {
-    const int s = done & (kStages - 1);
-    issue((s + kStages - 1) & (kStages - 1));
-    cp_async_wait<kStages - 1>();
+  // Two full pages of the current segment: the same steps with the two
+  // pages' independent work interleaved and one softmax update.
+  auto page_pair = [&](const uint8_t* sa, const uint8_t* sb) {
+    float a0, a1, b0, b1;
+    logits(sa, a0, a1);
+    logits(sb, b0, b1);
+    uint32_t vma[2 * kGroups], vmb[2 * kGroups];
+    const float smax = fmaxf(vmeta(sa, vma), vmeta(sb, vmb));
+    reference(fmaxf(fmaxf(a0, a1), fmaxf(b0, b1)), smax);
+    const float pa0 = ex2(a0 - m_ref), pa1 = ex2(a1 - m_ref);
+    const float pb0 = ex2(b0 - m_ref), pb1 = ex2(b1 - m_ref);
+    l_lane += (pa0 + pa1) + (pb0 + pb1);
+    vprod(pa0, pa1, vma, S.pt[0]);
+    vprod(pb0, pb1, vmb, S.pt[1]);
     __syncwarp();
+    vcodes(sa, S.pt[0]);
+    vcodes(sb, S.pt[1]);
+  };
+
+  // one staged page through the segment bookkeeping
+  auto single = [&](int s) {
     const int2 inf = S.info[s];
-    const int nvalid = inf.y;
     if (inf.x != cur_key) {
       if (cur_key >= 0) flush();
       begin_segment(inf.x);
     }
-    if (nvalid == kPage)
-      page(S.stage[s], nvalid, std::true_type{});
+    if (inf.y == kPage)
+      page(S.stage[s], inf.y, std::true_type{});
     else
-      page(S.stage[s], nvalid, std::false_type{});
+      page(S.stage[s], inf.y, std::false_type{});
     __syncwarp();
+  };
+
+  // Pages go through the stages in pairs: pair q (stages 2q, 2q+1) is
+  // processed while the other pair is in flight.
+  static_assert(kStages == 4, "two pairs of stages");
+  const int total = f1 - f0;
+#pragma unroll 1
+  for (int done = 0; done < total; done += 2) {
+    const int q = (done >> 1) & 1;
+    issue_pair(1 - q);
+    cp_async_wait<1>();
+    __syncwarp();
+    const int2 ia = S.info[2 * q], ib = S.info[2 * q + 1];
+    if (done + 1 < total && ia.x == cur_key && ib.x == cur_key && ia.y == kPage &&
+        ib.y == kPage) {
+      page_pair(S.stage[2 * q], S.stage[2 * q + 1]);
+      __syncwarp();
+    } else {
+      single(2 * q);
+      if (done + 1 < total) single(2 * q + 1);
+    }
   }
   flush();
 }
