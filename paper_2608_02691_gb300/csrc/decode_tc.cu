@@ -191,6 +191,32 @@ __device__ __forceinline__ void load_chunk(PageChunk& ch, int base, int f1,
   }
 }
 
+// spref[b] = pages of sequences < b (b <= B <= kPrefCache; invalid lengths
+// count as empty), by one block-wide scan; ends with __syncthreads().
+__device__ __noinline__ void page_prefix(const int32_t* __restrict__ seq_lens,
+                                         int B, int max_pages, int* spref,
+                                         int* wsum) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  int np = 0;
+  if ((int)threadIdx.x < B) {
+    const int len = __ldg(seq_lens + threadIdx.x);
+    if (len >= 0 && (long long)len <= (long long)max_pages * kPage) np = (len + kPage - 1) / kPage;
+  }
+  int x = np;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) wsum[warp] = x;
+  __syncthreads();
+  int off = 0;
+  for (int i = 0; i < warp; ++i) off += wsum[i];
+  if ((int)threadIdx.x < B) spref[threadIdx.x + 1] = off + x;
+  if (threadIdx.x == 0) spref[0] = 0;
+  __syncthreads();
+}
+
 __global__ void __launch_bounds__(kWarps * 32, 1)
 partial_tensor_kernel(const uint8_t* __restrict__ pool,
                       const int32_t* __restrict__ bt,
@@ -209,23 +235,36 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
   extern __shared__ __align__(16) unsigned char dsm_[];
   WarpSmemTC* smem = reinterpret_cast<WarpSmemTC*>(dsm_);  // [kWarps]
   __shared__ int spref[kPrefCache + 1];
-  pdl_wait();
-  pdl_trigger();
+  __shared__ int wsum[kWarps];
   uint32_t e1024;
   asm volatile("mov.b32 %0, 0x64006400;" : "=r"(e1024));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int g = lane >> 2, c = lane & 3;
   WarpSmemTC& S = smem[warp];
   const int w = blockIdx.x * kWarps + warp;
-  const int F = __ldcg(pref + B) * h_kv;
-  const int f0 = (int)((long long)w * F / W), f1 = (int)((long long)(w + 1) * F / W);
 
-  // first segment of this warp: sequence b with pref[b]*h_kv <= f0
+  // Page prefix sums.  For up to kPrefCache sequences the CTA scans the
+  // lengths itself (the values qrot writes to pref for the combine): the
+  // lengths, the block table and the pool are inputs, complete before qrot
+  // began (qrot passes its pdl_wait() before it lets this grid launch), so
+  // the page tables and the first page copies are set up before this grid's
+  // own pdl_wait(), overlapping qrot; only the query fragments wait.
   const bool cached = B <= kPrefCache;
-  if (cached)
-    for (int i = threadIdx.x; i <= B; i += kWarps * 32) spref[i] = __ldcg(pref + i);
-  __syncthreads();
-  if (f0 >= f1) return;
+  static_assert(kPrefCache < kWarps * 32, "one thread per sequence");
+  int F;
+  if (cached) {
+    page_prefix(seq_lens, B, max_pages, spref, wsum);
+    F = spref[B] * h_kv;
+  } else {
+    pdl_wait();
+    F = __ldcg(pref + B) * h_kv;
+  }
+  const int f0 = (int)((long long)w * F / W), f1 = (int)((long long)(w + 1) * F / W);
+  if (f0 >= f1) {
+    pdl_wait();
+    pdl_trigger();
+    return;
+  }
   PageChunk chk;
   int f_issue = f0;
   load_chunk(chk, f0, f1, pref, spref, cached, seq_lens, bt, B, h_kv,
@@ -260,6 +299,8 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
     cp_async_commit();
   };
   issue_pair(0);
+  pdl_wait();  // (returns at once when already passed above)
+  pdl_trigger();
 
   // per-segment state
   uint32_t bq[kGroups][2][2];  // query B fragments [group][kk][reg]
