@@ -48,6 +48,11 @@ struct WarpSmemTC {
   alignas(16) uint8_t stage[kStages][kChunk];
   alignas(16) uint32_t pt[2][kGroups][kPage][4];  // p*scale_v (hi, lo) per head, 2 pages
   int2 info[kStages];  // per staged page: (segment key b*h_kv+h, valid tokens)
+  // per segment, per lane (kept here, not in registers, so that the page
+  // loop has registers to spare): query B fragments, and the key MMAs'
+  // start values (-offset hi, -offset lo) twice, in accumulator order
+  uint4 qfr[kGroups][32];
+  float4 kq[kGroups][32];
 };
 
 constexpr int kPrefCache = 256;  // sequences whose page prefix sums a CTA caches
@@ -60,18 +65,6 @@ __device__ __forceinline__ void mma16816(float* d, uint32_t a0, uint32_t a1,
       "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};\n"
       : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
       : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
-}
-
-// d = a * b + (c0, c1, c0, c1): the first MMA of a chain, started from a
-// per-column value instead of the accumulator.
-__device__ __forceinline__ void mma16816_c(float* d, uint32_t a0, uint32_t a1,
-                                           uint32_t a2, uint32_t a3, uint32_t b0,
-                                           uint32_t b1, float c0, float c1) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 "
-      "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%10,%11,%10,%11};\n"
-      : "=f"(d[0]), "=f"(d[1]), "=f"(d[2]), "=f"(d[3])
-      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1), "f"(c0), "f"(c1));
 }
 
 __device__ __forceinline__ void ldsm_x4_trans(uint32_t& r0, uint32_t& r1,
@@ -303,8 +296,6 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
   pdl_trigger();
 
   // per-segment state
-  uint32_t bq[kGroups][2][2];  // query B fragments [group][kk][reg]
-  float kneg[kGroups][2];      // minus the key-code offset sums, head c
   uint32_t bmin = 0;           // key min-term B fragment (sum q' per group)
   float inv_s = 0.f;           // 1 / prescale of head c
   float acc_o[kGroups][2][4];  // values: [group][half][c-frag]
@@ -353,19 +344,16 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
 #pragma unroll
     for (int G = 0; G < kGroups; ++G) {
       const uint4 v = __ldcg(fq + G);
-      bq[G][0][0] = v.x;
-      bq[G][0][1] = v.y;
-      bq[G][1][0] = v.z;
-      bq[G][1][1] = v.w;
+      S.qfr[G][lane] = v;
     }
     {
       const float4* ko = reinterpret_cast<const float4*>(
           koff + ((size_t)cb * h_kv + ch) * 32 + c * 8);
       const float4 k01 = __ldcg(ko), k23 = __ldcg(ko + 1);
-      kneg[0][0] = -k01.x; kneg[0][1] = -k01.y;
-      kneg[1][0] = -k01.z; kneg[1][1] = -k01.w;
-      kneg[2][0] = -k23.x; kneg[2][1] = -k23.y;
-      kneg[3][0] = -k23.z; kneg[3][1] = -k23.w;
+      S.kq[0][lane] = make_float4(-k01.x, -k01.y, -k01.x, -k01.y);
+      S.kq[1][lane] = make_float4(-k01.z, -k01.w, -k01.z, -k01.w);
+      S.kq[2][lane] = make_float4(-k23.x, -k23.y, -k23.x, -k23.y);
+      S.kq[3][lane] = make_float4(-k23.z, -k23.w, -k23.z, -k23.w);
     }
     const size_t row = (size_t)cb * h_q + 4 * ch + c;
     {
@@ -410,10 +398,11 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
 #pragma unroll
       for (int par = 0; par < 2; ++par) {
         const int G = 2 * j + par;
-        mma16816_c(s_acc[G], f0[par][0], f1[par][0], f0[par][1], f1[par][1],
-                   bq[G][0][0], bq[G][0][1], kneg[G][0], kneg[G][1]);
-        mma16816(s_acc[G], f0[par][2], f1[par][2], f0[par][3], f1[par][3],
-                 bq[G][1][0], bq[G][1][1]);
+        const uint4 qv = S.qfr[G][lane];
+        const float4 kv = S.kq[G][lane];
+        s_acc[G][0] = kv.x; s_acc[G][1] = kv.y; s_acc[G][2] = kv.z; s_acc[G][3] = kv.w;
+        mma16816(s_acc[G], f0[par][0], f1[par][0], f0[par][1], f1[par][1], qv.x, qv.y);
+        mma16816(s_acc[G], f0[par][2], f1[par][2], f0[par][3], f1[par][3], qv.z, qv.w);
       }
     }
     const uint4 km0 = *reinterpret_cast<const uint4*>(st + OPTR_K_META_OFFSET + g * 16);
