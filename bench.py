@@ -217,8 +217,10 @@ def run_ours(args, rank, world, dev):
     stream = torch.cuda.current_stream()
 
     def step():
-        optr.optr_kv_append(p, k_new, v_new, cu_new, pos0, bt, pool)
-        optr.optr_decode_attention(p, q, bt, seq, pool, out, ws)
+        # the cache write of the step's new tokens, then decode over the
+        # updated cache (optr_kv_append + optr_decode_attention in one call)
+        optr.optr_decode_step(p, q, k_new, v_new, cu_new, pos0, bt, seq, pool,
+                              out, ws)
 
     step_bytes = (decode_bytes(case["seq_lens"].tolist(), h_kv, h_q) +
                   append_bytes(k_new.shape[0], h_kv))
@@ -303,8 +305,8 @@ def e2e_time(args, case, p, pool, bt, seq, cu_new, pos0, out, ws, flush,
         q_d.copy_(q_h, non_blocking=True)
         k_d.copy_(k_h, non_blocking=True)
         v_d.copy_(v_h, non_blocking=True)
-        optr.optr_kv_append(p, k_d, v_d, cu_new, pos0, bt, pool)
-        optr.optr_decode_attention(p, q_d, bt, seq, pool, out, ws)
+        optr.optr_decode_step(p, q_d, k_d, v_d, cu_new, pos0, bt, seq, pool,
+                              out, ws)
         out_h.copy_(out, non_blocking=True)
 
     for _ in range(args.warmup):
@@ -574,7 +576,10 @@ def main():
                        "bytes_per_step": m["bytes"], "l2": "flushed (512 MiB write) "
                        "before every timed step; step timed alone with CUDA events",
                        "decode_variant": args.variant, "append_variant": args.append_variant},
-            "gpu_launches": 4 * args.steps,
+            # optr_decode_step: fused cache write + query rotation, partial,
+            # combine (4 launches when a CUDA-core variant is selected)
+            "gpu_launches": (3 if args.variant != 1 and args.append_variant != 1
+                             else 4) * args.steps,
             "stage_ms": {k: round(v, 5) for k, v in m["stage_ms"].items()},
             "roofline": m["roofline"],
             "e2e": None if e2e is None else {

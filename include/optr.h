@@ -227,6 +227,27 @@ optr_status optr_decode_attention(const optr_params* p, const void* q,
                                   size_t ws_bytes, cudaStream_t stream);
 
 /*
+ * One decode step: optr_kv_append(p, k, v, n_tok, cu_new, pos0, ...) of the
+ * step's new tokens followed by optr_decode_attention(p, q, ...) over the
+ * updated cache, with the same arguments, layouts, results and errors
+ * (seq_lens counts the new tokens).  The paper's serving loop writes each
+ * new token's rotated INT2 record and then attends over the cache (Sec. 4.1;
+ * Appendix, key-mean estimation and rotated-query implementation); the two
+ * first launches of that pair are independent (the cache write does not
+ * touch the query), so for decode-step sized writes (n_tok <= 256) with the
+ * default variants they run as one launch.  Other cases run exactly as the
+ * two calls.  No allocation, no synchronisation.
+ */
+optr_status optr_decode_step(const optr_params* p, const void* q,
+                             const void* k, const void* v, int n_tok,
+                             const int32_t* cu_new, const int32_t* pos0,
+                             const int32_t* block_table,
+                             const int32_t* seq_lens, int B, int max_pages,
+                             uint8_t* pool, int num_pages, float* out,
+                             void* workspace, size_t ws_bytes,
+                             cudaStream_t stream);
+
+/*
  * Read and clear the device error word of p (OPTR_DEVERR_* bits).
  * Synchronises the device.  *flags receives 0 when no kernel reported a
  * table error since the last call.
@@ -235,9 +256,11 @@ optr_status optr_device_error(const optr_params* p, uint32_t* flags);
 
 /*
  * Stage timing for measurement (off by default).  optr_profile_enable(p, 1)
- * creates library-owned CUDA events; afterwards every optr_kv_append and
- * optr_decode_attention call made with p records an event on its stream
- * before and after each kernel it launches.  optr_profile_last waits for the
+ * creates library-owned CUDA events; afterwards every optr_kv_append,
+ * optr_decode_attention and optr_decode_step call made with p records an
+ * event on its stream before and after each kernel it launches (for the
+ * step's fused first launch the append stage covers it and the query
+ * rotation stage is empty).  optr_profile_last waits for the
  * most recent calls' events and returns their durations in milliseconds:
  *   ms[0] append kernel, ms[1] query rotation + plan, ms[2] split-K partial,
  *   ms[3] combine (a stage that did not run reports 0).

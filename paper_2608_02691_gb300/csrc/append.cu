@@ -5,6 +5,7 @@
 #include "optr_internal.cuh"
 #include "quant.cuh"
 #include "append_common.cuh"
+#include "append_small.cuh"
 
 namespace optr {
 namespace {
@@ -103,14 +104,7 @@ append_cuda_core_kernel(const __nv_bfloat16* __restrict__ k,
   }
 }
 
-// Decode-step variant for few new tokens (one per sequence per step): one
-// CTA per (tile of 16 tokens, KV head, K or V), 512 threads = 4 slices x 128
-// channels.  Slice s accumulates z_j over i in [32s, 32s+32) for all 16
-// tokens; the slices are added in shared memory, then warp t quantizes and
-// packs token t group by group.
-constexpr int kSmallTok = 16;
-constexpr int kSmallCuCache = 512;   // sequences whose cu_new / pos0 a CTA caches
-
+// Decode-step variant for few new tokens: append_small.cuh.
 __global__ void __launch_bounds__(512)
 append_small_kernel(const __nv_bfloat16* __restrict__ k,
                     const __nv_bfloat16* __restrict__ v, int n_tok,
@@ -122,95 +116,10 @@ append_small_kernel(const __nv_bfloat16* __restrict__ k,
                     const float* __restrict__ R_v,
                     const float* __restrict__ muR, float clip_k, float clip_v,
                     unsigned* err) {
-  constexpr int T = kSmallTok;
-  __shared__ float xs[T][kD];
-  __shared__ float zp[4][T][kD];
-  __shared__ long long dst[T];
-  __shared__ int dslot[T];
-  __shared__ int s_cu[kSmallCuCache + 1];
-  __shared__ int s_p0[kSmallCuCache];
-  const int h = blockIdx.y, kind = blockIdx.z;
-  const int t0 = blockIdx.x * T;
-  const int tid = threadIdx.x;
-  const int sl = tid >> 7, j = tid & 127;
-  // rotation column first (independent of everything else): all in flight
-  const float* R = (kind ? R_v : R_k) + (size_t)h * kD * kD + (size_t)(32 * sl) * kD + j;
-  float rv[32];
-#pragma unroll
-  for (int i = 0; i < 32; ++i) rv[i] = __ldg(R + i * kD);
-  float musub[kGroups];  // mu R_k of this lane's channel in each group (keys)
-#pragma unroll
-  for (int g = 0; g < kGroups; ++g)
-    musub[g] = kind ? 0.f : __ldg(muR + h * kD + 32 * g + (tid & 31));
-  pdl_wait();  // inputs and the pool may come from earlier kernels
-  pdl_trigger();
-  const __nv_bfloat16* src = kind ? v : k;
-  for (int idx = tid; idx < T * kD; idx += 512) {
-    const int t = idx >> 7, i = idx & 127;
-    const int tok = t0 + t;
-    xs[t][i] = tok < n_tok ? __bfloat162float(src[((size_t)tok * h_kv + h) * kD + i]) : 0.f;
-  }
-  const bool cached = B <= kSmallCuCache;
-  if (cached) {
-    for (int i = tid; i <= B; i += 512) {
-      s_cu[i] = __ldg(cu_new + i);
-      if (i < B) s_p0[i] = __ldg(pos0 + i);
-    }
-    __syncthreads();
-  }
-  if (tid < T) {
-    const int tok = t0 + tid;
-    int slot = 0;
-    long long off = -1;
-    if (tok < n_tok)
-      off = cached ? resolve_slot_cached(tok, h, s_cu, s_p0, bt, B, max_pages,
-                                         num_pages, h_kv, &slot, err)
-                   : resolve_slot(tok, h, cu_new, pos0, bt, B, max_pages,
-                                  num_pages, h_kv, &slot, err);
-    dst[tid] = off;
-    dslot[tid] = slot;
-  }
-  __syncthreads();
-  float acc[T];
-#pragma unroll
-  for (int t = 0; t < T; ++t) acc[t] = 0.f;
-#pragma unroll
-  for (int i = 0; i < 32; ++i)
-#pragma unroll
-    for (int t = 0; t < T; ++t) acc[t] = fmaf(xs[t][32 * sl + i], rv[i], acc[t]);
-#pragma unroll
-  for (int t = 0; t < T; ++t) zp[sl][t][j] = acc[t];
-  __syncthreads();
-
-  const int warp = tid >> 5, lane = tid & 31;  // warp = token of the tile
-  const long long off = dst[warp];
-  if (t0 + warp >= n_tok || off < 0) return;
-  const int slot = dslot[warp];
-  const float clip = kind ? clip_v : clip_k;
-  const int codes_off = kind ? OPTR_V_CODES_OFFSET : OPTR_K_CODES_OFFSET;
-  const int meta_off = kind ? OPTR_V_META_OFFSET : OPTR_K_META_OFFSET;
-  uint8_t* chunk = pool + off;
-#pragma unroll
-  for (int g = 0; g < kGroups; ++g) {
-    const int jj = 32 * g + lane;
-    const float zsum = ((zp[0][warp][jj] + zp[1][warp][jj]) + zp[2][warp][jj]) + zp[3][warp][jj];
-    const float z = __fsub_rn(zsum, musub[g]);
-    float lo = z, hi = z;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, o));
-      hi = fmaxf(hi, __shfl_xor_sync(0xffffffffu, hi, o));
-    }
-    GroupQuant gq = group_quant_params(lo, hi, clip);
-    unsigned bits = (unsigned)quant_code(z, gq) << (2 * (lane & 3));
-    bits |= __shfl_xor_sync(0xffffffffu, bits, 1);
-    bits |= __shfl_xor_sync(0xffffffffu, bits, 2);
-    if ((lane & 3) == 0)
-      chunk[codes_off + slot * 32 + 4 * (lane >> 2) + g] = (uint8_t)bits;
-    if (lane == 0)
-      *reinterpret_cast<__half2*>(chunk + meta_off + slot * 16 + 4 * g) =
-          __halves2half2(gq.scale, gq.min);
-  }
+  __shared__ AppendSmallSmem sm;
+  append_small_body(blockIdx.x, blockIdx.y, blockIdx.z, sm, k, v, n_tok,
+                    cu_new, pos0, bt, B, max_pages, pool, num_pages, h_kv, R_k,
+                    R_v, muR, clip_k, clip_v, err);
 }
 
 }  // namespace

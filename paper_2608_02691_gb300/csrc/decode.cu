@@ -14,6 +14,7 @@
 // Logits are kept in the log2 domain: q' carries log2(e)/sqrt(d), so
 // softmax weights are exp2(l - m) (Sec. 3 Eq. 1 with the 1/sqrt(d) scale).
 #include "decode_common.cuh"
+#include "append_small.cuh"
 
 namespace optr {
 namespace {
@@ -27,22 +28,30 @@ constexpr float kLog2e = 1.4426950408889634f;
 // the group, the slices are added in shared memory.
 constexpr int kQrotThreads = 512;
 
-__global__ void __launch_bounds__(kQrotThreads)
-qrot_kernel(const __nv_bfloat16* __restrict__ q, const float* __restrict__ R_k,
-            int B, int h_q, int h_kv, float qscale,
-            const int32_t* __restrict__ seq_lens, int max_pages,
-            float* __restrict__ qf, float* __restrict__ qs,
-            uint32_t* __restrict__ frag, float* __restrict__ koff,
-            float* __restrict__ invs, int* __restrict__ pref,
-            int* __restrict__ nzpref, int* __restrict__ cnt_ws,
-            unsigned* err) {
-  __shared__ float qsm[4][kD];
-  __shared__ float part[4][4][kD];  // [slice][head][channel]
-  __shared__ float qrs[4][kD];
-  __shared__ float hmax[4][4];
-  __shared__ int warp_tot[2][kQrotThreads / 32];
-  __shared__ double koff_part[kQrotThreads / 32][kGroups];
-  const int b = blockIdx.x, h = blockIdx.y, tid = threadIdx.x;
+struct QrotSmem {
+  float qsm[4][kD];
+  float part[4][4][kD];  // [slice][head][channel]
+  float qrs[4][kD];
+  float hmax[4][4];
+  int warp_tot[2][kQrotThreads / 32];
+  double koff_part[kQrotThreads / 32][kGroups];
+};
+
+// CTA (b, h) of the query rotation; 512 threads.
+__device__ __forceinline__ void qrot_body(
+    int b, int h, QrotSmem& sm, const __nv_bfloat16* __restrict__ q,
+    const float* __restrict__ R_k, int B, int h_q, int h_kv, float qscale,
+    const int32_t* __restrict__ seq_lens, int max_pages,
+    float* __restrict__ qf, float* __restrict__ qs, uint32_t* __restrict__ frag,
+    float* __restrict__ koff, float* __restrict__ invs, int* __restrict__ pref,
+    int* __restrict__ nzpref, int* __restrict__ cnt_ws, unsigned* err) {
+  float (&qsm)[4][kD] = sm.qsm;
+  float (&part)[4][4][kD] = sm.part;
+  float (&qrs)[4][kD] = sm.qrs;
+  float (&hmax)[4][4] = sm.hmax;
+  int (&warp_tot)[2][kQrotThreads / 32] = sm.warp_tot;
+  double (&koff_part)[kQrotThreads / 32][kGroups] = sm.koff_part;
+  const int tid = threadIdx.x;
   const int sl = tid >> 7, j = tid & 127;
   const int warp = tid >> 5, lane = tid & 31;
   float acc[4] = {0.f, 0.f, 0.f, 0.f};
@@ -165,6 +174,57 @@ qrot_kernel(const __nv_bfloat16* __restrict__ q, const float* __restrict__ R_k,
     if (bb == 0) { pref[0] = 0; nzpref[0] = 0; }
     for (int w = 0; w < kW; ++w) { run_p += warp_tot[0][w]; run_n += warp_tot[1][w]; }
     __syncthreads();
+  }
+}
+
+__global__ void __launch_bounds__(kQrotThreads)
+qrot_kernel(const __nv_bfloat16* __restrict__ q, const float* __restrict__ R_k,
+            int B, int h_q, int h_kv, float qscale,
+            const int32_t* __restrict__ seq_lens, int max_pages,
+            float* __restrict__ qf, float* __restrict__ qs,
+            uint32_t* __restrict__ frag, float* __restrict__ koff,
+            float* __restrict__ invs, int* __restrict__ pref,
+            int* __restrict__ nzpref, int* __restrict__ cnt_ws,
+            unsigned* err) {
+  __shared__ QrotSmem sm;
+  qrot_body(blockIdx.x, blockIdx.y, sm, q, R_k, B, h_q, h_kv, qscale, seq_lens,
+            max_pages, qf, qs, frag, koff, invs, pref, nzpref, cnt_ws, err);
+}
+
+// ------------------------------------------------- decode-step prologue
+// One launch for the two independent first steps of a decode step: the
+// single-token cache write of every sequence (CTAs [0, n_app), as
+// append_small_kernel) and the query rotation (the following B * h_kv CTAs,
+// as qrot_kernel).  Both wait for the previous kernel before touching
+// inputs; the partial kernel then waits for this grid, i.e. for both.
+static_assert(kQrotThreads == 512, "one block size for both bodies");
+
+__global__ void __launch_bounds__(512)
+step_prologue_kernel(
+    int n_app, int app_tiles, const __nv_bfloat16* __restrict__ k,
+    const __nv_bfloat16* __restrict__ v, int n_tok,
+    const int32_t* __restrict__ cu_new, const int32_t* __restrict__ pos0,
+    const int32_t* __restrict__ bt, uint8_t* __restrict__ pool, int num_pages,
+    const float* __restrict__ R_v, const float* __restrict__ muR, float clip_k,
+    float clip_v, const __nv_bfloat16* __restrict__ q,
+    const float* __restrict__ R_k, int B, int h_q, int h_kv, float qscale,
+    const int32_t* __restrict__ seq_lens, int max_pages,
+    float* __restrict__ qf, float* __restrict__ qs, uint32_t* __restrict__ frag,
+    float* __restrict__ koff, float* __restrict__ invs, int* __restrict__ pref,
+    int* __restrict__ nzpref, int* __restrict__ cnt_ws, unsigned* err) {
+  extern __shared__ __align__(16) unsigned char dsm_[];
+  const int bid = blockIdx.x;
+  if (bid < n_app) {
+    const int tblk = bid % app_tiles, hk = (bid / app_tiles) % h_kv,
+              kind = bid / (app_tiles * h_kv);
+    append_small_body(tblk, hk, kind, *reinterpret_cast<AppendSmallSmem*>(dsm_),
+                      k, v, n_tok, cu_new, pos0, bt, B, max_pages, pool,
+                      num_pages, h_kv, R_k, R_v, muR, clip_k, clip_v, err);
+  } else {
+    const int r = bid - n_app;
+    qrot_body(r / h_kv, r % h_kv, *reinterpret_cast<QrotSmem*>(dsm_), q, R_k, B,
+              h_q, h_kv, qscale, seq_lens, max_pages, qf, qs, frag, koff, invs,
+              pref, nzpref, cnt_ws, err);
   }
 }
 
@@ -564,13 +624,15 @@ cudaError_t launch_partial_tensor(const optr_params* p, const uint8_t* pool,
                                   const uint32_t* frag, const float* koff,
                                   const float* invs, const float* qs,
                                   const int* pref, const int* nzpref,
-                                  float* part, int W, cudaStream_t s);
+                                  float* part, int W, bool early_pages,
+                                  cudaStream_t s);
 
 cudaError_t launch_decode(const optr_params* p, int variant,
                           const __nv_bfloat16* q, const int32_t* bt,
                           const int32_t* seq_lens, int B, int max_pages,
                           const uint8_t* pool, int num_pages, float* out,
-                          void* ws, const DecodePlan& plan, cudaStream_t s) {
+                          void* ws, const DecodePlan& plan, cudaStream_t s,
+                          const StepAppend* app) {
   char* w = static_cast<char*>(ws);
   float* qf = reinterpret_cast<float*>(w + plan.off_qf);
   float* qs = reinterpret_cast<float*>(w + plan.off_qs);
@@ -583,17 +645,43 @@ cudaError_t launch_decode(const optr_params* p, int variant,
   const int h_q = p->cfg.h_q, h_kv = p->cfg.h_kv;
   const float qscale = kLog2e / sqrtf((float)kD);
 
-  prof_mark(p, 2, s);
-  cudaError_t e = launch_pdl(qrot_kernel, dim3(B, h_kv), dim3(kQrotThreads), 0,
-                             s, q, p->R_k, B, h_q, h_kv, qscale, seq_lens,
-                             max_pages, qf, qs, frag, koff, invs, pref, nzpref,
-                             reinterpret_cast<int*>(w + plan.off_cnt), p->err);
-  if (e != cudaSuccess) return e;
+  int* cnt_ws = reinterpret_cast<int*>(w + plan.off_cnt);
+  cudaError_t e;
+  if (app) {
+    // the cache write of the step and the query rotation in one launch
+    prof_mark(p, 0, s);
+    const int tiles = (app->n_tok + kSmallTok - 1) / kSmallTok;
+    const int n_app = tiles * h_kv * 2;
+    const size_t sm_bytes = sizeof(AppendSmallSmem) > sizeof(QrotSmem)
+                                ? sizeof(AppendSmallSmem) : sizeof(QrotSmem);
+    e = ensure_dynamic_smem(reinterpret_cast<const void*>(&step_prologue_kernel),
+                            sm_bytes);
+    if (e != cudaSuccess) return e;
+    e = launch_pdl(step_prologue_kernel, dim3(n_app + B * h_kv), dim3(512),
+                   sm_bytes, s, n_app, tiles, app->k, app->v, app->n_tok,
+                   app->cu_new, app->pos0, bt, app->pool, num_pages,
+                   (const float*)p->R_v, (const float*)p->muR, p->cfg.clip_k,
+                   p->cfg.clip_v, q, (const float*)p->R_k, B, h_q, h_kv, qscale,
+                   seq_lens, max_pages, qf, qs, frag, koff, invs, pref, nzpref,
+                   cnt_ws, p->err);
+    if (e != cudaSuccess) return e;
+    prof_mark(p, 1, s);  // the append stage covers the fused launch,
+    prof_mark(p, 2, s);  // the query-rotation stage is empty
+  } else {
+    prof_mark(p, 2, s);
+    e = launch_pdl(qrot_kernel, dim3(B, h_kv), dim3(kQrotThreads), 0, s, q,
+                   p->R_k, B, h_q, h_kv, qscale, seq_lens, max_pages, qf, qs,
+                   frag, koff, invs, pref, nzpref, cnt_ws, p->err);
+    if (e != cudaSuccess) return e;
+  }
   prof_mark(p, 3, s);
   if (variant != OPTR_VARIANT_CUDA_CORE) {
+    // after a separate append the pool is complete before qrot starts, so
+    // the partial kernel may fetch pages before waiting for qrot; after the
+    // fused prologue it must wait first
     e = launch_partial_tensor(p, pool, bt, seq_lens, B, max_pages, num_pages,
                               frag, koff, invs, qs, pref, nzpref, part, plan.W,
-                              s);
+                              app == nullptr, s);
   } else {
     e = launch_pdl(partial_cuda_core_kernel, dim3(plan.W / 4), dim3(128), 0, s,
                    pool, bt, seq_lens, B, max_pages, num_pages, h_q, h_kv, qf,

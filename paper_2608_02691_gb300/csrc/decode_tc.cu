@@ -221,7 +221,8 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
                       const float* __restrict__ qs,
                       const int* __restrict__ pref,
                       const int* __restrict__ nzpref,
-                      float* __restrict__ part, int W, unsigned* err) {
+                      float* __restrict__ part, int W, int early_pages,
+                      unsigned* err) {
   // One 16-warp CTA per SM: the warp schedulers favour the CTAs that
   // arrived first on an SM, and with four 4-warp CTAs per SM the last CTA
   // finished ~20% after the first; within one CTA the warps keep pace.
@@ -238,10 +239,14 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
 
   // Page prefix sums.  For up to kPrefCache sequences the CTA scans the
   // lengths itself (the values qrot writes to pref for the combine): the
-  // lengths, the block table and the pool are inputs, complete before qrot
-  // began (qrot passes its pdl_wait() before it lets this grid launch), so
-  // the page tables and the first page copies are set up before this grid's
-  // own pdl_wait(), overlapping qrot; only the query fragments wait.
+  // lengths and the block table are inputs, complete before the previous
+  // kernel (qrot, or the fused step prologue) began, since that kernel
+  // passes its pdl_wait() before it lets this grid launch.  So the page
+  // tables are set up before this grid's own pdl_wait(), overlapping the
+  // previous kernel.  The first page copies also go before the wait when the
+  // pool was complete before the previous kernel began (early_pages: a
+  // separate append); after the fused step prologue, which writes the pool,
+  // they follow the wait.
   const bool cached = B <= kPrefCache;
   static_assert(kPrefCache < kWarps * 32, "one thread per sequence");
   int F;
@@ -291,9 +296,10 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
     issue(2 * q + 1);
     cp_async_commit();
   };
-  issue_pair(0);
+  if (early_pages) issue_pair(0);
   pdl_wait();  // (returns at once when already passed above)
   pdl_trigger();
+  if (!early_pages) issue_pair(0);
 
   // per-segment state
   uint32_t bmin = 0;           // key min-term B fragment (sum q' per group)
@@ -634,7 +640,8 @@ cudaError_t launch_partial_tensor(const optr_params* p, const uint8_t* pool,
                                   const uint32_t* frag, const float* koff,
                                   const float* invs, const float* qs,
                                   const int* pref, const int* nzpref,
-                                  float* part, int W, cudaStream_t s) {
+                                  float* part, int W, bool early_pages,
+                                  cudaStream_t s) {
   const size_t dsmem = sizeof(WarpSmemTC) * kWarps;
   cudaError_t e =
       ensure_dynamic_smem(reinterpret_cast<const void*>(&partial_tensor_kernel), dsmem);
@@ -642,7 +649,7 @@ cudaError_t launch_partial_tensor(const optr_params* p, const uint8_t* pool,
   return launch_pdl(partial_tensor_kernel, dim3(W / kWarps), dim3(kWarps * 32),
                     dsmem, s, pool, bt, seq_lens, B, max_pages, num_pages,
                     p->cfg.h_q, p->cfg.h_kv, frag, koff, invs, qs, pref, nzpref,
-                    part, W, p->err);
+                    part, W, early_pages ? 1 : 0, p->err);
 }
 
 }  // namespace optr

@@ -288,6 +288,48 @@ optr_status optr_decode_attention(const optr_params* p, const void* q,
   return cuda_status(e);
 }
 
+optr_status optr_decode_step(const optr_params* p, const void* q,
+                             const void* k, const void* v, int n_tok,
+                             const int32_t* cu_new, const int32_t* pos0,
+                             const int32_t* block_table,
+                             const int32_t* seq_lens, int B, int max_pages,
+                             uint8_t* pool, int num_pages, float* out,
+                             void* workspace, size_t ws_bytes,
+                             cudaStream_t stream) {
+  if (!p || n_tok < 0 || B <= 0 || max_pages <= 0 || num_pages <= 0)
+    return OPTR_ERR_INVALID_ARG;
+  if (!q || !block_table || !seq_lens || !pool || !out)
+    return OPTR_ERR_INVALID_ARG;
+  if (n_tok > 0 && (!k || !v || !cu_new || !pos0)) return OPTR_ERR_INVALID_ARG;
+  if (!aligned(pool, 16) || !aligned(q, 16) || !aligned(out, 16) ||
+      (n_tok > 0 && (!aligned(k, 16) || !aligned(v, 16))))
+    return OPTR_ERR_INVALID_ARG;
+  if ((long long)max_pages * kPage > (1LL << 30) || B > (1 << 24))
+    return OPTR_ERR_OUT_OF_RANGE;
+  if ((long long)B * max_pages * p->cfg.h_kv >= (1LL << 31))
+    return OPTR_ERR_OUT_OF_RANGE;
+  DecodePlan plan = decode_plan(p, B, max_pages);
+  if (!workspace || ws_bytes < plan.total || !aligned(workspace, 256))
+    return OPTR_ERR_WORKSPACE;
+  // the fused launch covers decode-step sized writes with the tensor decode;
+  // anything else runs as the two calls
+  if (n_tok == 0 || n_tok > 256 || p->cfg.decode_variant == OPTR_VARIANT_CUDA_CORE ||
+      p->cfg.append_variant == OPTR_VARIANT_CUDA_CORE) {
+    optr_status st = optr_kv_append(p, k, v, n_tok, cu_new, pos0, block_table,
+                                    B, max_pages, pool, num_pages, stream);
+    if (st != OPTR_OK) return st;
+    return optr_decode_attention(p, q, block_table, seq_lens, B, max_pages, pool,
+                                 num_pages, out, workspace, ws_bytes, stream);
+  }
+  StepAppend app{(const __nv_bfloat16*)k, (const __nv_bfloat16*)v, n_tok,
+                 cu_new, pos0, pool};
+  cudaError_t e = launch_decode(p, p->cfg.decode_variant, (const __nv_bfloat16*)q,
+                                block_table, seq_lens, B, max_pages, pool,
+                                num_pages, out, workspace, plan, stream, &app);
+  if (p->prof) const_cast<optr_params*>(p)->ran[0] = const_cast<optr_params*>(p)->ran[1] = 1;
+  return cuda_status(e);
+}
+
 optr_status optr_profile_enable(optr_params* p, int on) {
   if (!p) return OPTR_ERR_INVALID_ARG;
   if (on && !p->prof) {

@@ -123,10 +123,22 @@ cudaError_t launch_append_tensor(const optr_params* p, const __nv_bfloat16* k,
                                  const int32_t* cu_new, const int32_t* pos0,
                                  const int32_t* bt, int B, int max_pages,
                                  uint8_t* pool, int num_pages, cudaStream_t s);
+// The decode step's single-token cache write, fused into the decode's first
+// launch (optr_decode_step); null for a decode alone.
+struct StepAppend {
+  const __nv_bfloat16* k;
+  const __nv_bfloat16* v;
+  int n_tok;
+  const int32_t* cu_new;
+  const int32_t* pos0;
+  uint8_t* pool;
+};
+
 cudaError_t launch_decode(const optr_params* p, int variant,
                           const __nv_bfloat16* q, const int32_t* bt,
                           const int32_t* seq_lens, int B, int max_pages,
                           const uint8_t* pool, int num_pages, float* out,
-                          void* ws, const DecodePlan& plan, cudaStream_t s);
+                          void* ws, const DecodePlan& plan, cudaStream_t s,
+                          const StepAppend* app = nullptr);
 
 }  // namespace optr

@@ -56,6 +56,8 @@ _SIG = {
     "optr_strerror": (ctypes.c_char_p, [_I]),
     "optr_decode_attention_noalloc": (_I, [_V, _V, _V, _V, _I, _I, _V, _I,
                                            _V, _V]),
+    "optr_decode_step": (_I, [_V, _V, _V, _V, _I, _V, _V, _V, _V, _I, _I, _V,
+                              _I, _V, _V, ctypes.c_size_t, _V]),
     "optr_profile_enable": (_I, [_V, _I]),
     "optr_profile_last": (_I, [_V, ctypes.POINTER(ctypes.c_float)]),
 }
@@ -193,6 +195,27 @@ def optr_decode_attention(p: Params, q, block_table, seq_lens, pool, out,
         p.handle, _ptr(q), _ptr(block_table), _ptr(seq_lens), B, max_pages,
         _ptr(pool), pool.shape[0], _ptr(out), _ptr(workspace),
         workspace.numel(), _stream(stream)), "optr_decode_attention")
+
+
+def optr_decode_step(p: Params, q, k, v, cu_new, pos0, block_table, seq_lens,
+                     pool, out, workspace, stream=None) -> None:
+    """optr_kv_append of the step's new tokens (k, v, cu_new, pos0) followed
+    by optr_decode_attention over the updated cache; seq_lens counts the new
+    tokens."""
+    for t, dt, nm in ((q, torch.bfloat16, "q"), (k, torch.bfloat16, "k"),
+                      (v, torch.bfloat16, "v"), (cu_new, torch.int32, "cu_new"),
+                      (pos0, torch.int32, "pos0"),
+                      (block_table, torch.int32, "block_table"),
+                      (seq_lens, torch.int32, "seq_lens"),
+                      (pool, torch.uint8, "pool"), (out, torch.float32, "out"),
+                      (workspace, torch.uint8, "workspace")):
+        _dev(t, dt, nm)
+    B, max_pages = block_table.shape
+    _check(lib().optr_decode_step(
+        p.handle, _ptr(q), _ptr(k), _ptr(v), k.shape[0], _ptr(cu_new),
+        _ptr(pos0), _ptr(block_table), _ptr(seq_lens), B, max_pages,
+        _ptr(pool), pool.shape[0], _ptr(out), _ptr(workspace),
+        workspace.numel(), _stream(stream)), "optr_decode_step")
 
 
 NOALLOC_SCRATCH_BYTES = 16 << 20

@@ -249,3 +249,36 @@ def test_decode_value_magnitudes(variant, kscale, vscale):
     ref = ph.oracle_decode(c, pool_ref)
     r = ph.assert_decode_close(got, ref, f"k x{kscale} v x{vscale}")
     print(f"k x{kscale} v x{vscale} variant {variant}: err/rms {r:.2e}")
+
+
+@pytest.mark.parametrize("variant", VARIANTS)
+@pytest.mark.parametrize("name,scale", [("tiny", 1.0), ("decode8k", 1 / 16),
+                                        ("ragged", 1 / 32)])
+def test_decode_step_equals_append_then_decode(name, scale, variant):
+    """optr_decode_step (the step's cache write fused with the query rotation
+    into one launch) leaves the same pool bytes and returns the same output,
+    bit for bit, as optr_kv_append followed by optr_decode_attention."""
+    c = synth.build_case(synth.workload(name, 0, scale), 0)
+    dev = "cuda"
+    p = optr.optr_params_create(c["R_k"], c["R_v"], c["mu"], c["h_q"],
+                                decode_variant=variant)
+    pool = optr.new_pool(p, c["num_pages"], device=dev)
+    bt = c["block_table"].to(dev)
+    optr.optr_kv_append(p, c["k_ctx"].to(dev), c["v_ctx"].to(dev),
+                        c["cu_ctx"].to(dev), c["pos0_ctx"].to(dev), bt, pool)
+    pool2 = pool.clone()
+    args = dict(k=c["k_new"].to(dev), v=c["v_new"].to(dev),
+                cu_new=c["cu_new"].to(dev), pos0=c["pos0_new"].to(dev))
+    q, seq = c["q"].to(dev), c["seq_lens"].to(dev)
+    ws = optr.new_workspace(p, c["B"], bt.shape[1], device=dev)
+    out1 = torch.empty(c["B"], c["h_q"], 128, dtype=torch.float32, device=dev)
+    out2 = torch.full_like(out1, 7.0)
+    optr.optr_kv_append(p, args["k"], args["v"], args["cu_new"], args["pos0"],
+                        bt, pool)
+    optr.optr_decode_attention(p, q, bt, seq, pool, out1, ws)
+    optr.optr_decode_step(p, q, args["k"], args["v"], args["cu_new"],
+                          args["pos0"], bt, seq, pool2, out2, ws)
+    torch.cuda.synchronize()
+    assert optr.optr_device_error(p) == 0
+    assert torch.equal(pool, pool2)
+    assert torch.equal(out1, out2)
