@@ -134,6 +134,7 @@ typedef enum {
 #define OPTR_DEVERR_SEQ_LEN 4u   /* seq_lens[b] < 0 or > max_pages * 16     */
 #define OPTR_DEVERR_CU_NEW 8u    /* cu_new not non-decreasing within n_tok  */
 #define OPTR_DEVERR_FP16_RANGE 16u /* tensor-core append: |k| or |v| >= 65504 */
+#define OPTR_DEVERR_TIMEOUT 32u  /* internal: a kernel's bounded wait gave up */
 
 /* Kernel variants (for measurement; 0 picks the library default). */
 #define OPTR_VARIANT_DEFAULT 0

@@ -170,19 +170,19 @@ optr_status optr_params_create(const optr_config* cfg, const float* R_k,
   if (e == cudaSuccess) e = cudaMalloc(&p->R_vT, sizeof(float) * H * mat);
   if (e == cudaSuccess) e = cudaMalloc(&p->muR, sizeof(float) * H * kD);
   if (e == cudaSuccess) e = cudaMalloc(&p->err, sizeof(unsigned));
-  std::vector<uint32_t> frags((size_t)H * kRFragWords);
-  if (e == cudaSuccess) e = cudaMalloc(&p->Rk_tc, sizeof(uint32_t) * frags.size());
-  if (e == cudaSuccess) e = cudaMalloc(&p->Rv_tc, sizeof(uint32_t) * frags.size());
+  std::vector<uint16_t> t5((size_t)H * kRT5Halves);
+  if (e == cudaSuccess) e = cudaMalloc(&p->Rk_t5, sizeof(uint16_t) * t5.size());
+  if (e == cudaSuccess) e = cudaMalloc(&p->Rv_t5, sizeof(uint16_t) * t5.size());
   if (e == cudaSuccess) {
     for (int h = 0; h < H; ++h)
-      build_rotation_fragments(R_k + h * mat, frags.data() + (size_t)h * kRFragWords);
-    e = cudaMemcpy(p->Rk_tc, frags.data(), sizeof(uint32_t) * frags.size(),
+      build_rotation_tc05(R_k + h * mat, t5.data() + (size_t)h * kRT5Halves);
+    e = cudaMemcpy(p->Rk_t5, t5.data(), sizeof(uint16_t) * t5.size(),
                    cudaMemcpyHostToDevice);
   }
   if (e == cudaSuccess) {
     for (int h = 0; h < H; ++h)
-      build_rotation_fragments(R_v + h * mat, frags.data() + (size_t)h * kRFragWords);
-    e = cudaMemcpy(p->Rv_tc, frags.data(), sizeof(uint32_t) * frags.size(),
+      build_rotation_tc05(R_v + h * mat, t5.data() + (size_t)h * kRT5Halves);
+    e = cudaMemcpy(p->Rv_t5, t5.data(), sizeof(uint16_t) * t5.size(),
                    cudaMemcpyHostToDevice);
   }
   if (e == cudaSuccess)
@@ -211,8 +211,8 @@ void optr_params_destroy(optr_params* p) {
   cudaFree(p->R_v);
   cudaFree(p->R_vT);
   cudaFree(p->muR);
-  cudaFree(p->Rk_tc);
-  cudaFree(p->Rv_tc);
+  cudaFree(p->Rk_t5);
+  cudaFree(p->Rv_t5);
   cudaFree(p->err);
   free(p);
 }
@@ -246,7 +246,7 @@ optr_status optr_kv_append(const optr_params* p, const void* k, const void* v,
                                 block_table, B, max_pages, pool, num_pages,
                                 stream);
   else
-    e = launch_append_tensor(p, (const __nv_bfloat16*)k,
+    e = launch_append_tc05(p, (const __nv_bfloat16*)k,
                              (const __nv_bfloat16*)v, n_tok, cu_new, pos0,
                              block_table, B, max_pages, pool, num_pages,
                              stream);

@@ -34,8 +34,8 @@ struct optr_params {
   float* R_v;          // device [h_kv][D][D]
   float* R_vT;         // device [h_kv][D][D], R_vT[h][j][i] = R_v[h][i][j]
   float* muR;          // device [h_kv][D], mu R_k computed in fp64
-  uint32_t* Rk_tc;     // device tensor-core B fragments of R_k (append_tc.cu)
-  uint32_t* Rv_tc;     // device tensor-core B fragments of R_v
+  uint16_t* Rk_t5;     // device tcgen05 B operands of R_k (append_tc05.cu)
+  uint16_t* Rv_t5;     // device tcgen05 B operands of R_v
   unsigned* err;       // device error word
   // stage timing (optr_profile_enable): ev[0..1] bracket the append kernel,
   // ev[2..5] the decode stages (before qrot, partial, combine, after).
@@ -115,14 +115,14 @@ cudaError_t launch_append_cuda_core(const optr_params* p, const __nv_bfloat16* k
                                     const int32_t* bt, int B, int max_pages,
                                     uint8_t* pool, int num_pages,
                                     cudaStream_t s);
-// Tensor-core append operand: B fragments of one rotation, see append_tc.cu.
-constexpr int kRFragWords = 8 * 16 * 32 * 4;  // k-steps x n-tiles x lanes x 4
-void build_rotation_fragments(const float* R /*[D][D]*/, uint32_t* out);
-cudaError_t launch_append_tensor(const optr_params* p, const __nv_bfloat16* k,
-                                 const __nv_bfloat16* v, int n_tok,
-                                 const int32_t* cu_new, const int32_t* pos0,
-                                 const int32_t* bt, int B, int max_pages,
-                                 uint8_t* pool, int num_pages, cudaStream_t s);
+// tcgen05 append operand: [hi, lo][128 x 128] fp16 per head, see append_tc05.cu.
+constexpr int kRT5Halves = 2 * kD * kD;
+void build_rotation_tc05(const float* R /*[D][D]*/, uint16_t* out);
+cudaError_t launch_append_tc05(const optr_params* p, const __nv_bfloat16* k,
+                               const __nv_bfloat16* v, int n_tok,
+                               const int32_t* cu_new, const int32_t* pos0,
+                               const int32_t* bt, int B, int max_pages,
+                               uint8_t* pool, int num_pages, cudaStream_t s);
 // The decode step's single-token cache write, fused into the decode's first
 // launch (optr_decode_step); null for a decode alone.
 struct StepAppend {
