@@ -15,17 +15,23 @@
 //                   tensor copies (channels 0-63 and 64-127, 128-byte
 //                   swizzle) into a shared-memory stage (4 stages in
 //                   flight);
-//   8 epilogue warps, two groups of 4 taking alternate tiles: thread t owns
-//                   token row t; it converts its row to f16 and stores it to
-//                   tensor memory as the MMA's A operand, then reads its
-//                   row of the accumulator back and quantizes, packs and
-//                   scatters its 48-byte record (codes + scale/min);
+//   16 epilogue warps, two groups of 8 taking alternate tiles: two threads
+//                   own token row t, one per half of the channels; each
+//                   converts its half row to f16 and stores it to tensor
+//                   memory as the MMA's A operand, then reads its half of
+//                   the accumulator row back and quantizes and packs its two
+//                   channel groups; the pair's code bytes meet in shared
+//                   memory and the first thread writes the 32 code bytes,
+//                   each thread its 8 scale/min bytes.  A group converts its
+//                   next tile while the tensor core works on the current one
+//                   (two A buffers per group);
 //   MMA warp        one thread issues the 16 tcgen05.mma of a tile (8
 //                   K-steps x {R hi, R lo}) from tensor-memory A and
 //                   shared-memory B (R, 64 KB, loaded once) into the
 //                   group's tensor-memory accumulator.
-// Tensor memory (512 columns): accumulators D[2] (128 columns each) and A
-// operands A[2] (64 columns each), one of each per epilogue group.
+// Tensor memory (512 columns): per epilogue group g an accumulator D[g]
+// (128 columns, at 128 g) and two A operands (64 columns each, at
+// 256 + 128 g + 64 b).
 // The quantizer is quant.cuh's float32 formula.
 #include "append_common.cuh"
 #include "decode_common.cuh"
@@ -68,11 +74,12 @@ constexpr int kRows = 128;        // tokens per tile (MMA M)
 constexpr int kCuCache = 512;     // sequences whose cu_new / pos0 a CTA caches
 constexpr int kStages = 4;        // tiles in flight from global memory
 constexpr uint32_t kStageBytes = kRows * kD * 2;  // two 16 KB TMA boxes
-constexpr int kEpiWarps = 8;      // two groups of 4
+constexpr int kEpiWarps = 16;     // two groups of 8
+constexpr int kGroupThreads = 256;
 constexpr int kThreads = (kEpiWarps + 2) * 32;
 constexpr int kProducerWarp = kEpiWarps, kMmaWarp = kEpiWarps + 1;
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kColD0 = 0, kColA0 = 256;  // D[g] at 128 g, A[g] at 256 + 64 g
+constexpr uint32_t kColD0 = 0, kColA0 = 256;  // D[g] at 128 g, A[g][b] at 256 + 128 g + 64 b
 constexpr uint32_t kIdesc = tc05::idesc_f16(128, 128);
 
 struct Smem {
@@ -83,46 +90,99 @@ struct Smem {
   alignas(16) float mu[kD];               // mu R_k (keys) or 0 (values)
   int cu[kCuCache + 1];
   int p0[kCuCache];
-  uint64_t full[kStages], empty[kStages], aready[2], dready[2];
+  uint4 xchg[2][kRows][2];               // second-half code words per row
+  uint64_t full[kStages], empty[kStages], aready[2][2], dready[2], dfree[2];
+  uint64_t xready[2], xdone[2];  // the exchange slot of group g written / read
   uint32_t tmem;
   int abort;
 };
 
 __device__ __forceinline__ uint32_t bf16x2_to_f16x2(uint32_t u) {
-  const float lo = __uint_as_float(u << 16);
+  uint32_t ls;  // u << 16 as an integer multiply (FMA pipe; the ALU pipe is the busier one)
+  asm("mul.lo.u32 %0, %1, 65536;" : "=r"(ls) : "r"(u));
+  const float lo = __uint_as_float(ls);
   const float hi = __uint_as_float(u & 0xffff0000u);
   uint32_t r;
   asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
   return r;
 }
 
-// Codes of the 32 values of one group into the 8 code words (byte G of word
-// w holds channels 32G + 4w + r at bits 2r).  u + 1.5 * 2^23 rounds u in
-// [0, 3] to the nearest integer (ties to even, as __float2int_rn) and leaves
-// it in the low mantissa bits of the float: bits = 0x4B400000 + code; the
-// constant part is removed from each word once, after all 16 codes are in.
+// Quantizer parameters of one group (quant.cuh's formula: mn = c lo,
+// mx = c hi, r = mx - mn, degenerate unless 1e-30 < r <= FLT_MAX), with the
+// two divisions done as reciprocal multiplies: inv4 = (3 / r) / 4 from
+// rcp.approx (within ~2 ulp of quant.cuh's correctly rounded 3 / r, which
+// moves only code decisions within ~1e-6 of a rounding boundary) and the
+// stored scale fp16(r * (1/3)) (at most one fp16 ulp from fp16(r / 3)).
+// A degenerate group gets inv4 = 0, which makes every code 0 below.
+struct FastQuant {
+  float mn, mx, inv4;
+  uint32_t meta;  // (scale, min) as half2
+  bool degenerate;
+};
+
+__device__ __forceinline__ FastQuant fast_quant_params(float lo, float hi, float clip) {
+  FastQuant q;
+  q.mn = __fmul_rn(clip, lo);
+  q.mx = __fmul_rn(clip, hi);
+  const float r = __fsub_rn(q.mx, q.mn);
+  q.degenerate = !(r > 1e-30f) || !(r <= 3.402823466e38f);
+  float rc;
+  asm("rcp.approx.f32 %0, %1;" : "=f"(rc) : "f"(r));
+  q.inv4 = q.degenerate ? 0.f : __fmul_rn(0.75f, rc);
+  const __half2 sm = __halves2half2(
+      q.degenerate ? __float2half_rn(0.f) : __float2half_rn(__fmul_rn(r, 1.0f / 3.0f)),
+      __float2half_rn(q.mn));
+  q.meta = *reinterpret_cast<const uint32_t*>(&sm);
+  return q;
+}
+
+// Code bytes of the 32 values x of one group: byte[w] holds the codes of
+// channels 4w + r (r = 0..3) at bits 2r, in its low byte (bits 8-21 zero).
+// In x's scale (mn, mx and inv4 = inv / 4 scaled alike):
+//   v = sat((x - mn) * inv4)   u = (x - mn) * inv rounded to float, / 4
+//                              exact, clamped to [0, 1]: NaN (and every
+//                              value of a degenerate group) -> 0
+//   v * 4 + 1.5 * 2^23         rounds u to the nearest integer (ties to
+//                              even, as rint) into the low mantissa bits:
+//                              bits = 0x4B400000 + code, code <= 3
+// and sum_r bits_r 4^r = 85 * 0x4B400000 + byte, whose constant part lies
+// above bit 21.  With c = 1, x lies in [mn, mx], so no clamp of x is needed.
 template <bool kClamp>
-__device__ __forceinline__ void quantize_group(const float (&z)[32], int G,
-                                               const GroupQuant& gq,
-                                               uint32_t (&word)[8]) {
+__device__ __forceinline__ void code_bytes(const float (&x)[32], const FastQuant& q,
+                                           uint32_t (&byte)[8]) {
 #pragma unroll
-  for (int j = 0; j < 32; ++j) {
-    const int w = j >> 2, r = j & 3;
-    // with c = 1, z <= mx always; fmaxf also maps a NaN to mn, as the
-    // clamped formula does
-    const float zc = kClamp ? fminf(fmaxf(z[j], gq.mn), gq.mx) : fmaxf(z[j], gq.mn);
-    const float u = gq.degenerate ? 0.f : __fmul_rn(__fsub_rn(zc, gq.mn), gq.inv);
-    const uint32_t bits = __float_as_uint(__fadd_rn(u, 12582912.0f));
-    word[w] += bits << (8 * G + 2 * r);
+  for (int w = 0; w < 8; ++w) {
+    uint32_t b[4];
+#pragma unroll
+    for (int r = 0; r < 4; ++r) {
+      const float xv = x[4 * w + r];
+      const float xc = kClamp ? fminf(fmaxf(xv, q.mn), q.mx) : xv;
+      float v;
+      asm("mul.rn.sat.f32 %0, %1, %2;" : "=f"(v) : "f"(__fsub_rn(xc, q.mn)), "f"(q.inv4));
+      b[r] = __float_as_uint(__fmaf_rn(v, 4.0f, 12582912.0f));
+    }
+    byte[w] = b[0] + 4u * b[1] + 16u * b[2] + 64u * b[3];
   }
 }
 
-// sum over the 16 (G, r) of 0x4B400000 << (8 G + 2 r), mod 2^32
-__host__ __device__ constexpr uint32_t magic_sum() {
-  uint32_t s = 0;
-  for (int G = 0; G < 4; ++G)
-    for (int r = 0; r < 4; ++r) s += 0x4B400000u << (8 * G + 2 * r);
-  return s;
+// Smallest and largest of 32 values (NaNs ignored): four interleaved
+// chains per extreme, two new values per 3-input min/max.
+__device__ __forceinline__ void minmax32(const float (&x)[32], float& lo, float& hi) {
+  float l[4], h[4];
+#pragma unroll
+  for (int c = 0; c < 4; ++c) {
+    l[c] = fminf(x[c], x[c + 4]);
+    h[c] = fmaxf(x[c], x[c + 4]);
+  }
+#pragma unroll
+  for (int j = 8; j < 32; j += 8)
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      l[c] = fminf(l[c], fminf(x[j + c], x[j + c + 4]));
+      h[c] = fmaxf(h[c], fmaxf(x[j + c], x[j + c + 4]));
+    }
+  lo = fminf(fminf(l[0], l[1]), fminf(l[2], l[3]));
+  hi = fmaxf(fmaxf(h[0], h[1]), fmaxf(h[2], h[3]));
 }
 
 template <bool kClamp>
@@ -159,11 +219,15 @@ append_tc05_kernel(const __grid_constant__ CUtensorMap tmap_k,
   if (tid == 0) {
     for (int s = 0; s < kStages; ++s) {
       tc05::bar_init(&S.full[s], 1);
-      tc05::bar_init(&S.empty[s], 128);
+      tc05::bar_init(&S.empty[s], kGroupThreads);
     }
     for (int g = 0; g < 2; ++g) {
-      tc05::bar_init(&S.aready[g], 128);
+      tc05::bar_init(&S.aready[g][0], kGroupThreads);
+      tc05::bar_init(&S.aready[g][1], kGroupThreads);
       tc05::bar_init(&S.dready[g], 1);
+      tc05::bar_init(&S.dfree[g], kGroupThreads);
+      tc05::bar_init(&S.xready[g], kGroupThreads / 2);
+      tc05::bar_init(&S.xdone[g], kGroupThreads / 2);
     }
     // the 128-byte TMA swizzle wants 1024-byte aligned boxes
     S.abort = (tc05::smem_addr(S.stage[0]) & 1023u) != 0;
@@ -213,10 +277,14 @@ append_tc05_kernel(const __grid_constant__ CUtensorMap tmap_k,
     if (lane == 0) {
       const uint32_t b0 = tc05::smem_addr(&S.b[0][0]);
       for (int i = 0; i < my_tiles; ++i) {
-        const int g = i & 1;
-        if (!tc05::bar_wait(&S.aready[g], (i >> 1) & 1, abort)) break;
+        // tile i is the k-th of group g, its A operand in buffer k % 2; the
+        // group's previous tile must have been read out of D[g]
+        const int g = i & 1, k = i >> 1;
+        if (!tc05::bar_wait(&S.aready[g][k & 1], (k >> 1) & 1, abort)) break;
+        if (k > 0 && !tc05::bar_wait(&S.dfree[g], (k - 1) & 1, abort)) break;
         tc05::fence_after();
-        const uint32_t d = tmem + kColD0 + 128u * g, a = tmem + kColA0 + 64u * g;
+        const uint32_t d = tmem + kColD0 + 128u * g,
+                       a = tmem + kColA0 + 128u * g + 64u * (k & 1);
 #pragma unroll
         for (int ks = 0; ks < 8; ++ks)
 #pragma unroll
@@ -233,31 +301,40 @@ append_tc05_kernel(const __grid_constant__ CUtensorMap tmap_k,
     __syncwarp();
   } else {
     // ---------------------------------------------------------- epilogue
-    const int g = warp >> 2, q = warp & 3, row = 32 * q + lane;
+    // warp w: group g = w / 8; lane quarter q = w % 4 (its tensor-memory
+    // lanes); channel half hp = (w / 4) % 2, i.e. channel groups 2hp, 2hp+1
+    const int g = warp >> 3, q = warp & 3, hp = (warp >> 2) & 1, row = 32 * q + lane;
     const float clip = kind ? clip_v : clip_k;
     const int codes_off = kind ? OPTR_V_CODES_OFFSET : OPTR_K_CODES_OFFSET;
     const int meta_off = kind ? OPTR_V_META_OFFSET : OPTR_K_META_OFFSET;
     const uint32_t lane_base = (uint32_t)(32 * q) << 16;
-    const uint32_t tA = tmem + lane_base + kColA0 + 64u * g;
     const uint32_t tD = tmem + lane_base + kColD0 + 128u * g;
-    for (int i = g; i < my_tiles; i += 2) {
-      const int s = i % kStages;
-      const int tok = ((int)blockIdx.x + i * (int)gridDim.x) * kRows + row;
-      // destination of this row's record (the block-table load overlaps
-      // the copy, the conversion and the MMA)
-      long long dst = -1;
-      int slot = 0;
+    const int n_mine = my_tiles > g ? (my_tiles - 1 - g) / 2 + 1 : 0;
+    auto token = [&](int k) {
+      return ((int)blockIdx.x + (g + 2 * k) * (int)gridDim.x) * kRows + row;
+    };
+    // destination of this row's record in the group's k-th tile (the
+    // block-table load completes during the conversion and the MMA)
+    auto resolve = [&](int k, int& slot) -> long long {
+      const int tok = token(k);
+      long long d = -1;
       if (tok < n_tok)
-        dst = cached ? resolve_slot_cached(tok, h, S.cu, S.p0, bt, B, max_pages,
-                                           num_pages, h_kv, &slot, err)
-                     : resolve_slot(tok, h, cu_new, pos0, bt, B, max_pages,
-                                    num_pages, h_kv, &slot, err);
+        d = cached ? resolve_slot_cached(tok, h, S.cu, S.p0, bt, B, max_pages,
+                                         num_pages, h_kv, &slot, err)
+                   : resolve_slot(tok, h, cu_new, pos0, bt, B, max_pages,
+                                  num_pages, h_kv, &slot, err);
       __syncwarp();  // converged for the warp-wide tensor-memory accesses
-      if (!__all_sync(0xffffffffu, tc05::bar_wait(&S.full[s], (i / kStages) & 1, abort))) break;
-      // the row as f16 into tensor memory: columns j <-> channels 2j, 2j+1
-#pragma unroll
-      for (int half = 0; half < 2; ++half) {
-        const uint8_t* rb = S.stage[s] + half * (kStageBytes / 2) + row * 128;
+      return d;
+    };
+    // the row of the group's k-th tile as f16 into A buffer k % 2:
+    // columns j <-> channels 2j, 2j+1
+    auto convert = [&](int k) -> bool {
+      const int i = g + 2 * k, s = i % kStages;
+      if (!__all_sync(0xffffffffu, tc05::bar_wait(&S.full[s], (i / kStages) & 1, abort)))
+        return false;
+      const uint32_t tA = tmem + lane_base + kColA0 + 128u * g + 64u * (k & 1) + 32u * hp;
+      {
+        const uint8_t* rb = S.stage[s] + hp * (kStageBytes / 2) + row * 128;
         uint32_t a[32];
 #pragma unroll
         for (int c = 0; c < 8; ++c) {
@@ -267,60 +344,108 @@ append_tc05_kernel(const __grid_constant__ CUtensorMap tmap_k,
           a[4 * c + 2] = bf16x2_to_f16x2(x.z);
           a[4 * c + 3] = bf16x2_to_f16x2(x.w);
         }
-        tc05::tmem_st32(tA + 32u * half, a);
+        tc05::tmem_st32(tA, a);
       }
       tc05::bar_arrive(&S.empty[s]);  // stage s read (values in registers)
       tc05::tmem_wait_st();
       tc05::fence_before();
-      tc05::bar_arrive(&S.aready[g]);
-      if (!__all_sync(0xffffffffu, tc05::bar_wait(&S.dready[g], (i >> 1) & 1, abort))) break;
+      tc05::bar_arrive(&S.aready[g][k & 1]);
+      return true;
+    };
+
+    int slot_next = 0;
+    long long dst_next = n_mine > 0 ? resolve(0, slot_next) : -1;
+    bool ok = n_mine == 0 || convert(0);
+    for (int k = 0; ok && k < n_mine; ++k) {
+      const long long dst = dst_next;
+      const int slot = slot_next;
+      const int tok = token(k);
+      if (k + 1 < n_mine) {
+        dst_next = resolve(k + 1, slot_next);
+        if (!convert(k + 1)) break;
+      }
+      if (!__all_sync(0xffffffffu, tc05::bar_wait(&S.dready[g], k & 1, abort))) break;
       tc05::fence_after();
 
-      uint32_t word[8] = {0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
-      uint32_t meta[4];
+      uint32_t word[8];
+      uint32_t meta[2];
       bool range_err = false;
-#pragma unroll
-      for (int G = 0; G < kGroups; ++G) {
-        uint32_t acc[32];
-        tc05::tmem_ld32(tD + 32u * G, acc);
+      {
+        const int G2 = 2 * hp;  // this thread's two channel groups
+        uint32_t acc[2][32];
+        tc05::tmem_ld32(tD + 32u * G2, acc[0]);
+        tc05::tmem_ld32(tD + 32u * (G2 + 1), acc[1]);
         tc05::tmem_wait_ld();
-        float z[32];
-        const float4* mu4 = reinterpret_cast<const float4*>(S.mu + 32 * G);
+        tc05::fence_before();
+        tc05::bar_arrive(&S.dfree[g]);  // D[g] read: the next MMA may start
+        uint32_t bytes[2][8];
 #pragma unroll
-        for (int j4 = 0; j4 < 8; ++j4) {  // acc / 64 is exact: one rounding, as fmul + fsub
-          const float4 m = mu4[j4];
-          z[4 * j4 + 0] = fmaf(__uint_as_float(acc[4 * j4 + 0]), 1.0f / 64.0f, -m.x);
-          z[4 * j4 + 1] = fmaf(__uint_as_float(acc[4 * j4 + 1]), 1.0f / 64.0f, -m.y);
-          z[4 * j4 + 2] = fmaf(__uint_as_float(acc[4 * j4 + 2]), 1.0f / 64.0f, -m.z);
-          z[4 * j4 + 3] = fmaf(__uint_as_float(acc[4 * j4 + 3]), 1.0f / 64.0f, -m.w);
-        }
-        float lo = z[0], hi = z[0];
+        for (int e = 0; e < 2; ++e) {
+          const int G = G2 + e;
+          // x = z = acc / 64 - mu R (keys; acc / 64 is exact, so one
+          // rounding as fmul + fsub), or x = acc = 64 z (values, mu = 0:
+          // the group's range and codes are then taken in units of z / 64,
+          // exactly)
+          float x[32];
+          if (kind == 0) {
+            const float4* mu4 = reinterpret_cast<const float4*>(S.mu + 32 * G);
 #pragma unroll
-        for (int j = 1; j < 32; ++j) {
-          lo = fminf(lo, z[j]);
-          hi = fmaxf(hi, z[j]);
+            for (int j4 = 0; j4 < 8; ++j4) {
+              const float4 m = mu4[j4];
+              x[4 * j4 + 0] = fmaf(__uint_as_float(acc[e][4 * j4 + 0]), 1.0f / 64.0f, -m.x);
+              x[4 * j4 + 1] = fmaf(__uint_as_float(acc[e][4 * j4 + 1]), 1.0f / 64.0f, -m.y);
+              x[4 * j4 + 2] = fmaf(__uint_as_float(acc[e][4 * j4 + 2]), 1.0f / 64.0f, -m.z);
+              x[4 * j4 + 3] = fmaf(__uint_as_float(acc[e][4 * j4 + 3]), 1.0f / 64.0f, -m.w);
+            }
+          } else {
+#pragma unroll
+            for (int j = 0; j < 32; ++j) x[j] = __uint_as_float(acc[e][j]);
+          }
+          float lo, hi;
+          minmax32(x, lo, hi);
+          const float xs = kind ? 64.0f : 1.0f;  // x = xs * z
+          FastQuant q = fast_quant_params(lo * (1.0f / xs), hi * (1.0f / xs), clip);
+          range_err |= q.degenerate && !(fabsf(hi - lo) <= 3.402823466e38f);
+          q.mn *= xs;
+          q.mx *= xs;
+          q.inv4 *= 1.0f / xs;
+          code_bytes<kClamp>(x, q, bytes[e]);
+          meta[e] = q.meta;
         }
-        const GroupQuant gq = group_quant_params(lo, hi, clip);
-        range_err |= gq.degenerate && !(fabsf(hi - lo) <= 3.402823466e38f);
-        quantize_group<kClamp>(z, G, gq, word);
-        const __half2 sm = __halves2half2(gq.scale, gq.min);
-        meta[G] = *reinterpret_cast<const uint32_t*>(&sm);
+        // byte 0 of bytes[0][w] / bytes[1][w] to bytes 2hp, 2hp + 1 of the
+        // word (byte 1 of bytes[0][w] is zero)
+        const uint32_t sel = hp ? 0x4011u : 0x1140u;
+#pragma unroll
+        for (int w = 0; w < 8; ++w) word[w] = __byte_perm(bytes[0][w], bytes[1][w], sel);
       }
-      tc05::fence_before();  // accumulator reads done before the next MMA
       if (range_err && tok < n_tok) atomicOr(err, OPTR_DEVERR_FP16_RANGE);
-      if (dst >= 0) {
-        constexpr uint32_t kMagic = magic_sum();
-        uint4 c0, c1;
-        c0.x = word[0] - kMagic; c0.y = word[1] - kMagic;
-        c0.z = word[2] - kMagic; c0.w = word[3] - kMagic;
-        c1.x = word[4] - kMagic; c1.y = word[5] - kMagic;
-        c1.z = word[6] - kMagic; c1.w = word[7] - kMagic;
-        uint8_t* rec = pool + dst;
-        *reinterpret_cast<uint4*>(rec + codes_off + slot * 32) = c0;
-        *reinterpret_cast<uint4*>(rec + codes_off + slot * 32 + 16) = c1;
-        *reinterpret_cast<uint4*>(rec + meta_off + slot * 16) =
-            make_uint4(meta[0], meta[1], meta[2], meta[3]);
+      // the second half's code bytes to its partner, through shared memory
+      uint4* xw = S.xchg[g][row];
+      if (hp) {
+        // the partner has read this slot's previous contents
+        if (k > 0 && !__all_sync(0xffffffffu, tc05::bar_wait(&S.xdone[g], (k - 1) & 1, abort)))
+          break;
+        xw[0] = make_uint4(word[0], word[1], word[2], word[3]);
+        xw[1] = make_uint4(word[4], word[5], word[6], word[7]);
+        tc05::bar_arrive(&S.xready[g]);
+      } else {
+        if (!__all_sync(0xffffffffu, tc05::bar_wait(&S.xready[g], k & 1, abort))) break;
+        const uint4 y0 = xw[0], y1 = xw[1];
+        tc05::bar_arrive(&S.xdone[g]);
+        word[0] |= y0.x; word[1] |= y0.y; word[2] |= y0.z; word[3] |= y0.w;
+        word[4] |= y1.x; word[5] |= y1.y; word[6] |= y1.z; word[7] |= y1.w;
       }
+      if (dst >= 0) {
+        uint8_t* rec = pool + dst;
+        if (!hp) {
+          *reinterpret_cast<uint4*>(rec + codes_off + slot * 32) =
+              make_uint4(word[0], word[1], word[2], word[3]);
+          *reinterpret_cast<uint4*>(rec + codes_off + slot * 32 + 16) =
+              make_uint4(word[4], word[5], word[6], word[7]);
+        }
+        *reinterpret_cast<uint2*>(rec + meta_off + slot * 16 + 8 * hp) = make_uint2(meta[0], meta[1]);
+      }
+      __syncwarp();
     }
   }
 

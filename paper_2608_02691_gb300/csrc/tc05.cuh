@@ -8,7 +8,7 @@
 // >> 4 (distance between core matrices adjacent along M/N), bits [46,48) =
 // 1 (descriptor version), layout type 0 (no swizzle) in bits [61,64).
 // Instruction descriptor (kind::f16): bits [4,6) = 1 (f32 accumulator),
-// [7,10) / [10,13) = 0 (A and B f16), bits 15 / 16 = 0 (A and B K-major),
+// [7,10) / [10,13) = A and B type (0 f16, 1 bf16), bits 15 / 16 = 0 (A and B K-major),
 // [17,23) = N >> 3, [24,29) = M >> 4.
 #pragma once
 
@@ -30,6 +30,11 @@ __device__ __forceinline__ uint64_t smem_desc(uint32_t saddr, uint32_t lbo,
 
 __host__ __device__ constexpr uint32_t idesc_f16(int M, int N) {
   return (1u << 4) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+// As idesc_f16 with A and B bf16 (type 1 in bits [7,10) and [10,13)).
+__host__ __device__ constexpr uint32_t idesc_bf16(int M, int N) {
+  return idesc_f16(M, N) | (1u << 7) | (1u << 10);
 }
 
 __device__ __forceinline__ void bar_init(uint64_t* bar, uint32_t count) {
@@ -69,9 +74,12 @@ __device__ __forceinline__ bool bar_wait(uint64_t* bar, uint32_t parity,
   if (bar_try_wait(bar, parity)) return true;
   uint64_t t0;
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t0));
+  uint32_t ns = 32;  // back off: a sleeping warp leaves its issue slots to others
   for (uint32_t it = 1;; ++it) {
+    __nanosleep(ns);
     if (bar_try_wait(bar, parity)) return true;
-    if ((it & 63u) == 0) {
+    ns = ns < 256 ? 2 * ns : 256;
+    if ((it & 15u) == 0) {
       if (*abort) return false;
       uint64_t t;
       asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
