@@ -105,6 +105,7 @@ append_cuda_core_kernel(const __nv_bfloat16* __restrict__ k,
 }
 
 // Decode-step variant for few new tokens: append_small.cuh.
+template <int T>
 __global__ void __launch_bounds__(512)
 append_small_kernel(const __nv_bfloat16* __restrict__ k,
                     const __nv_bfloat16* __restrict__ v, int n_tok,
@@ -116,8 +117,8 @@ append_small_kernel(const __nv_bfloat16* __restrict__ k,
                     const float* __restrict__ R_v,
                     const float* __restrict__ muR, float clip_k, float clip_v,
                     unsigned* err) {
-  __shared__ AppendSmallSmem sm;
-  append_small_body(blockIdx.x, blockIdx.y, blockIdx.z, sm, k, v, n_tok,
+  __shared__ AppendSmallSmemT<T> sm;
+  append_small_body<T>(blockIdx.x, blockIdx.y, blockIdx.z, sm, k, v, n_tok,
                     cu_new, pos0, bt, B, max_pages, pool, num_pages, h_kv, R_k,
                     R_v, muR, clip_k, clip_v, err);
 }
@@ -133,8 +134,14 @@ cudaError_t launch_append_cuda_core(const optr_params* p,
                                     cudaStream_t s) {
   // few tokens (decode steps): slice-parallel rotation
   if (n_tok <= 256) {
-    dim3 grid((n_tok + kSmallTok - 1) / kSmallTok, p->cfg.h_kv, 2);
-    return launch_pdl(append_small_kernel, grid, dim3(512), 0, s, k, v, n_tok,
+    const int T = small_tile(n_tok);
+    dim3 grid((n_tok + T - 1) / T, p->cfg.h_kv, 2);
+    if (T == kSmallTokFew)
+      return launch_pdl(append_small_kernel<kSmallTokFew>, grid, dim3(512), 0, s, k, v,
+                        n_tok, cu_new, pos0, bt, B, max_pages, pool, num_pages,
+                        p->cfg.h_kv, p->R_k, p->R_v, p->muR, p->cfg.clip_k,
+                        p->cfg.clip_v, p->err);
+    return launch_pdl(append_small_kernel<kSmallTok>, grid, dim3(512), 0, s, k, v, n_tok,
                       cu_new, pos0, bt, B, max_pages, pool, num_pages,
                       p->cfg.h_kv, p->R_k, p->R_v, p->muR, p->cfg.clip_k,
                       p->cfg.clip_v, p->err);

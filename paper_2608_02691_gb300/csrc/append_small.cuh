@@ -9,33 +9,43 @@
 namespace optr {
 
 // Decode-step variant for few new tokens (one per sequence per step): one
-// CTA per (tile of 16 tokens, KV head, K or V), 512 threads = 4 slices x 128
-// channels.  Slice s accumulates z_j over i in [32s, 32s+32) for all 16
+// CTA per (tile of T tokens, KV head, K or V), 512 threads = 4 slices x 128
+// channels.  Slice s accumulates z_j over i in [32s, 32s+32) for all T
 // tokens; the slices are added in shared memory, then warp t quantizes and
-// packs token t group by group.
+// packs token t group by group.  T = 4 for at most 64 new tokens (4x the
+// CTAs, a quarter of the FMAs per thread: the decode step's latency), else
+// 16.
 constexpr int kSmallTok = 16;
+constexpr int kSmallTokFew = 4;
 constexpr int kSmallCuCache = 512;   // sequences whose cu_new / pos0 a CTA caches
 
-struct AppendSmallSmem {
-  float xs[kSmallTok][kD];
-  float zp[4][kSmallTok][kD];
-  long long dst[kSmallTok];
-  int dslot[kSmallTok];
+__host__ __device__ constexpr int small_tile(int n_tok) {
+  return n_tok <= 64 ? kSmallTokFew : kSmallTok;
+}
+
+template <int T>
+struct AppendSmallSmemT {
+  float xs[T][kD];
+  float zp[4][T][kD];
+  long long dst[T];
+  int dslot[T];
   int s_cu[kSmallCuCache + 1];
   int s_p0[kSmallCuCache];
 };
+using AppendSmallSmem = AppendSmallSmemT<kSmallTok>;  // the larger one
 
-// CTA (tblk, h, kind) of the cache write: tokens [16*tblk, 16*tblk + 16),
+// CTA (tblk, h, kind) of the cache write: tokens [T*tblk, T*tblk + T),
 // KV head h, kind 0 = keys, 1 = values.  512 threads.
+template <int T>
 __device__ __forceinline__ void append_small_body(
-    int tblk, int h, int kind, AppendSmallSmem& sm,
+    int tblk, int h, int kind, AppendSmallSmemT<T>& sm,
     const __nv_bfloat16* __restrict__ k, const __nv_bfloat16* __restrict__ v,
     int n_tok, const int32_t* __restrict__ cu_new,
     const int32_t* __restrict__ pos0, const int32_t* __restrict__ bt, int B,
     int max_pages, uint8_t* __restrict__ pool, int num_pages, int h_kv,
     const float* __restrict__ R_k, const float* __restrict__ R_v,
     const float* __restrict__ muR, float clip_k, float clip_v, unsigned* err) {
-  constexpr int T = kSmallTok;
+  static_assert(T <= 16, "one quantizing warp per token");
   float (&xs)[T][kD] = sm.xs;
   float (&zp)[4][T][kD] = sm.zp;
   long long (&dst)[T] = sm.dst;
@@ -68,21 +78,40 @@ __device__ __forceinline__ void append_small_body(
       s_cu[i] = __ldg(cu_new + i);
       if (i < B) s_p0[i] = __ldg(pos0 + i);
     }
-    __syncthreads();
-  }
-  if (tid < T) {
-    const int tok = t0 + tid;
-    int slot = 0;
-    long long off = -1;
-    if (tok < n_tok)
-      off = cached ? resolve_slot_cached(tok, h, s_cu, s_p0, bt, B, max_pages,
-                                         num_pages, h_kv, &slot, err)
-                   : resolve_slot(tok, h, cu_new, pos0, bt, B, max_pages,
-                                  num_pages, h_kv, &slot, err);
-    dst[tid] = off;
-    dslot[tid] = slot;
   }
   __syncthreads();
+  // Slot of token t0 + tid (threads < T), in two halves around the
+  // rotation: the block-table entry is requested here and checked after the
+  // FMAs, so its load latency overlaps them (resolve_slot's checks).
+  const int my_tok = t0 + tid;
+  const bool resolver = tid < T && my_tok < n_tok;
+  long long off = -1;
+  int slot = 0, page = -1;
+  unsigned bad = 0;
+  if (resolver) {
+    if (cached) {
+      int lo = 0, hi = B;
+      while (hi - lo > 1) {
+        const int mid = (lo + hi) >> 1;
+        if (s_cu[mid] <= my_tok) lo = mid; else hi = mid;
+      }
+      const int c0 = s_cu[lo], c1 = s_cu[lo + 1];
+      if (!(c0 <= my_tok && my_tok < c1)) {
+        bad = OPTR_DEVERR_CU_NEW;
+      } else {
+        const long long pos = (long long)s_p0[lo] + (my_tok - c0);
+        if (pos < 0 || pos >= (long long)max_pages * kPage) {
+          bad = OPTR_DEVERR_POSITION;
+        } else {
+          slot = (int)(pos % kPage);
+          page = __ldg(bt + (size_t)lo * max_pages + pos / kPage);
+        }
+      }
+    } else {
+      off = resolve_slot(my_tok, h, cu_new, pos0, bt, B, max_pages, num_pages,
+                         h_kv, &slot, err);
+    }
+  }
   float acc[T];
 #pragma unroll
   for (int t = 0; t < T; ++t) acc[t] = 0.f;
@@ -92,16 +121,30 @@ __device__ __forceinline__ void append_small_body(
     for (int t = 0; t < T; ++t) acc[t] = fmaf(xs[t][32 * sl + i], rv[i], acc[t]);
 #pragma unroll
   for (int t = 0; t < T; ++t) zp[sl][t][j] = acc[t];
+  if (tid < T) {
+    if (resolver && cached) {
+      if (bad) {
+        atomicOr(err, bad);
+      } else if (page < 0 || page >= num_pages) {
+        atomicOr(err, OPTR_DEVERR_PAGE_ID);
+      } else {
+        off = ((long long)page * h_kv + h) * kChunk;
+      }
+    }
+    dst[tid] = off;
+    dslot[tid] = slot;
+  }
   __syncthreads();
 
   const int warp = tid >> 5, lane = tid & 31;  // warp = token of the tile
-  const long long off = dst[warp];
-  if (t0 + warp >= n_tok || off < 0) return;
-  const int slot = dslot[warp];
+  if (warp >= T) return;
+  const long long woff = dst[warp];
+  if (t0 + warp >= n_tok || woff < 0) return;
+  const int wslot = dslot[warp];
   const float clip = kind ? clip_v : clip_k;
   const int codes_off = kind ? OPTR_V_CODES_OFFSET : OPTR_K_CODES_OFFSET;
   const int meta_off = kind ? OPTR_V_META_OFFSET : OPTR_K_META_OFFSET;
-  uint8_t* chunk = pool + off;
+  uint8_t* chunk = pool + woff;
 #pragma unroll
   for (int g = 0; g < kGroups; ++g) {
     const int jj = 32 * g + lane;
@@ -118,9 +161,9 @@ __device__ __forceinline__ void append_small_body(
     bits |= __shfl_xor_sync(0xffffffffu, bits, 1);
     bits |= __shfl_xor_sync(0xffffffffu, bits, 2);
     if ((lane & 3) == 0)
-      chunk[codes_off + slot * 32 + 4 * (lane >> 2) + g] = (uint8_t)bits;
+      chunk[codes_off + wslot * 32 + 4 * (lane >> 2) + g] = (uint8_t)bits;
     if (lane == 0)
-      *reinterpret_cast<__half2*>(chunk + meta_off + slot * 16 + 4 * g) =
+      *reinterpret_cast<__half2*>(chunk + meta_off + wslot * 16 + 4 * g) =
           __halves2half2(gq.scale, gq.min);
   }
 }

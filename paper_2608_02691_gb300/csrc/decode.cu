@@ -34,7 +34,7 @@ struct QrotSmem {
   float qrs[4][kD];
   float hmax[4][4];
   int warp_tot[2][kQrotThreads / 32];
-  double koff_part[kQrotThreads / 32][kGroups];
+  long long koff_part[kQrotThreads / 32][kGroups];
 };
 
 // CTA (b, h) of the query rotation; 512 threads.
@@ -50,7 +50,7 @@ __device__ __forceinline__ void qrot_body(
   float (&qrs)[4][kD] = sm.qrs;
   float (&hmax)[4][4] = sm.hmax;
   int (&warp_tot)[2][kQrotThreads / 32] = sm.warp_tot;
-  double (&koff_part)[kQrotThreads / 32][kGroups] = sm.koff_part;
+  long long (&koff_part)[kQrotThreads / 32][kGroups] = sm.koff_part;
   const int tid = threadIdx.x;
   const int sl = tid >> 7, j = tid & 127;
   const int warp = tid >> 5, lane = tid & 31;
@@ -68,9 +68,15 @@ __device__ __forceinline__ void qrot_body(
   }
   __syncthreads();
 #pragma unroll
-  for (int i = 0; i < 32; ++i)
+  for (int i4 = 0; i4 < 8; ++i4)
 #pragma unroll
-    for (int r = 0; r < 4; ++r) acc[r] = fmaf(qsm[r][32 * sl + i], rv[i], acc[r]);
+    for (int r = 0; r < 4; ++r) {
+      const float4 qv = *reinterpret_cast<const float4*>(&qsm[r][32 * sl + 4 * i4]);
+      acc[r] = fmaf(qv.x, rv[4 * i4 + 0], acc[r]);
+      acc[r] = fmaf(qv.y, rv[4 * i4 + 1], acc[r]);
+      acc[r] = fmaf(qv.z, rv[4 * i4 + 2], acc[r]);
+      acc[r] = fmaf(qv.w, rv[4 * i4 + 3], acc[r]);
+    }
 #pragma unroll
   for (int r = 0; r < 4; ++r) part[sl][r][j] = acc[r];
   __syncthreads();
@@ -123,8 +129,12 @@ __device__ __forceinline__ void qrot_body(
     frag[((size_t)b * h_kv + h) * 512 + ridx] =
         (uint32_t)__half_as_ushort(v0) | ((uint32_t)__half_as_ushort(v1) << 16);
     // offset sum over the 32 channels of group G for column g: reduce over
-    // (kk, which) = lane bits 0-1, c bit 0 = lane bit 4, c bit 1 = warp bit 0
-    double t = (double)__half2float(v0) + (double)__half2float(v1);
+    // (kk, which) = lane bits 0-1, c bit 0 = lane bit 4, c bit 1 = warp bit 0.
+    // Exact, in fixed point: an fp16 value times 2^24 is an integer below
+    // 2^40, so 64 of them sum exactly in int64; one rounding to float, then
+    // 1024 * 2^-24 = 2^-14 (exact) gives the correctly rounded koff.
+    long long t = __float2ll_rn(__half2float(v0) * 16777216.0f) +
+                  __float2ll_rn(__half2float(v1) * 16777216.0f);
     t += __shfl_xor_sync(0xffffffffu, t, 1);
     t += __shfl_xor_sync(0xffffffffu, t, 2);
     t += __shfl_xor_sync(0xffffffffu, t, 16);
@@ -132,9 +142,9 @@ __device__ __forceinline__ void qrot_body(
     __syncthreads();
     if (tid < 32) {  // tid = (g, G): koff[head][G][hl] for column g
       const int gg = tid >> 2, GG = tid & 3;
-      const double tot = koff_part[2 * gg][GG] + koff_part[2 * gg + 1][GG];
+      const long long tot = koff_part[2 * gg][GG] + koff_part[2 * gg + 1][GG];
       koff[((size_t)b * h_kv + h) * 32 + (gg >> 1) * 8 + GG * 2 + (gg & 1)] =
-          (float)(1024.0 * tot);
+          __ll2float_rn(tot) * 0x1p-14f;
     }
     if (ridx < 4) {
       const float m2 = fmaxf(fmaxf(hmax[ridx][0], hmax[ridx][1]),
@@ -199,6 +209,7 @@ qrot_kernel(const __nv_bfloat16* __restrict__ q, const float* __restrict__ R_k,
 // inputs; the partial kernel then waits for this grid, i.e. for both.
 static_assert(kQrotThreads == 512, "one block size for both bodies");
 
+template <int T>
 __global__ void __launch_bounds__(512)
 step_prologue_kernel(
     int n_app, int app_tiles, const __nv_bfloat16* __restrict__ k,
@@ -217,7 +228,7 @@ step_prologue_kernel(
   if (bid < n_app) {
     const int tblk = bid % app_tiles, hk = (bid / app_tiles) % h_kv,
               kind = bid / (app_tiles * h_kv);
-    append_small_body(tblk, hk, kind, *reinterpret_cast<AppendSmallSmem*>(dsm_),
+    append_small_body<T>(tblk, hk, kind, *reinterpret_cast<AppendSmallSmemT<T>*>(dsm_),
                       k, v, n_tok, cu_new, pos0, bt, B, max_pages, pool,
                       num_pages, h_kv, R_k, R_v, muR, clip_k, clip_v, err);
   } else {
@@ -650,14 +661,17 @@ cudaError_t launch_decode(const optr_params* p, int variant,
   if (app) {
     // the cache write of the step and the query rotation in one launch
     prof_mark(p, 0, s);
-    const int tiles = (app->n_tok + kSmallTok - 1) / kSmallTok;
+    const int T = small_tile(app->n_tok);
+    const int tiles = (app->n_tok + T - 1) / T;
     const int n_app = tiles * h_kv * 2;
-    const size_t sm_bytes = sizeof(AppendSmallSmem) > sizeof(QrotSmem)
-                                ? sizeof(AppendSmallSmem) : sizeof(QrotSmem);
-    e = ensure_dynamic_smem(reinterpret_cast<const void*>(&step_prologue_kernel),
-                            sm_bytes);
+    const size_t sm_app = T == kSmallTokFew ? sizeof(AppendSmallSmemT<kSmallTokFew>)
+                                            : sizeof(AppendSmallSmemT<kSmallTok>);
+    const size_t sm_bytes = sm_app > sizeof(QrotSmem) ? sm_app : sizeof(QrotSmem);
+    auto fn = T == kSmallTokFew ? step_prologue_kernel<kSmallTokFew>
+                                : step_prologue_kernel<kSmallTok>;
+    e = ensure_dynamic_smem(reinterpret_cast<const void*>(fn), sm_bytes);
     if (e != cudaSuccess) return e;
-    e = launch_pdl(step_prologue_kernel, dim3(n_app + B * h_kv), dim3(512),
+    e = launch_pdl(fn, dim3(n_app + B * h_kv), dim3(512),
                    sm_bytes, s, n_app, tiles, app->k, app->v, app->n_tok,
                    app->cu_new, app->pos0, bt, app->pool, num_pages,
                    (const float*)p->R_v, (const float*)p->muR, p->cfg.clip_k,
