@@ -61,7 +61,8 @@ __device__ __forceinline__ void qrot_body(
   for (int i = 0; i < 32; ++i) rv[i] = __ldg(R + i * kD);  // all in flight
   pdl_wait();  // the query, lengths and workspace may belong to earlier kernels
   pdl_trigger();
-  if (tid == 0) cnt_ws[(size_t)b * h_kv + h] = 0;  // combine arrivals
+  // Global stores wait until the end: a __syncthreads() after a store waits
+  // for it to complete, which made each phase an L2 round trip.
   {
     const int r = tid >> 7;  // 512 threads load the 4 x 128 query values
     qsm[r][j] = __bfloat162float(q[((size_t)b * h_q + 4 * h + r) * kD + j]);
@@ -80,12 +81,14 @@ __device__ __forceinline__ void qrot_body(
 #pragma unroll
   for (int r = 0; r < 4; ++r) part[sl][r][j] = acc[r];
   __syncthreads();
-  if (tid < 4 * kD) {
-    // thread (r, j): the 4 slices of head r, channel j
-    const int r = tid >> 7;
-    const float x = (part[0][r][j] + part[1][r][j] + part[2][r][j] + part[3][r][j]) * qscale;
-    const size_t row = (size_t)b * h_q + 4 * h + r;
-    qf[row * kD + j] = x;
+  // thread (r, j): the 4 slices of head r, channel j (512 threads)
+  const int qr = tid >> 7;
+  const size_t qrow = (size_t)b * h_q + 4 * h + qr;
+  const float qx = (part[0][qr][j] + part[1][qr][j] + part[2][qr][j] + part[3][qr][j]) * qscale;
+  float qsum = qx;
+  {
+    const int r = qr;
+    const float x = qx;
     qrs[r][j] = x;
     float s = x, a = fabsf(x);
 #pragma unroll
@@ -93,10 +96,8 @@ __device__ __forceinline__ void qrot_body(
       s += __shfl_xor_sync(0xffffffffu, s, o);
       a = fmaxf(a, __shfl_xor_sync(0xffffffffu, a, o));
     }
-    if (lane == 0) {
-      qs[row * kGroups + (j >> 5)] = s;
-      hmax[r][j >> 5] = a;
-    }
+    qsum = s;
+    if (lane == 0) hmax[r][j >> 5] = a;
   }
   __syncthreads();
   // Tensor-core B fragments (see decode_tc.cu): per head a power-of-two
@@ -126,7 +127,7 @@ __device__ __forceinline__ void qrot_body(
       v0 = __float2half_rn(x0 - __half2float(h0));
       v1 = __float2half_rn(x1 - __half2float(h1));
     }
-    frag[((size_t)b * h_kv + h) * 512 + ridx] =
+    const uint32_t fragv =
         (uint32_t)__half_as_ushort(v0) | ((uint32_t)__half_as_ushort(v1) << 16);
     // offset sum over the 32 channels of group G for column g: reduce over
     // (kk, which) = lane bits 0-1, c bit 0 = lane bit 4, c bit 1 = warp bit 0.
@@ -152,7 +153,11 @@ __device__ __forceinline__ void qrot_body(
       const int e2 = max(-100, min(100, m2 > 0.f ? 13 - ilogbf(m2) : 0));
       invs[(size_t)b * h_q + 4 * h + ridx] = ldexpf(1.f, -e2);
     }
+    frag[((size_t)b * h_kv + h) * 512 + ridx] = fragv;
   }
+  qf[qrow * kD + j] = qx;
+  if (lane == 0) qs[qrow * kGroups + (j >> 5)] = qsum;
+  if (tid == 0) cnt_ws[(size_t)b * h_kv + h] = 0;  // combine arrivals
 
   if (b != 0 || h != 0) return;
   // Split-K plan: pref[b] = pages of sequences < b, nzpref[b] = non-empty
