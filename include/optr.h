@@ -161,7 +161,13 @@ typedef struct {
  *   cfg   host; shapes and clip ratios (copied).
  *   R_k   host float32 [h_kv][D][D]: key rotation per KV head (orthogonal;
  *         orthogonality is the caller's contract and is not checked).
- *   R_v   host float32 [h_kv][D][D]: value rotation per KV head.
+ *   R_v   host float32 [h_kv][D][D]: value rotation per KV head, or NULL
+ *         when the value rotation is folded into the model's projections
+ *         (Appendix "Equivalent Inference Implementation": W_V and W_O
+ *         pre-multiplied by R_v): values are then quantized as given and
+ *         the decode output is returned in that basis (as R_v = I; the
+ *         decode skips its R_v^T step, the decode-step cache write its
+ *         value rotation).
  *   mu    host float32 [h_kv][D]: per-channel key mean (Appendix, key-mean
  *         estimation).  Pass all zeros for no centering.
  *   out   host; receives the new handle, or NULL on error.

@@ -116,11 +116,11 @@ append_small_kernel(const __nv_bfloat16* __restrict__ k,
                     const float* __restrict__ R_k,
                     const float* __restrict__ R_v,
                     const float* __restrict__ muR, float clip_k, float clip_v,
-                    unsigned* err) {
+                    unsigned* err, int fold_v) {
   __shared__ AppendSmallSmemT<T> sm;
   append_small_body<T>(blockIdx.x, blockIdx.y, blockIdx.z, sm, k, v, n_tok,
                     cu_new, pos0, bt, B, max_pages, pool, num_pages, h_kv, R_k,
-                    R_v, muR, clip_k, clip_v, err);
+                    R_v, muR, clip_k, clip_v, err, fold_v && blockIdx.z == 1);
 }
 
 }  // namespace
@@ -140,11 +140,11 @@ cudaError_t launch_append_cuda_core(const optr_params* p,
       return launch_pdl(append_small_kernel<kSmallTokFew>, grid, dim3(512), 0, s, k, v,
                         n_tok, cu_new, pos0, bt, B, max_pages, pool, num_pages,
                         p->cfg.h_kv, p->R_k, p->R_v, p->muR, p->cfg.clip_k,
-                        p->cfg.clip_v, p->err);
+                        p->cfg.clip_v, p->err, p->fold_v);
     return launch_pdl(append_small_kernel<kSmallTok>, grid, dim3(512), 0, s, k, v, n_tok,
                       cu_new, pos0, bt, B, max_pages, pool, num_pages,
                       p->cfg.h_kv, p->R_k, p->R_v, p->muR, p->cfg.clip_k,
-                      p->cfg.clip_v, p->err);
+                      p->cfg.clip_v, p->err, p->fold_v);
   } else {
     constexpr int T = 32;
     dim3 grid((n_tok + T - 1) / T, p->cfg.h_kv);

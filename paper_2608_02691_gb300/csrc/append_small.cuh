@@ -44,7 +44,10 @@ __device__ __forceinline__ void append_small_body(
     const int32_t* __restrict__ pos0, const int32_t* __restrict__ bt, int B,
     int max_pages, uint8_t* __restrict__ pool, int num_pages, int h_kv,
     const float* __restrict__ R_k, const float* __restrict__ R_v,
-    const float* __restrict__ muR, float clip_k, float clip_v, unsigned* err) {
+    const float* __restrict__ muR, float clip_k, float clip_v, unsigned* err,
+    bool identity = false) {
+  // identity: z = x, no rotation (values with the rotation folded into the
+  // model's projections)
   static_assert(T <= 16, "one quantizing warp per token");
   float (&xs)[T][kD] = sm.xs;
   float (&zp)[4][T][kD] = sm.zp;
@@ -59,7 +62,7 @@ __device__ __forceinline__ void append_small_body(
   const float* R = (kind ? R_v : R_k) + (size_t)h * kD * kD + (size_t)(32 * sl) * kD + j;
   float rv[32];
 #pragma unroll
-  for (int i = 0; i < 32; ++i) rv[i] = __ldg(R + i * kD);
+  for (int i = 0; i < 32; ++i) rv[i] = identity ? 0.f : __ldg(R + i * kD);
   float musub[kGroups];  // mu R_k of this lane's channel in each group (keys)
 #pragma unroll
   for (int g = 0; g < kGroups; ++g)
@@ -112,15 +115,20 @@ __device__ __forceinline__ void append_small_body(
                          h_kv, &slot, err);
     }
   }
-  float acc[T];
+  if (identity) {
 #pragma unroll
-  for (int t = 0; t < T; ++t) acc[t] = 0.f;
+    for (int t = 0; t < T; ++t) zp[sl][t][j] = sl == 0 ? xs[t][j] : 0.f;
+  } else {
+    float acc[T];
 #pragma unroll
-  for (int i = 0; i < 32; ++i)
+    for (int t = 0; t < T; ++t) acc[t] = 0.f;
 #pragma unroll
-    for (int t = 0; t < T; ++t) acc[t] = fmaf(xs[t][32 * sl + i], rv[i], acc[t]);
+    for (int i = 0; i < 32; ++i)
 #pragma unroll
-  for (int t = 0; t < T; ++t) zp[sl][t][j] = acc[t];
+      for (int t = 0; t < T; ++t) acc[t] = fmaf(xs[t][32 * sl + i], rv[i], acc[t]);
+#pragma unroll
+    for (int t = 0; t < T; ++t) zp[sl][t][j] = acc[t];
+  }
   if (tid < T) {
     if (resolver && cached) {
       if (bad) {

@@ -227,7 +227,7 @@ step_prologue_kernel(
     const int32_t* __restrict__ seq_lens, int max_pages,
     float* __restrict__ qf, float* __restrict__ qs, uint32_t* __restrict__ frag,
     float* __restrict__ koff, float* __restrict__ invs, int* __restrict__ pref,
-    int* __restrict__ nzpref, int* __restrict__ cnt_ws, unsigned* err) {
+    int* __restrict__ nzpref, int* __restrict__ cnt_ws, unsigned* err, int fold_v) {
   extern __shared__ __align__(16) unsigned char dsm_[];
   const int bid = blockIdx.x;
   if (bid < n_app) {
@@ -235,7 +235,8 @@ step_prologue_kernel(
               kind = bid / (app_tiles * h_kv);
     append_small_body<T>(tblk, hk, kind, *reinterpret_cast<AppendSmallSmemT<T>*>(dsm_),
                       k, v, n_tok, cu_new, pos0, bt, B, max_pages, pool,
-                      num_pages, h_kv, R_k, R_v, muR, clip_k, clip_v, err);
+                      num_pages, h_kv, R_k, R_v, muR, clip_k, clip_v, err,
+                      fold_v && kind == 1);
   } else {
     const int r = bid - n_app;
     qrot_body(r / h_kv, r % h_kv, *reinterpret_cast<QrotSmem*>(dsm_), q, R_k, B,
@@ -511,7 +512,7 @@ __global__ void __launch_bounds__(kCombineThreads)
 combine_kernel(const float* __restrict__ part, const int* __restrict__ pref,
                const int* __restrict__ nzpref, int B, int h_q, int h_kv, int W,
                const float* __restrict__ R_vT, float* __restrict__ cpart,
-               int* __restrict__ cnt_ws, float* __restrict__ out) {
+               int* __restrict__ cnt_ws, float* __restrict__ out, int fold_v) {
   extern __shared__ float4 dsm[];
   float* rts = reinterpret_cast<float*>(dsm);  // [128][128] R_v^T[h]
   __shared__ float4 msum[4][kD];               // [phase][float4 of o']
@@ -520,13 +521,13 @@ combine_kernel(const float* __restrict__ part, const int* __restrict__ pref,
   __shared__ int last;
   const int b = blockIdx.x, h = blockIdx.y, sp = blockIdx.z, S = gridDim.z;
   const int tid = threadIdx.x;
-  {
+  if (!fold_v) {
     const float4* src = reinterpret_cast<const float4*>(R_vT + (size_t)h * kD * kD);
 #pragma unroll
     for (int u = 0; u < kD * kD / 4 / kCombineThreads; ++u)
       cp_async16(&dsm[tid + u * kCombineThreads], src + tid + u * kCombineThreads);
-    cp_async_commit();
   }
+  cp_async_commit();
   if (tid < 4) {
     st.M[tid] = -INFINITY;
     st.L[tid] = 0.f;
@@ -610,6 +611,10 @@ combine_kernel(const float* __restrict__ part, const int* __restrict__ pref,
   }
   cp_async_wait<0>();
   __syncthreads();
+  if (fold_v) {  // output in the folded value basis: no R_v^T
+    ob[tid] = orot[tid >> 7][tid & 127];
+    return;
+  }
   // out[r][i] = sum_k o'[r][k] R_v[i][k] = sum_k o'[r][k] R_vT[k][i]:
   // thread (i, q) sums k in [32q, 32q + 32) for the 4 heads, reading each
   // R_v^T element once; the 4 quarters are added through shared memory.
@@ -682,7 +687,7 @@ cudaError_t launch_decode(const optr_params* p, int variant,
                    (const float*)p->R_v, (const float*)p->muR, p->cfg.clip_k,
                    p->cfg.clip_v, q, (const float*)p->R_k, B, h_q, h_kv, qscale,
                    seq_lens, max_pages, qf, qs, frag, koff, invs, pref, nzpref,
-                   cnt_ws, p->err);
+                   cnt_ws, p->err, p->fold_v);
     if (e != cudaSuccess) return e;
     prof_mark(p, 1, s);  // the append stage covers the fused launch,
     prof_mark(p, 2, s);  // the query-rotation stage is empty
@@ -716,7 +721,7 @@ cudaError_t launch_decode(const optr_params* p, int variant,
                  cmb_bytes, s, (const float*)part, (const int*)pref,
                  (const int*)nzpref, B, h_q, h_kv, plan.W, (const float*)p->R_vT,
                  reinterpret_cast<float*>(w + plan.off_cpart),
-                 reinterpret_cast<int*>(w + plan.off_cnt), out);
+                 reinterpret_cast<int*>(w + plan.off_cnt), out, p->fold_v);
   if (e != cudaSuccess) return e;
   prof_mark(p, 5, s);
   return cudaSuccess;

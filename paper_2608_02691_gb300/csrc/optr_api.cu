@@ -128,7 +128,7 @@ optr_status optr_params_create(const optr_config* cfg, const float* R_k,
                                const float* R_v, const float* mu,
                                optr_params** out) {
   if (out) *out = nullptr;
-  if (!cfg || !R_k || !R_v || !mu || !out) return OPTR_ERR_INVALID_ARG;
+  if (!cfg || !R_k || !mu || !out) return OPTR_ERR_INVALID_ARG;
   if (cfg->h_kv <= 0 || cfg->h_q <= 0 || cfg->h_q % cfg->h_kv != 0)
     return OPTR_ERR_INVALID_ARG;
   if (cfg->head_dim != kD || cfg->group != kG || cfg->page_size != kPage ||
@@ -141,6 +141,18 @@ optr_status optr_params_create(const optr_config* cfg, const float* R_k,
 
   const int H = cfg->h_kv;
   const size_t mat = (size_t)kD * kD;
+  // R_v = NULL: the value rotation is folded into the model's W_V and W_O
+  // (Appendix "Equivalent Inference Implementation"); the library then
+  // quantizes values as given and returns the output in that basis, i.e.
+  // it runs with R_v = I and skips the work where that is cheap.
+  const bool fold_v = R_v == nullptr;
+  std::vector<float> eye;
+  if (fold_v) {
+    eye.assign((size_t)H * mat, 0.f);
+    for (int h = 0; h < H; ++h)
+      for (int i = 0; i < kD; ++i) eye[(size_t)h * mat + (size_t)i * kD + i] = 1.f;
+    R_v = eye.data();
+  }
   // Host-side preparation: mu R_k in fp64, R_v transposed.
   std::vector<float> muR((size_t)H * kD), RvT((size_t)H * mat);
   for (int h = 0; h < H; ++h) {
@@ -161,6 +173,7 @@ optr_status optr_params_create(const optr_config* cfg, const float* R_k,
   if (!p) return OPTR_ERR_OUT_OF_RANGE;
   p->cfg = *cfg;
   p->ratio = cfg->h_q / cfg->h_kv;
+  p->fold_v = fold_v ? 1 : 0;
   cudaError_t e = cudaGetDevice(&p->device);
   if (e == cudaSuccess)
     e = cudaDeviceGetAttribute(&p->num_sms, cudaDevAttrMultiProcessorCount,

@@ -30,6 +30,7 @@ struct optr_params {
   int device;
   int num_sms;
   int ratio;           // h_q / h_kv
+  int fold_v;          // R_v folded into the model's W_V / W_O (R_v = I here)
   float* R_k;          // device [h_kv][D][D]
   float* R_v;          // device [h_kv][D][D]
   float* R_vT;         // device [h_kv][D][D], R_vT[h][j][i] = R_v[h][i][j]

@@ -137,18 +137,21 @@ def optr_params_create(R_k, R_v, mu, h_q: int, clip_k: float = 1.0,
                        append_variant: int = OPTR_VARIANT_DEFAULT,
                        decode_variant: int = OPTR_VARIANT_DEFAULT) -> Params:
     """R_k, R_v float32 [h_kv][128][128] and mu float32 [h_kv][128] (host
-    tensors); the library copies them to the current CUDA device."""
+    tensors); the library copies them to the current CUDA device.  R_v may be
+    None: the value rotation is folded into the model's W_V / W_O."""
     R_k = R_k.detach().to("cpu", torch.float32).contiguous()
-    R_v = R_v.detach().to("cpu", torch.float32).contiguous()
+    if R_v is not None:
+        R_v = R_v.detach().to("cpu", torch.float32).contiguous()
     mu = mu.detach().to("cpu", torch.float32).contiguous()
     h_kv = R_k.shape[0]
-    if R_k.shape != (h_kv, 128, 128) or R_v.shape != R_k.shape or \
+    if R_k.shape != (h_kv, 128, 128) or (R_v is not None and R_v.shape != R_k.shape) or \
             mu.shape != (h_kv, 128):
         raise ValueError("R_k, R_v must be [h_kv][128][128], mu [h_kv][128]")
     cfg = optr_config(h_q, h_kv, 128, 32, 16, clip_k, clip_v, append_variant,
                       decode_variant)
     h = ctypes.c_void_p()
-    _check(lib().optr_params_create(ctypes.byref(cfg), _ptr(R_k), _ptr(R_v),
+    _check(lib().optr_params_create(ctypes.byref(cfg), _ptr(R_k),
+                                    None if R_v is None else _ptr(R_v),
                                     _ptr(mu), ctypes.byref(h)),
            "optr_params_create")
     return Params(h, cfg)
