@@ -290,28 +290,109 @@ static void attend(const double* qr, const double* khat, const double* vhat,
   free(l);
 }
 
+/* ------------------------------------------------------- BF16 windows */
+
+/*
+ * BF16 windows (Sec. 3.1, opening paragraph: the long history is stored in
+ * INT2 while a small BF16 window is kept; Sec. 4.1: sink and recent tokens
+ * stay in BF16 and their keys receive the same centering by mu; Sec. 5,
+ * "Implementation Details": 64 sink and 256 recent tokens).  Of a sequence
+ * that holds n tokens, position s is a window position when s < sink (the
+ * attention sink) or s >= n - recent (the most recent tokens).  Its
+ * effective key is k_s - mu and its effective value v_s, from the exact bf16
+ * inputs, with no rotation or quantization; every other position attends
+ * with its rotated INT2 record.
+ *
+ * Window store (the library's layout, restated from include/optr.h):
+ * bf16 bits [n_slots][h_kv][2][sink + recent][128], index 0 keys, 1 values;
+ * position s lives in row s when s < sink, else in row
+ * sink + (s - sink) % recent.
+ */
+static int in_window(int s, int n, int sink, int recent) {
+  return s < sink || s >= n - recent;
+}
+
+static int window_row(int s, int sink, int recent) {
+  return s < sink ? s : sink + (s - sink) % recent;
+}
+
+static const uint16_t* window_vec(const uint16_t* win, int slot, int h_kv,
+                                  int h, int kind, int row, int sink,
+                                  int recent) {
+  size_t rows = (size_t)(sink + recent);
+  return win + ((((size_t)slot * h_kv + h) * 2 + kind) * rows + row) * OR_D;
+}
+
+/*
+ * Window part of a cache write.  Sequence b's new tokens (rows cu_new[b] ..
+ * cu_new[b+1]-1 of k / v) take positions pos0[b] .. end-1; a position s is
+ * copied into the store when s < sink, or when recent > 0 and
+ * s >= end - recent (those still in the recent window once this write is
+ * cached; the ring row of an older position is overwritten in position
+ * order).  k, v: bf16 bits [n_tok][h_kv][128].  Returns 0, or -1 when a
+ * window slot is out of range (nothing is written for that sequence).
+ */
+int oracle_window_write(const uint16_t* k, const uint16_t* v, int n_tok,
+                        const int32_t* cu_new, const int32_t* pos0, int B,
+                        const int32_t* win_slot, int n_slots, int h_kv,
+                        int sink, int recent, uint16_t* win) {
+  int bad = 0;
+  if (cu_new[0] != 0 || cu_new[B] != n_tok) return -1;
+  for (int b = 0; b < B; ++b) {
+    int m = cu_new[b + 1] - cu_new[b];
+    if (m <= 0) continue;
+    int slot = win_slot[b];
+    if (slot < 0 || slot >= n_slots) { bad = 1; continue; }
+    int end = pos0[b] + m;
+    for (int i = 0; i < m; ++i) {
+      int s = pos0[b] + i;
+      if (!(s < sink || (recent > 0 && s >= end - recent))) continue;
+      int row = window_row(s, sink, recent);
+      int t = cu_new[b] + i;
+      for (int h = 0; h < h_kv; ++h) {
+        memcpy((void*)window_vec(win, slot, h_kv, h, 0, row, sink, recent),
+               k + ((size_t)t * h_kv + h) * OR_D, OR_D * sizeof(uint16_t));
+        memcpy((void*)window_vec(win, slot, h_kv, h, 1, row, sink, recent),
+               v + ((size_t)t * h_kv + h) * OR_D, OR_D * sizeof(uint16_t));
+      }
+    }
+  }
+  return bad ? -1 : 0;
+}
+
 /*
  * Decode attention over the paged INT2 cache (Sec. 3 Eq. 1-2; Appendix,
  * "Rotated-query implementation": the cache stores k_R = Q2((k-mu)R_K) and
  * the query is rotated instead, q' = q R_K; Appendix, "Equivalent Inference
- * Implementation": o' = o R_V and o = o' R_V^T).  For each selected
- * (b, j): h = j / (h_q / h_kv), tokens s < seq_lens[b],
- *     l_s = <q_j R_K,h, khat_R,s> / sqrt(128),  p = softmax(l),
- *     out_j = (sum_s p_s vhat_R,s) R_V,h^T.
+ * Implementation": o' = o R_V and o = o' R_V^T), with BF16 windows (above).
+ * For each selected (b, j): h = j / (h_q / h_kv), tokens s < n = seq_lens[b],
+ *     INT2 s:    l_s = <q_j R_K,h, khat_R,s> / sqrt(128), value vhat_R,s
+ *     window s:  l_s = <q_j, k_s - mu_h> / sqrt(128),     value v_s
+ *     p = softmax(l),
+ *     out_j = (sum_INT2 p_s vhat_R,s) R_V,h^T + sum_window p_s v_s.
+ * Without windows (sink = recent = 0) this is the INT2 path alone, and the
+ * query-independent -q.mu term of the INT2 logits needs no explicit
+ * treatment (softmax invariance); with windows the window logits carry it
+ * explicitly so that both kinds of logits are those of centered keys.
  * q: bf16 bits [B][h_q][128].  out: float64 [B][h_q][128]; only selected
  * rows are written (sel_b/sel_j of length n_sel; n_sel = 0 selects all).
  * p_out (optional, float64, used with exactly one selected row) receives
- * the softmax weights.  Returns 0, or -1 on an out-of-range table entry.
+ * the softmax weights.  mu float32 [h_kv][128]; win / win_slot may be NULL
+ * when sink = recent = 0.  Returns 0, or -1 on an out-of-range table entry
+ * or window slot.
  */
-int oracle_decode_attention(const uint16_t* q, const int32_t* block_table,
-                            const int32_t* seq_lens, int B, int max_pages,
-                            const uint8_t* pool, int num_pages, int h_q,
-                            int h_kv, const float* R_k, const float* R_v,
-                            double* out, const int32_t* sel_b,
-                            const int32_t* sel_j, int n_sel, double* p_out) {
+int oracle_decode_attention_win(const uint16_t* q, const int32_t* block_table,
+                                const int32_t* seq_lens, int B, int max_pages,
+                                const uint8_t* pool, int num_pages, int h_q,
+                                int h_kv, const float* R_k, const float* R_v,
+                                const float* mu, const uint16_t* win,
+                                const int32_t* win_slot, int n_slots, int sink,
+                                int recent, double* out, const int32_t* sel_b,
+                                const int32_t* sel_j, int n_sel, double* p_out) {
   int n_rows = n_sel > 0 ? n_sel : B * h_q;
   int ratio = h_q / h_kv;
   int bad = 0;
+  const double scale = 1.0 / sqrt((double)OR_D);
 #pragma omp parallel for schedule(dynamic, 1) num_threads(g_threads) reduction(|: bad)
   for (int r = 0; r < n_rows; ++r) {
     int b = n_sel > 0 ? sel_b[r] : r / h_q;
@@ -324,30 +405,84 @@ int oracle_decode_attention(const uint16_t* q, const int32_t* block_table,
       continue;
     }
     if (n > max_pages * OR_P) { bad = 1; continue; }
-    double* khat = (double*)malloc(sizeof(double) * (size_t)n * OR_D);
-    double* vhat = (double*)malloc(sizeof(double) * (size_t)n * OR_D);
+    int slot = (sink > 0 || recent > 0) ? win_slot[b] : 0;
+    if ((sink > 0 || recent > 0) && (slot < 0 || slot >= n_slots)) {
+      bad = 1;
+      continue;
+    }
+    double qx[OR_D], qr[OR_D];
+    const uint16_t* qrow = q + ((size_t)b * h_q + j) * OR_D;
+    for (int i = 0; i < OR_D; ++i) qx[i] = bf16_to_f64(qrow[i]);
+    rotate(qx, R_k + (size_t)h * OR_D * OR_D, qr);
+    /* per token: logit, value, and whether the value is in the rotated basis */
+    double* l = (double*)malloc(sizeof(double) * (size_t)n);
+    double* val = (double*)malloc(sizeof(double) * (size_t)n * OR_D);
+    char* rot = (char*)malloc((size_t)n);
     int ok = 1;
     for (int s = 0; s < n && ok; ++s) {
-      int page = block_table[(size_t)b * max_pages + s / OR_P];
-      if (page < 0 || page >= num_pages) { ok = 0; break; }
-      const uint8_t* c = pool + ((size_t)page * h_kv + h) * OR_CHUNK;
-      load_slot(c, 0, s % OR_P, khat + (size_t)s * OR_D);
-      load_slot(c, 1, s % OR_P, vhat + (size_t)s * OR_D);
+      double* vs = val + (size_t)s * OR_D;
+      double acc = 0.0;
+      if (in_window(s, n, sink, recent)) {
+        int row = window_row(s, sink, recent);
+        const uint16_t* kw = window_vec(win, slot, h_kv, h, 0, row, sink, recent);
+        const uint16_t* vw = window_vec(win, slot, h_kv, h, 1, row, sink, recent);
+        for (int i = 0; i < OR_D; ++i)
+          acc += qx[i] * (bf16_to_f64(kw[i]) - (double)mu[h * OR_D + i]);
+        for (int i = 0; i < OR_D; ++i) vs[i] = bf16_to_f64(vw[i]);
+        rot[s] = 0;
+      } else {
+        int page = block_table[(size_t)b * max_pages + s / OR_P];
+        if (page < 0 || page >= num_pages) { ok = 0; break; }
+        const uint8_t* c = pool + ((size_t)page * h_kv + h) * OR_CHUNK;
+        double kh[OR_D];
+        load_slot(c, 0, s % OR_P, kh);
+        load_slot(c, 1, s % OR_P, vs);
+        for (int i = 0; i < OR_D; ++i) acc += qr[i] * kh[i];
+        rot[s] = 1;
+      }
+      l[s] = acc * scale;
     }
     if (ok) {
-      double x[OR_D], qr[OR_D], orot[OR_D];
-      const uint16_t* qrow = q + ((size_t)b * h_q + j) * OR_D;
-      for (int i = 0; i < OR_D; ++i) x[i] = bf16_to_f64(qrow[i]);
-      rotate(x, R_k + (size_t)h * OR_D * OR_D, qr);
-      attend(qr, khat, vhat, n, orot, (n_sel == 1) ? p_out : NULL);
-      rotate_back(orot, R_v + (size_t)h * OR_D * OR_D, o);
+      /* two-pass softmax, then the two value sums */
+      double mx = -INFINITY, z = 0.0;
+      for (int s = 0; s < n; ++s)
+        if (l[s] > mx) mx = l[s];
+      for (int s = 0; s < n; ++s) {
+        l[s] = exp(l[s] - mx);
+        z += l[s];
+      }
+      double orot[OR_D], owin[OR_D], oback[OR_D];
+      for (int i = 0; i < OR_D; ++i) orot[i] = owin[i] = 0.0;
+      for (int s = 0; s < n; ++s) {
+        double p = l[s] / z;
+        if (p_out && n_sel == 1) p_out[s] = p;
+        double* acc = rot[s] ? orot : owin;
+        for (int i = 0; i < OR_D; ++i) acc[i] += p * val[(size_t)s * OR_D + i];
+      }
+      rotate_back(orot, R_v + (size_t)h * OR_D * OR_D, oback);
+      for (int i = 0; i < OR_D; ++i) o[i] = oback[i] + owin[i];
     } else {
       bad = 1;
     }
-    free(khat);
-    free(vhat);
+    free(l);
+    free(val);
+    free(rot);
   }
   return bad ? -1 : 0;
+}
+
+/* The INT2 path alone (no windows): oracle_decode_attention_win with
+ * sink = recent = 0. */
+int oracle_decode_attention(const uint16_t* q, const int32_t* block_table,
+                            const int32_t* seq_lens, int B, int max_pages,
+                            const uint8_t* pool, int num_pages, int h_q,
+                            int h_kv, const float* R_k, const float* R_v,
+                            double* out, const int32_t* sel_b,
+                            const int32_t* sel_j, int n_sel, double* p_out) {
+  return oracle_decode_attention_win(q, block_table, seq_lens, B, max_pages,
+                                     pool, num_pages, h_q, h_kv, R_k, R_v,
+                                     NULL, NULL, NULL, 0, 0, 0, out, sel_b,
+                                     sel_j, n_sel, p_out);
 }
 
 /*
@@ -356,13 +491,18 @@ int oracle_decode_attention(const uint16_t* q, const int32_t* block_table,
  * Q2((k_s - mu) R_K) R_K^T, vbar_s = D_{R_V,c_V}(v_s) = Q2(v_s R_V) R_V^T,
  * then Eq. 1-2 with the plain query: a_s = <q, kbar_s>/sqrt(d),
  * p = softmax(a), out = sum_s p_s vbar_s.  With quantize = 0 the map Q2 is
- * the identity, so D_{R,c}(z) = z (Sec. 3.1).  q float64 [128]; K, V
- * float64 [n][128]; R_k, R_v float32 [128][128]; mu float64 [128].
+ * the identity, so D_{R,c}(z) = z (Sec. 3.1).  Window positions (s < sink or
+ * s >= n - recent; Sec. 3.1 and Sec. 4.1, BF16 sink and recent tokens with
+ * the same key centering) keep kbar_s = k_s - mu and vbar_s = v_s.
+ * q float64 [128]; K, V float64 [n][128]; R_k, R_v float32 [128][128];
+ * mu float64 [128].
  */
-int oracle_attention_dense(const double* q, const double* K, const double* V,
-                           int n, const float* R_k, const float* R_v,
-                           const double* mu, int quantize, float clip_k,
-                           float clip_v, double* out, double* p_out) {
+int oracle_attention_dense_win(const double* q, const double* K,
+                               const double* V, int n, const float* R_k,
+                               const float* R_v, const double* mu,
+                               int quantize, float clip_k, float clip_v,
+                               int sink, int recent, double* out,
+                               double* p_out) {
   if (n <= 0) {
     for (int i = 0; i < OR_D; ++i) out[i] = 0.0;
     return 0;
@@ -372,6 +512,13 @@ int oracle_attention_dense(const double* q, const double* K, const double* V,
   for (int s = 0; s < n; ++s) {
     double x[OR_D], z[OR_D], zq[OR_D];
     for (int i = 0; i < OR_D; ++i) x[i] = K[(size_t)s * OR_D + i] - mu[i];
+    if (in_window(s, n, sink, recent)) {
+      for (int i = 0; i < OR_D; ++i) {
+        kbar[(size_t)s * OR_D + i] = x[i];
+        vbar[(size_t)s * OR_D + i] = V[(size_t)s * OR_D + i];
+      }
+      continue;
+    }
     rotate(x, R_k, z);
     if (quantize) {
       uint8_t c[OR_D];
@@ -399,6 +546,15 @@ int oracle_attention_dense(const double* q, const double* K, const double* V,
   free(kbar);
   free(vbar);
   return 0;
+}
+
+/* The dense statement without windows. */
+int oracle_attention_dense(const double* q, const double* K, const double* V,
+                           int n, const float* R_k, const float* R_v,
+                           const double* mu, int quantize, float clip_k,
+                           float clip_v, double* out, double* p_out) {
+  return oracle_attention_dense_win(q, K, V, n, R_k, R_v, mu, quantize, clip_k,
+                                    clip_v, 0, 0, out, p_out);
 }
 
 /* Exported for tests: z = x R (fp64) and the group quantization of z, for

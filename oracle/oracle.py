@@ -65,6 +65,15 @@ def _declare(L):
     L.oracle_decode_attention.argtypes = [_P, _P, _P, i, i, _P, i, i, i, _P,
                                           _P, _P, _P, _P, i, _P]
     L.oracle_decode_attention.restype = i
+    L.oracle_decode_attention_win.argtypes = [_P, _P, _P, i, i, _P, i, i, i,
+                                              _P, _P, _P, _P, _P, i, i, i, _P,
+                                              _P, _P, i, _P]
+    L.oracle_decode_attention_win.restype = i
+    L.oracle_window_write.argtypes = [_P, _P, i, _P, _P, i, _P, i, i, i, i, _P]
+    L.oracle_window_write.restype = i
+    L.oracle_attention_dense_win.argtypes = [_P, _P, _P, i, _P, _P, _P, i, f,
+                                             f, i, i, _P, _P]
+    L.oracle_attention_dense_win.restype = i
     L.oracle_attention_dense.argtypes = [_P, _P, _P, i, _P, _P, _P, i, f, f,
                                          _P, _P]
     L.oracle_attention_dense.restype = i
@@ -153,9 +162,13 @@ def kv_append(k_bits, v_bits, cu_new, pos0, block_table, pool, R_k, R_v, mu,
 
 
 def decode_attention(q_bits, block_table, seq_lens, pool, R_k, R_v, h_kv,
-                     rows=None, want_p=False):
+                     rows=None, want_p=False, win=None, win_slot=None, sink=0,
+                     recent=0, mu=None):
     """Oracle decode.  Returns float64 [B][h_q][128]; when ``rows`` (a list of
-    (b, j)) is given only those rows are computed (others stay zero)."""
+    (b, j)) is given only those rows are computed (others stay zero).  With
+    ``sink`` / ``recent`` > 0 the BF16 window positions are read from ``win``
+    (uint16 bf16 bits [n_slots][h_kv][2][sink + recent][128]) at the slots
+    ``win_slot`` [B], and ``mu`` (float32 [h_kv][128]) centers their keys."""
     q_bits = _c(q_bits, np.uint16)
     bt = _c(block_table, np.int32)
     sl = _c(seq_lens, np.int32)
@@ -172,31 +185,66 @@ def decode_attention(q_bits, block_table, seq_lens, pool, R_k, R_v, h_kv,
     if want_p:
         assert n_sel == 1
         p = np.zeros(int(sl[rows[0][0]]), np.float64)
-    rc = lib().oracle_decode_attention(
+    windows = sink > 0 or recent > 0
+    if windows:
+        win = _c(win, np.uint16)
+        assert win.shape[1:] == (h_kv, 2, sink + recent, D)
+        win_slot = _c(win_slot, np.int32)
+        mu = _c(mu, np.float32)
+        n_slots = win.shape[0]
+    else:
+        win = win_slot = mu = None
+        n_slots = 0
+    rc = lib().oracle_decode_attention_win(
         _ptr(q_bits), _ptr(bt), _ptr(sl), B, bt.shape[1], _ptr(pool),
         pool.shape[0], h_q, h_kv, _ptr(_c(R_k, np.float32)),
-        _ptr(_c(R_v, np.float32)), _ptr(out), _ptr(sb), _ptr(sj), n_sel,
+        _ptr(_c(R_v, np.float32)), _ptr(mu), _ptr(win), _ptr(win_slot),
+        n_slots, int(sink), int(recent), _ptr(out), _ptr(sb), _ptr(sj), n_sel,
         _ptr(p))
     if rc != 0:
-        raise ValueError("oracle_decode_attention: table entry out of range")
+        raise ValueError("oracle_decode_attention: table entry or window slot out of range")
     return (out, p) if want_p else out
 
 
+def new_windows(n_slots, h_kv, sink, recent):
+    """Zeroed window store (bf16 bits) for n_slots sequences."""
+    return np.zeros((n_slots, h_kv, 2, sink + recent, D), np.uint16)
+
+
+def window_write(k_bits, v_bits, cu_new, pos0, win, win_slot, sink, recent):
+    """Window part of the oracle cache write; ``win`` is modified in place."""
+    k_bits = _c(k_bits, np.uint16)
+    v_bits = _c(v_bits, np.uint16)
+    cu_new = _c(cu_new, np.int32)
+    pos0 = _c(pos0, np.int32)
+    win_slot = _c(win_slot, np.int32)
+    assert win.dtype == np.uint16 and win.flags["C_CONTIGUOUS"]
+    n_tok, h_kv = k_bits.shape[0], k_bits.shape[1]
+    assert win.shape[1:] == (h_kv, 2, sink + recent, D)
+    rc = lib().oracle_window_write(
+        _ptr(k_bits), _ptr(v_bits), n_tok, _ptr(cu_new), _ptr(pos0), pos0.size,
+        _ptr(win_slot), win.shape[0], h_kv, int(sink), int(recent), _ptr(win))
+    if rc != 0:
+        raise ValueError("oracle_window_write: window slot out of range")
+
+
 def attention_dense(q, K, V, R_k, R_v, mu, quantize=True, clip_k=1.0,
-                    clip_v=1.0, want_p=False):
-    """Single-head dense statement in the inverse-rotation form."""
+                    clip_v=1.0, want_p=False, sink=0, recent=0):
+    """Single-head dense statement in the inverse-rotation form; positions
+    s < sink or s >= n - recent are BF16 window positions."""
     q = _c(q, np.float64)
     K = _c(K, np.float64)
     V = _c(V, np.float64)
     n = K.shape[0]
     out = np.zeros(D, np.float64)
     p = np.zeros(max(n, 1), np.float64) if want_p else None
-    lib().oracle_attention_dense(_ptr(q), _ptr(K), _ptr(V), n,
-                                 _ptr(_c(R_k, np.float32)),
-                                 _ptr(_c(R_v, np.float32)),
-                                 _ptr(_c(mu, np.float64)), int(bool(quantize)),
-                                 float(clip_k), float(clip_v), _ptr(out),
-                                 _ptr(p))
+    lib().oracle_attention_dense_win(_ptr(q), _ptr(K), _ptr(V), n,
+                                     _ptr(_c(R_k, np.float32)),
+                                     _ptr(_c(R_v, np.float32)),
+                                     _ptr(_c(mu, np.float64)),
+                                     int(bool(quantize)), float(clip_k),
+                                     float(clip_v), int(sink), int(recent),
+                                     _ptr(out), _ptr(p))
     return (out, p[:n]) if want_p else out
 
 
