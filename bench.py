@@ -157,6 +157,29 @@ def append_bytes(n_tok, h_kv):
     return n_tok * h_kv * (512 + 96)
 
 
+def window_split(n, sink, recent):
+    """(INT2 tokens, BF16 window tokens) of a sequence of n tokens: window
+    positions are s < sink and s >= n - recent."""
+    ns = min(n, sink)
+    r0 = max(sink, n - recent)
+    nw = ns + max(0, n - r0)
+    return n - nw, nw
+
+
+def decode_bytes_win(seq_lens, h_kv, h_q, sink, recent):
+    """Algorithmic bytes of one decode with BF16 windows: 96 B per INT2
+    token and KV head, 512 B (bf16 K and V rows) per window token and KV
+    head, bf16 query, fp32 output."""
+    i2 = wt = 0
+    for x in seq_lens:
+        a, b = window_split(int(x), sink, recent)
+        i2 += a
+        wt += b
+    B = len(seq_lens)
+    return (i2 * h_kv * 96 + wt * h_kv * 512 + B * h_q * D * 2 +
+            B * h_q * D * 4)
+
+
 # ------------------------------------------------------------------- ours
 
 class Flusher:
@@ -370,6 +393,9 @@ def extra_workloads(args, dev):
     del pool, k, v, case
     torch.cuda.empty_cache()
 
+    res["decode8k_windows"] = windows_step(args, dev, flush, hbm_peak)
+    torch.cuda.empty_cache()
+
     for name in ("long128k", "ragged"):
         wl, case, p, pool, bt = setup_decode(name, args.seed, dev, args.variant,
                                              args.append_variant)
@@ -404,6 +430,73 @@ def extra_workloads(args, dev):
         del pool, case
         torch.cuda.empty_cache()
     return res
+
+
+def windows_step(args, dev, flush, hbm_peak, sink=64, recent=256):
+    """The decode8k step with the paper's BF16 windows (64 sink, 256 recent
+    tokens; Sec. 5): optr_decode_step_win, L2 flushed before every step."""
+    from paper_2608_02691_gb300 import optr, synth
+    wl = synth.workload("decode8k", args.seed)
+    case = synth.build_case(wl, args.seed, device=dev)
+    p = optr.optr_params_create(case["R_k"], case["R_v"], case["mu"],
+                                case["h_q"], decode_variant=args.variant,
+                                append_variant=args.append_variant, sink=sink,
+                                recent=recent)
+    B, h_q, h_kv = case["B"], case["h_q"], case["h_kv"]
+    pool = optr.new_pool(p, case["num_pages"], device=dev)
+    win = optr.new_windows(p, B, device=dev)
+    slot = torch.arange(B, dtype=torch.int32, device=dev)
+    bt = case["block_table"].to(dev)
+    optr.optr_kv_append_win(p, case["k_ctx"], case["v_ctx"],
+                            case["cu_ctx"].to(dev), case["pos0_ctx"].to(dev),
+                            bt, pool, win, slot)
+    seq = case["seq_lens"].to(dev)
+    q = case["q"].to(dev)
+    k_new, v_new = case["k_new"].to(dev), case["v_new"].to(dev)
+    cu_new, pos0 = case["cu_new"].to(dev), case["pos0_new"].to(dev)
+    out = torch.empty(B, h_q, D, dtype=torch.float32, device=dev)
+    ws = optr.new_workspace(p, B, bt.shape[1], device=dev)
+    stream = torch.cuda.current_stream()
+
+    def step():
+        optr.optr_decode_step_win(p, q, k_new, v_new, cu_new, pos0, bt, seq,
+                                  pool, win, slot, out, ws)
+
+    for _ in range(3):
+        flush()
+        step()
+    torch.cuda.synchronize()
+    assert optr.optr_device_error(p) == 0
+    n = max(5, args.steps // 2)
+    evs = [(torch.cuda.Event(enable_timing=True),
+            torch.cuda.Event(enable_timing=True)) for _ in range(n)]
+    for i in range(n):
+        flush()
+        evs[i][0].record(stream)
+        step()
+        evs[i][1].record(stream)
+    torch.cuda.synchronize()
+    ms = float(np.mean([a.elapsed_time(b) for a, b in evs]))
+    optr.optr_profile_enable(p, True)
+    part = []
+    for _ in range(n):
+        flush()
+        step()
+        part.append(optr.optr_profile_last(p)["partial"])
+    optr.optr_profile_enable(p, False)
+    lens = case["seq_lens"].tolist()
+    n_new = k_new.shape[0]
+    nb = (decode_bytes_win(lens, h_kv, h_q, sink, recent) +
+          append_bytes(n_new, h_kv) + n_new * h_kv * 512)  # + window copies
+    i2 = sum(window_split(x, sink, recent)[0] for x in lens)
+    wt = sum(window_split(x, sink, recent)[1] for x in lens)
+    pb = i2 * h_kv * 96 + wt * h_kv * 512  # what the partial kernel streams
+    pm = float(np.mean(part))
+    return {"sink": sink, "recent": recent, "step_ms": round(ms, 4),
+            "bytes_per_step": nb, "gbs": round(nb / (ms * 1e-3) / 1e9, 1),
+            "partial_ms": round(pm, 4),
+            "partial_gbs": round(pb / (pm * 1e-3) / 1e9, 1),
+            "partial_frac": round(pb / (pm * 1e-3) / 1e9 / hbm_peak, 4)}
 
 
 # ---------------------------------------------------------- CPU baseline

@@ -135,6 +135,7 @@ typedef enum {
 #define OPTR_DEVERR_CU_NEW 8u    /* cu_new not non-decreasing within n_tok  */
 #define OPTR_DEVERR_FP16_RANGE 16u /* tensor-core append: |k| or |v| >= 65504 */
 #define OPTR_DEVERR_TIMEOUT 32u  /* internal: a kernel's bounded wait gave up */
+#define OPTR_DEVERR_WIN_SLOT 64u /* window slot of a sequence < 0 or >= n_slots */
 
 /* Kernel variants (for measurement; 0 picks the library default). */
 #define OPTR_VARIANT_DEFAULT 0
@@ -153,6 +154,10 @@ typedef struct {
   float clip_v;       /* value clip ratio c_V in (0, 1]; 1 = min-max        */
   int append_variant; /* OPTR_VARIANT_*                                    */
   int decode_variant; /* OPTR_VARIANT_*                                    */
+  int sink;           /* BF16 sink window: positions 0 .. sink-1; a multiple
+                         of 16 in [0, 1024]; 0 = none (see BF16 windows)    */
+  int recent;         /* BF16 recent window: the last `recent` positions;
+                         [0, 1024]; 0 = none                               */
 } optr_config;
 
 /*
@@ -310,6 +315,68 @@ optr_status optr_decode_attention_noalloc(const optr_params* p, const void* q,
                                           cudaStream_t stream);
 
 /* Static description of a status code. */
+/*
+ * BF16 windows (Sec. 3.1, opening paragraph: the long history is INT2 while
+ * a small BF16 window is kept; Sec. 4.1: sink and recent tokens stay in
+ * BF16 and their keys receive the same centering by mu; Sec. 5,
+ * "Implementation Details": 64 sink and 256 recent tokens).  With
+ * cfg.sink or cfg.recent > 0, a position s of a sequence holding n tokens
+ * is a window position when s < sink or s >= n - recent.  The decode then
+ * attends to it with its exact bf16 key and value:
+ *      l_s = <q_j, k_s - mu[h]> / sqrt(D),   value v_s (not rotated),
+ * and to every other position with its rotated INT2 record as above:
+ *      out_j = (sum_INT2 p_s vhat_R,s) R_v[h]^T + sum_window p_s v_s.
+ * Every token is still written to the INT2 pool (a token leaving the recent
+ * window needs no re-quantization); window positions are not read from it.
+ *
+ * Window store (caller-owned, optr_window_bytes(p, n_slots) bytes, 16-byte
+ * aligned): bf16 [n_slots][h_kv][2][sink + recent][D], plane 0 keys (as
+ * given, not centered), plane 1 values (as given: with R_v = NULL that is
+ * the folded basis).  Sequence b owns slot win_slot[b] (device int32 [B]);
+ * position s lives in row s when s < sink, else in row
+ * sink + (s - sink) % recent (a ring).  The cache write copies, for each
+ * sequence, the positions s < sink and the positions s >= end - recent,
+ * end = pos0[b] + its new-token count (those in the recent window once
+ * the write is cached); ring rows of older positions are overwritten, so
+ * a sequence's positions must be written in order.  A slot outside
+ * [0, n_slots) skips the sequence's window work and sets
+ * OPTR_DEVERR_WIN_SLOT.
+ *
+ * The entry points without _win require sink = recent = 0 and return
+ * OPTR_ERR_INVALID_ARG otherwise; the _win entry points take the same
+ * arguments plus the store (win, win_slot, n_slots), and with
+ * sink = recent = 0 behave exactly as the plain ones (the store arguments
+ * may then be NULL / 0).
+ */
+size_t optr_window_bytes(const optr_params* p, int n_slots);
+
+optr_status optr_kv_append_win(const optr_params* p, const void* k,
+                               const void* v, int n_tok, const int32_t* cu_new,
+                               const int32_t* pos0, const int32_t* block_table,
+                               int B, int max_pages, uint8_t* pool,
+                               int num_pages, void* win,
+                               const int32_t* win_slot, int n_slots,
+                               cudaStream_t stream);
+
+optr_status optr_decode_attention_win(const optr_params* p, const void* q,
+                                      const int32_t* block_table,
+                                      const int32_t* seq_lens, int B,
+                                      int max_pages, const uint8_t* pool,
+                                      int num_pages, const void* win,
+                                      const int32_t* win_slot, int n_slots,
+                                      float* out, void* workspace,
+                                      size_t ws_bytes, cudaStream_t stream);
+
+optr_status optr_decode_step_win(const optr_params* p, const void* q,
+                                 const void* k, const void* v, int n_tok,
+                                 const int32_t* cu_new, const int32_t* pos0,
+                                 const int32_t* block_table,
+                                 const int32_t* seq_lens, int B, int max_pages,
+                                 uint8_t* pool, int num_pages, void* win,
+                                 const int32_t* win_slot, int n_slots,
+                                 float* out, void* workspace, size_t ws_bytes,
+                                 cudaStream_t stream);
+
 const char* optr_strerror(optr_status s);
 
 #ifdef __cplusplus

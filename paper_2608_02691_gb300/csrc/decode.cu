@@ -15,6 +15,7 @@
 // softmax weights are exp2(l - m) (Sec. 3 Eq. 1 with the 1/sqrt(d) scale).
 #include "decode_common.cuh"
 #include "append_small.cuh"
+#include "window.cuh"
 
 namespace optr {
 namespace {
@@ -44,7 +45,8 @@ __device__ __forceinline__ void qrot_body(
     const int32_t* __restrict__ seq_lens, int max_pages,
     float* __restrict__ qf, float* __restrict__ qs, uint32_t* __restrict__ frag,
     float* __restrict__ koff, float* __restrict__ invs, int* __restrict__ pref,
-    int* __restrict__ nzpref, int* __restrict__ cnt_ws, unsigned* err) {
+    int* __restrict__ nzpref, int* __restrict__ cnt_ws, unsigned* err,
+    int sink, int recent) {
   float (&qsm)[4][kD] = sm.qsm;
   float (&part)[4][4][kD] = sm.part;
   float (&qrs)[4][kD] = sm.qrs;
@@ -160,8 +162,9 @@ __device__ __forceinline__ void qrot_body(
   if (tid == 0) cnt_ws[(size_t)b * h_kv + h] = 0;  // combine arrivals
 
   if (b != 0 || h != 0) return;
-  // Split-K plan: pref[b] = pages of sequences < b, nzpref[b] = non-empty
-  // sequences < b.  Invalid lengths count as empty and are flagged.
+  // Split-K plan: pref[b] = INT2 pages of sequences < b, nzpref[b] =
+  // sequences < b with INT2 pages.  Invalid lengths count as empty and are
+  // flagged.
   int run_p = 0, run_n = 0;
   constexpr int kW = kQrotThreads / 32;
   for (int base = 0; base < B; base += kQrotThreads) {
@@ -172,7 +175,7 @@ __device__ __forceinline__ void qrot_body(
       if (len < 0 || (long long)len > (long long)max_pages * kPage)
         atomicOr(err, OPTR_DEVERR_SEQ_LEN);
       else
-        np = (len + kPage - 1) / kPage;
+        np = int2_pages(len, sink, recent);
     }
     int xp = np, xn = np > 0;
 #pragma unroll
@@ -200,19 +203,22 @@ qrot_kernel(const __nv_bfloat16* __restrict__ q, const float* __restrict__ R_k,
             uint32_t* __restrict__ frag, float* __restrict__ koff,
             float* __restrict__ invs, int* __restrict__ pref,
             int* __restrict__ nzpref, int* __restrict__ cnt_ws,
-            unsigned* err) {
+            unsigned* err, int sink, int recent) {
   __shared__ QrotSmem sm;
   qrot_body(blockIdx.x, blockIdx.y, sm, q, R_k, B, h_q, h_kv, qscale, seq_lens,
-            max_pages, qf, qs, frag, koff, invs, pref, nzpref, cnt_ws, err);
+            max_pages, qf, qs, frag, koff, invs, pref, nzpref, cnt_ws, err,
+            sink, recent);
 }
 
 // ------------------------------------------------- decode-step prologue
-// One launch for the two independent first steps of a decode step: the
+// One launch for the independent first steps of a decode step: the
 // single-token cache write of every sequence (CTAs [0, n_app), as
-// append_small_kernel) and the query rotation (the following B * h_kv CTAs,
-// as qrot_kernel).  Both wait for the previous kernel before touching
-// inputs; the partial kernel then waits for this grid, i.e. for both.
-static_assert(kQrotThreads == 512, "one block size for both bodies");
+// append_small_kernel), the window copy of the new tokens (the next n_wcp
+// CTAs, BF16 windows only) and the query rotation (the following B * h_kv
+// CTAs, as qrot_kernel).  All wait for the previous kernel before touching
+// inputs; the partial kernel then waits for this grid, i.e. for all.
+static_assert(kQrotThreads == 512, "one block size for every body");
+static_assert(sizeof(float) * kPage * 4 >= (size_t)kWinPBytes, "window P scratch");
 
 template <int T>
 __global__ void __launch_bounds__(512)
@@ -227,7 +233,9 @@ step_prologue_kernel(
     const int32_t* __restrict__ seq_lens, int max_pages,
     float* __restrict__ qf, float* __restrict__ qs, uint32_t* __restrict__ frag,
     float* __restrict__ koff, float* __restrict__ invs, int* __restrict__ pref,
-    int* __restrict__ nzpref, int* __restrict__ cnt_ws, unsigned* err, int fold_v) {
+    int* __restrict__ nzpref, int* __restrict__ cnt_ws, unsigned* err, int fold_v,
+    int n_wcp, __nv_bfloat16* __restrict__ win,
+    const int32_t* __restrict__ win_slot, int n_slots, int sink, int recent) {
   extern __shared__ __align__(16) unsigned char dsm_[];
   const int bid = blockIdx.x;
   if (bid < n_app) {
@@ -237,23 +245,45 @@ step_prologue_kernel(
                       k, v, n_tok, cu_new, pos0, bt, B, max_pages, pool,
                       num_pages, h_kv, R_k, R_v, muR, clip_k, clip_v, err,
                       fold_v && kind == 1);
+  } else if (bid < n_app + n_wcp) {
+    window_copy_body(bid - n_app, *reinterpret_cast<WinCopySmem*>(dsm_), k, v,
+                     n_tok, cu_new, pos0, B, win, win_slot, n_slots, h_kv,
+                     sink, recent, err);
   } else {
-    const int r = bid - n_app;
+    const int r = bid - n_app - n_wcp;
     qrot_body(r / h_kv, r % h_kv, *reinterpret_cast<QrotSmem*>(dsm_), q, R_k, B,
               h_q, h_kv, qscale, seq_lens, max_pages, qf, qs, frag, koff, invs,
-              pref, nzpref, cnt_ws, err);
+              pref, nzpref, cnt_ws, err, sink, recent);
   }
+}
+
+// Window part of a separate cache write (512 threads per 16 new tokens).
+__global__ void __launch_bounds__(512)
+window_copy_kernel(const __nv_bfloat16* __restrict__ k,
+                   const __nv_bfloat16* __restrict__ v, int n_tok,
+                   const int32_t* __restrict__ cu_new,
+                   const int32_t* __restrict__ pos0, int B,
+                   __nv_bfloat16* __restrict__ win,
+                   const int32_t* __restrict__ win_slot, int n_slots, int h_kv,
+                   int sink, int recent, unsigned* err) {
+  __shared__ WinCopySmem sm;
+  window_copy_body(blockIdx.x, sm, k, v, n_tok, cu_new, pos0, B, win, win_slot,
+                   n_slots, h_kv, sink, recent, err);
 }
 
 // ------------------------------------------------- CUDA-core partial kernel
 
 struct WarpSmemCC {
-  alignas(16) uint8_t stage[2][kChunk];
+  union {  // the window phase runs before the first page is staged
+    alignas(16) uint8_t stage[2][kChunk];
+    alignas(16) uint8_t wst[kWinStageBytes];
+  };
   float qv[4][kD];
   float qsum[4][kGroups];
   float p[kPage][4];
 };
 
+template <bool WIN>  // WIN: with the BF16-window phase
 __global__ void __launch_bounds__(128)
 partial_cuda_core_kernel(const uint8_t* __restrict__ pool,
                          const int32_t* __restrict__ bt,
@@ -263,13 +293,21 @@ partial_cuda_core_kernel(const uint8_t* __restrict__ pool,
                          const float* __restrict__ qs,
                          const int* __restrict__ pref,
                          const int* __restrict__ nzpref,
-                         float* __restrict__ part, int W, unsigned* err) {
+                         float* __restrict__ part, int W, unsigned* err,
+                         int sink, int recent, WinPhase wp) {
   __shared__ WarpSmemCC smem[4];
-  pdl_wait();
-  pdl_trigger();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   WarpSmemCC& S = smem[warp];
   const int w = blockIdx.x * 4 + warp;
+  // BF16 windows first, before waiting for the previous kernel (the phase
+  // reads only inputs and library-owned state); stage and p are free until
+  // the first segment
+  if constexpr (WIN) {
+    if (w < wp.Ww) window_phase(w, wp, S.wst, reinterpret_cast<uint8_t*>(&S.p[0][0]));
+  }
+  pdl_wait();
+  pdl_trigger();
+  const int poff = sink / kPage;  // first INT2 page
   const long long F = (long long)__ldcg(pref + B) * h_kv;
   long long f = w * F / W;
   const long long f1 = (w + 1) * F / W;
@@ -277,7 +315,7 @@ partial_cuda_core_kernel(const uint8_t* __restrict__ pool,
   while (f < f1) {
     Segment sg = locate_segment(f, f1, pref, B, h_kv);
     const int b = sg.b, h = sg.h;
-    const int len = __ldg(seq_lens + b);
+    const int len = int2_end(__ldg(seq_lens + b), sink, recent);  // INT2 end
     // rotated queries of the GQA group
     for (int i = lane; i < 4 * kD; i += 32)
       S.qv[i / kD][i % kD] = __ldcg(qf + ((size_t)b * h_q + 4 * h) * kD + i);
@@ -293,19 +331,19 @@ partial_cuda_core_kernel(const uint8_t* __restrict__ pool,
     }
     const int32_t* btb = bt + (size_t)b * max_pages;
     // 2-stage cp.async pipeline over the segment's pages
-    bool ok0 = issue_page(S.stage[0], pool, btb, sg.p0, num_pages, h_kv, h, lane, err);
+    bool ok0 = issue_page(S.stage[0], pool, btb, poff + sg.p0, num_pages, h_kv, h, lane, err);
     bool okn = false;
     for (int i = 0; i < sg.n; ++i) {
       const bool ok = (i == 0) ? ok0 : okn;
       if (i + 1 < sg.n)
-        okn = issue_page(S.stage[(i + 1) & 1], pool, btb, sg.p0 + i + 1,
+        okn = issue_page(S.stage[(i + 1) & 1], pool, btb, poff + sg.p0 + i + 1,
                          num_pages, h_kv, h, lane, err);
       else
         cp_async_commit();
       cp_async_wait_1();
       __syncwarp();
       const uint8_t* st = S.stage[i & 1];
-      const int page = sg.p0 + i;
+      const int page = poff + sg.p0 + i;
       int nvalid = ok ? min(kPage, len - page * kPage) : 0;
       __syncwarp();
 
@@ -512,11 +550,16 @@ __global__ void __launch_bounds__(kCombineThreads)
 combine_kernel(const float* __restrict__ part, const int* __restrict__ pref,
                const int* __restrict__ nzpref, int B, int h_q, int h_kv, int W,
                const float* __restrict__ R_vT, float* __restrict__ cpart,
-               int* __restrict__ cnt_ws, float* __restrict__ out, int fold_v) {
+               int* __restrict__ cnt_ws, float* __restrict__ out, int fold_v,
+               const float* __restrict__ wpart,
+               const int32_t* __restrict__ seq_lens, int max_pages, int sink,
+               int recent, int Uw, int Ww) {
   extern __shared__ float4 dsm[];
   float* rts = reinterpret_cast<float*>(dsm);  // [128][128] R_v^T[h]
   __shared__ float4 msum[4][kD];               // [phase][float4 of o']
+  __shared__ float4 msumw[4][kD];              // the same for the windows
   __shared__ float orot[4][kD];
+  __shared__ float ow[4][kD];                  // window output (unrotated)
   __shared__ CombineState st;
   __shared__ int last;
   const int b = blockIdx.x, h = blockIdx.y, sp = blockIdx.z, S = gridDim.z;
@@ -548,10 +591,24 @@ combine_kernel(const float* __restrict__ part, const int* __restrict__ pref,
   const bool sparse = F < W;
   const float* pbase = part + ((size_t)nzb * h_kv + h + w0) * kPartFloats;
   const int i0 = sp * n / S, i1 = (sp + 1) * n / S;  // n <= W: no overflow
+  // BF16-window partials of (b, h): the window warps that own its units
+  // 0 .. nwu - 1 (window.cuh), one slot each, no gaps
+  int ww0 = 0, wn = 0;
+  if (Ww > 0) {
+    int len = __ldg(seq_lens + b);
+    if (len < 0 || (long long)len > (long long)max_pages * kPage) len = 0;
+    const int nwu = (win_count(len, sink, recent) + kWinUnit - 1) / kWinUnit;
+    if (nwu > 0) {
+      const long long U = (long long)B * h_kv * Uw;
+      const long long u0 = ((long long)b * h_kv + h) * Uw;
+      ww0 = warp_of(u0, U, Ww);
+      wn = warp_of(u0 + nwu - 1, U, Ww) - ww0 + 1;
+    }
+  }
   pdl_wait();
   pdl_trigger();
   float* ob = out + ((size_t)b * h_q + 4 * h) * kD;
-  if (np == 0) {
+  if (np == 0 && (wn == 0 || sp != 0)) {  // nothing, or windows only (CTA 0)
     if (sp == 0) ob[tid] = 0.f;
     cp_async_wait<0>();
     return;
@@ -562,9 +619,9 @@ combine_kernel(const float* __restrict__ part, const int* __restrict__ pref,
     combine_batch(pbase + (size_t)i * kPartFloats, min(kCombineBatch, i1 - i),
                   w0 + i, sparse, F, W, st, acc);
   const int v = tid & 127, ph = tid >> 7;
-  msum[ph][v] = acc;
-  __syncthreads();
-  if (S > 1) {
+  if (S > 1 && np > 0) {
+    msum[ph][v] = acc;
+    __syncthreads();
     // publish this chunk: o'[4][128], M[4], L[4] in the partial format
     const size_t seg = (size_t)b * h_kv + h;
     float* cp = cpart + (seg * S + sp) * kPartFloats;
@@ -596,9 +653,23 @@ combine_kernel(const float* __restrict__ part, const int* __restrict__ pref,
     for (int i = 0; i < S; i += kCombineBatch)
       combine_batch(cpart + (seg * S + i) * kPartFloats, min(kCombineBatch, S - i),
                     -1, false, F, W, st, acc);
-    msum[ph][v] = acc;
-    __syncthreads();
   }
+  // The final CTA of (b, h) merges the window partials into a second
+  // accumulator under the same running maxima; each batch's rescale of the
+  // maxima applies to the INT2 accumulator as well.
+  float4 accw = make_float4(0.f, 0.f, 0.f, 0.f);
+  for (int i = 0; i < wn; i += kCombineBatch) {
+    combine_batch(wpart + (size_t)(ww0 + b * h_kv + h + i) * kPartFloats,
+                  min(kCombineBatch, wn - i), -1, false, 0, 1, st, accw);
+    const float al = st.alpha[v >> 5];
+    acc.x *= al;
+    acc.y *= al;
+    acc.z *= al;
+    acc.w *= al;
+  }
+  msum[ph][v] = acc;
+  msumw[ph][v] = accw;
+  __syncthreads();
   if (tid < kD) {
     const float4 a = msum[0][tid], b1 = msum[1][tid], c = msum[2][tid], d = msum[3][tid];
     const int hd = tid >> 5, ch = (tid & 31) * 4;
@@ -608,11 +679,16 @@ combine_kernel(const float* __restrict__ part, const int* __restrict__ pref,
     orot[hd][ch + 1] = ((a.y + b1.y) + (c.y + d.y)) * il;
     orot[hd][ch + 2] = ((a.z + b1.z) + (c.z + d.z)) * il;
     orot[hd][ch + 3] = ((a.w + b1.w) + (c.w + d.w)) * il;
+    const float4 e = msumw[0][tid], f = msumw[1][tid], g = msumw[2][tid], k = msumw[3][tid];
+    ow[hd][ch + 0] = ((e.x + f.x) + (g.x + k.x)) * il;
+    ow[hd][ch + 1] = ((e.y + f.y) + (g.y + k.y)) * il;
+    ow[hd][ch + 2] = ((e.z + f.z) + (g.z + k.z)) * il;
+    ow[hd][ch + 3] = ((e.w + f.w) + (g.w + k.w)) * il;
   }
   cp_async_wait<0>();
   __syncthreads();
   if (fold_v) {  // output in the folded value basis: no R_v^T
-    ob[tid] = orot[tid >> 7][tid & 127];
+    ob[tid] = orot[tid >> 7][tid & 127] + ow[tid >> 7][tid & 127];
     return;
   }
   // out[r][i] = sum_k o'[r][k] R_v[i][k] = sum_k o'[r][k] R_vT[k][i]:
@@ -632,8 +708,9 @@ combine_kernel(const float* __restrict__ part, const int* __restrict__ pref,
     for (int r = 0; r < 4; ++r) qs4[(q * 4 + r) * kD + i] = acc4[r];
     __syncthreads();
     const int r = tid >> 7;
-    ob[r * kD + i] = (qs4[(0 * 4 + r) * kD + i] + qs4[(1 * 4 + r) * kD + i]) +
-                     (qs4[(2 * 4 + r) * kD + i] + qs4[(3 * 4 + r) * kD + i]);
+    ob[r * kD + i] = ((qs4[(0 * 4 + r) * kD + i] + qs4[(1 * 4 + r) * kD + i]) +
+                      (qs4[(2 * 4 + r) * kD + i] + qs4[(3 * 4 + r) * kD + i])) +
+                     ow[r][i];
   }
 }
 
@@ -646,14 +723,24 @@ cudaError_t launch_partial_tensor(const optr_params* p, const uint8_t* pool,
                                   const float* invs, const float* qs,
                                   const int* pref, const int* nzpref,
                                   float* part, int W, bool early_pages,
-                                  cudaStream_t s);
+                                  const WinPhase& wp, cudaStream_t s);
+
+cudaError_t launch_window_copy(const optr_params* p, const __nv_bfloat16* k,
+                               const __nv_bfloat16* v, int n_tok,
+                               const int32_t* cu_new, const int32_t* pos0,
+                               int B, const WinArgs& win, cudaStream_t s) {
+  const int tiles = (n_tok + kWinCopyTok - 1) / kWinCopyTok;
+  return launch_pdl(window_copy_kernel, dim3(tiles), dim3(512), 0, s, k, v,
+                    n_tok, cu_new, pos0, B, win.win, win.slot, win.n_slots,
+                    p->cfg.h_kv, p->cfg.sink, p->cfg.recent, p->err);
+}
 
 cudaError_t launch_decode(const optr_params* p, int variant,
                           const __nv_bfloat16* q, const int32_t* bt,
                           const int32_t* seq_lens, int B, int max_pages,
                           const uint8_t* pool, int num_pages, float* out,
                           void* ws, const DecodePlan& plan, cudaStream_t s,
-                          const StepAppend* app) {
+                          const StepAppend* app, const WinArgs* win) {
   char* w = static_cast<char*>(ws);
   float* qf = reinterpret_cast<float*>(w + plan.off_qf);
   float* qs = reinterpret_cast<float*>(w + plan.off_qs);
@@ -664,30 +751,66 @@ cudaError_t launch_decode(const optr_params* p, int variant,
   int* nzpref = pref + (B + 1);
   float* part = reinterpret_cast<float*>(w + plan.off_part);
   const int h_q = p->cfg.h_q, h_kv = p->cfg.h_kv;
+  const int sink = p->cfg.sink, recent = p->cfg.recent;
   const float qscale = kLog2e / sqrtf((float)kD);
+  // BF16 windows: the window partials, computed by the partial kernel
+  const bool windows = plan.Ww > 0;
+  WinPhase wp{};
+  wp.Ww = 0;
+  if (windows) {
+    wp.q = q;
+    wp.win = win->win;
+    wp.slot = win->slot;
+    wp.seq_lens = seq_lens;
+    wp.mu = p->mu;
+    wp.wpart = reinterpret_cast<float*>(w + plan.off_wpart);
+    if (app) {  // the step's new rows, read directly (see WinPhase)
+      wp.k_new = app->k;
+      wp.v_new = app->v;
+      wp.cu_new = app->cu_new;
+      wp.pos0 = app->pos0;
+    }
+    wp.err = p->err;
+    wp.n_slots = win->n_slots;
+    wp.B = B;
+    wp.h_q = h_q;
+    wp.h_kv = h_kv;
+    wp.max_pages = max_pages;
+    wp.sink = sink;
+    wp.recent = recent;
+    wp.Uw = plan.Uw;
+    wp.Ww = plan.Ww;
+    wp.qscale = qscale;
+  }
 
   int* cnt_ws = reinterpret_cast<int*>(w + plan.off_cnt);
   cudaError_t e;
   if (app) {
-    // the cache write of the step and the query rotation in one launch
+    // the cache write of the step (INT2 records and window copies) and the
+    // query rotation in one launch
     prof_mark(p, 0, s);
     const int T = small_tile(app->n_tok);
     const int tiles = (app->n_tok + T - 1) / T;
     const int n_app = tiles * h_kv * 2;
+    const int n_wcp = windows ? (app->n_tok + kWinCopyTok - 1) / kWinCopyTok : 0;
     const size_t sm_app = T == kSmallTokFew ? sizeof(AppendSmallSmemT<kSmallTokFew>)
                                             : sizeof(AppendSmallSmemT<kSmallTok>);
-    const size_t sm_bytes = sm_app > sizeof(QrotSmem) ? sm_app : sizeof(QrotSmem);
+    size_t sm_bytes = sm_app > sizeof(QrotSmem) ? sm_app : sizeof(QrotSmem);
+    if (sm_bytes < sizeof(WinCopySmem)) sm_bytes = sizeof(WinCopySmem);
     auto fn = T == kSmallTokFew ? step_prologue_kernel<kSmallTokFew>
                                 : step_prologue_kernel<kSmallTok>;
     e = ensure_dynamic_smem(reinterpret_cast<const void*>(fn), sm_bytes);
     if (e != cudaSuccess) return e;
-    e = launch_pdl(fn, dim3(n_app + B * h_kv), dim3(512),
+    e = launch_pdl(fn, dim3(n_app + n_wcp + B * h_kv), dim3(512),
                    sm_bytes, s, n_app, tiles, app->k, app->v, app->n_tok,
                    app->cu_new, app->pos0, bt, app->pool, num_pages,
                    (const float*)p->R_v, (const float*)p->muR, p->cfg.clip_k,
                    p->cfg.clip_v, q, (const float*)p->R_k, B, h_q, h_kv, qscale,
                    seq_lens, max_pages, qf, qs, frag, koff, invs, pref, nzpref,
-                   cnt_ws, p->err, p->fold_v);
+                   cnt_ws, p->err, p->fold_v, n_wcp,
+                   windows ? win->win : (__nv_bfloat16*)nullptr,
+                   windows ? win->slot : (const int32_t*)nullptr,
+                   windows ? win->n_slots : 0, sink, recent);
     if (e != cudaSuccess) return e;
     prof_mark(p, 1, s);  // the append stage covers the fused launch,
     prof_mark(p, 2, s);  // the query-rotation stage is empty
@@ -695,7 +818,8 @@ cudaError_t launch_decode(const optr_params* p, int variant,
     prof_mark(p, 2, s);
     e = launch_pdl(qrot_kernel, dim3(B, h_kv), dim3(kQrotThreads), 0, s, q,
                    p->R_k, B, h_q, h_kv, qscale, seq_lens, max_pages, qf, qs,
-                   frag, koff, invs, pref, nzpref, cnt_ws, p->err);
+                   frag, koff, invs, pref, nzpref, cnt_ws, p->err, sink,
+                   recent);
     if (e != cudaSuccess) return e;
   }
   prof_mark(p, 3, s);
@@ -705,11 +829,12 @@ cudaError_t launch_decode(const optr_params* p, int variant,
     // fused prologue it must wait first
     e = launch_partial_tensor(p, pool, bt, seq_lens, B, max_pages, num_pages,
                               frag, koff, invs, qs, pref, nzpref, part, plan.W,
-                              app == nullptr, s);
+                              app == nullptr, wp, s);
   } else {
-    e = launch_pdl(partial_cuda_core_kernel, dim3(plan.W / 4), dim3(128), 0, s,
+    e = launch_pdl(windows ? partial_cuda_core_kernel<true> : partial_cuda_core_kernel<false>,
+                   dim3(plan.W / 4), dim3(128), 0, s,
                    pool, bt, seq_lens, B, max_pages, num_pages, h_q, h_kv, qf,
-                   qs, pref, nzpref, part, plan.W, p->err);
+                   qs, pref, nzpref, part, plan.W, p->err, sink, recent, wp);
   }
   if (e != cudaSuccess) return e;
   prof_mark(p, 4, s);
@@ -721,7 +846,9 @@ cudaError_t launch_decode(const optr_params* p, int variant,
                  cmb_bytes, s, (const float*)part, (const int*)pref,
                  (const int*)nzpref, B, h_q, h_kv, plan.W, (const float*)p->R_vT,
                  reinterpret_cast<float*>(w + plan.off_cpart),
-                 reinterpret_cast<int*>(w + plan.off_cnt), out, p->fold_v);
+                 reinterpret_cast<int*>(w + plan.off_cnt), out, p->fold_v,
+                 (const float*)wp.wpart, seq_lens, max_pages, sink, recent,
+                 plan.Uw, plan.Ww);
   if (e != cudaSuccess) return e;
   prof_mark(p, 5, s);
   return cudaSuccess;

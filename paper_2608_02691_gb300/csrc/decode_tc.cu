@@ -36,6 +36,7 @@
 #include <type_traits>
 
 #include "decode_common.cuh"
+#include "window.cuh"
 
 namespace optr {
 namespace {
@@ -54,6 +55,13 @@ struct WarpSmemTC {
   uint4 qfr[kGroups][32];
   float4 kq[kGroups][32];
 };
+
+// the window phase stages 16 key and 16 value rows (8 KB) in the page
+// stages and pt, and its P tile in qfr, before any of them is used
+static_assert(offsetof(WarpSmemTC, pt) + sizeof(WarpSmemTC::pt) -
+                      offsetof(WarpSmemTC, stage) >= (size_t)kWinStageBytes,
+              "window row scratch");
+static_assert(sizeof(WarpSmemTC::qfr) >= (size_t)kWinPBytes, "window P scratch");
 
 constexpr int kPrefCache = 256;  // sequences whose page prefix sums a CTA caches
 
@@ -155,7 +163,7 @@ __device__ __forceinline__ void load_chunk(PageChunk& ch, int base, int f1,
                                            const int32_t* __restrict__ bt,
                                            int B, int h_kv, int max_pages,
                                            int num_pages, unsigned* err,
-                                           int lane) {
+                                           int lane, int sink, int recent) {
   ch.base = base;
   ch.unit = -1;
   ch.key = -1;
@@ -172,12 +180,12 @@ __device__ __forceinline__ void load_chunk(PageChunk& ch, int base, int f1,
     const int np = (cached ? spref[lo + 1] : __ldcg(pref + lo + 1)) - p0;
     const int r = f - p0 * h_kv;
     const int h = r / np;
-    const int page = r - h * np;
+    const int page = sink / kPage + (r - h * np);  // logical page (INT2 range)
     const int phys = __ldg(bt + (size_t)lo * max_pages + page);
     ch.key = lo * h_kv + h;
     if (phys >= 0 && phys < num_pages) {
       ch.unit = phys * h_kv + h;
-      ch.nvalid = min(kPage, __ldg(seq_lens + lo) - page * kPage);
+      ch.nvalid = min(kPage, int2_end(__ldg(seq_lens + lo), sink, recent) - page * kPage);
     } else {
       atomicOr(err, OPTR_DEVERR_PAGE_ID);  // skipped: its tokens count as masked
     }
@@ -188,12 +196,13 @@ __device__ __forceinline__ void load_chunk(PageChunk& ch, int base, int f1,
 // count as empty), by one block-wide scan; ends with __syncthreads().
 __device__ __noinline__ void page_prefix(const int32_t* __restrict__ seq_lens,
                                          int B, int max_pages, int* spref,
-                                         int* wsum) {
+                                         int* wsum, int sink, int recent) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   int np = 0;
   if ((int)threadIdx.x < B) {
     const int len = __ldg(seq_lens + threadIdx.x);
-    if (len >= 0 && (long long)len <= (long long)max_pages * kPage) np = (len + kPage - 1) / kPage;
+    if (len >= 0 && (long long)len <= (long long)max_pages * kPage)
+      np = int2_pages(len, sink, recent);
   }
   int x = np;
 #pragma unroll
@@ -210,6 +219,9 @@ __device__ __noinline__ void page_prefix(const int32_t* __restrict__ seq_lens,
   __syncthreads();
 }
 
+// WIN: the BF16-window phase is compiled in (a separate instance, so that
+// the INT2-only kernel keeps its own register allocation).
+template <bool WIN>
 __global__ void __launch_bounds__(kWarps * 32, 1)
 partial_tensor_kernel(const uint8_t* __restrict__ pool,
                       const int32_t* __restrict__ bt,
@@ -222,7 +234,7 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
                       const int* __restrict__ pref,
                       const int* __restrict__ nzpref,
                       float* __restrict__ part, int W, int early_pages,
-                      unsigned* err) {
+                      unsigned* err, int sink, int recent, WinPhase wp) {
   // One 16-warp CTA per SM: the warp schedulers favour the CTAs that
   // arrived first on an SM, and with four 4-warp CTAs per SM the last CTA
   // finished ~20% after the first; within one CTA the warps keep pace.
@@ -235,7 +247,11 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int g = lane >> 2, c = lane & 3;
   WarpSmemTC& S = smem[warp];
-  const int w = blockIdx.x * kWarps + warp;
+  // With BF16 windows, warps kWinIntWarps.. of every CTA are window warps
+  // (their loads overlap the INT2 pages of the others); the INT2 work is
+  // split over the first kWinIntWarps warps of each CTA.
+  constexpr int kInt = WIN ? kWinIntWarps : kWarps;
+  const int w = blockIdx.x * kInt + warp;  // INT2 warp index (warp < kInt)
 
   // Page prefix sums.  For up to kPrefCache sequences the CTA scans the
   // lengths itself (the values qrot writes to pref for the combine): the
@@ -251,11 +267,25 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
   static_assert(kPrefCache < kWarps * 32, "one thread per sequence");
   int F;
   if (cached) {
-    page_prefix(seq_lens, B, max_pages, spref, wsum);
+    page_prefix(seq_lens, B, max_pages, spref, wsum, sink, recent);
     F = spref[B] * h_kv;
   } else {
     pdl_wait();
     F = __ldcg(pref + B) * h_kv;
+  }
+  if constexpr (WIN) {
+    if (warp >= kInt) {
+      // window warp ww, numbered across the CTAs first so that a partial set
+      // is spread over the SMs.  The phase reads only inputs and
+      // library-owned state, so it runs before this grid waits for the
+      // previous kernel, in the warp's own page stages.
+      const int ww = (warp - kInt) * gridDim.x + blockIdx.x;
+      if (ww < wp.Ww)
+        window_phase(ww, wp, &S.stage[0][0], reinterpret_cast<uint8_t*>(&S.qfr[0][0]));
+      pdl_wait();
+      pdl_trigger();
+      return;
+    }
   }
   const int f0 = (int)((long long)w * F / W), f1 = (int)((long long)(w + 1) * F / W);
   if (f0 >= f1) {
@@ -266,7 +296,7 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
   PageChunk chk;
   int f_issue = f0;
   load_chunk(chk, f0, f1, pref, spref, cached, seq_lens, bt, B, h_kv,
-             max_pages, num_pages, err, lane);
+             max_pages, num_pages, err, lane, sink, recent);
 
   // issue one page into stage s (no commit); every lane records what the
   // stage holds
@@ -274,7 +304,7 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
     if (f_issue < f1) {
       if (f_issue - chk.base == 32)
         load_chunk(chk, f_issue, f1, pref, spref, cached, seq_lens, bt, B, h_kv,
-                   max_pages, num_pages, err, lane);
+                   max_pages, num_pages, err, lane, sink, recent);
       const int j = f_issue - chk.base;
       const int unit = __shfl_sync(0xffffffffu, chk.unit, j);
       const int key = __shfl_sync(0xffffffffu, chk.key, j);
@@ -641,15 +671,17 @@ cudaError_t launch_partial_tensor(const optr_params* p, const uint8_t* pool,
                                   const float* invs, const float* qs,
                                   const int* pref, const int* nzpref,
                                   float* part, int W, bool early_pages,
-                                  cudaStream_t s) {
+                                  const WinPhase& wp, cudaStream_t s) {
   const size_t dsmem = sizeof(WarpSmemTC) * kWarps;
-  cudaError_t e =
-      ensure_dynamic_smem(reinterpret_cast<const void*>(&partial_tensor_kernel), dsmem);
+  const bool win = wp.Ww > 0;
+  auto fn = win ? partial_tensor_kernel<true> : partial_tensor_kernel<false>;
+  cudaError_t e = ensure_dynamic_smem(reinterpret_cast<const void*>(fn), dsmem);
   if (e != cudaSuccess) return e;
-  return launch_pdl(partial_tensor_kernel, dim3(W / kWarps), dim3(kWarps * 32),
+  return launch_pdl(fn, dim3(W / (win ? kWinIntWarps : kWarps)), dim3(kWarps * 32),
                     dsmem, s, pool, bt, seq_lens, B, max_pages, num_pages,
                     p->cfg.h_q, p->cfg.h_kv, frag, koff, invs, qs, pref, nzpref,
-                    part, W, early_pages ? 1 : 0, p->err);
+                    part, W, early_pages ? 1 : 0, p->err, p->cfg.sink,
+                    p->cfg.recent, wp);
 }
 
 }  // namespace optr

@@ -67,6 +67,7 @@ cudaError_t ensure_dynamic_smem(const void* kernel, size_t bytes) {
 //   cnt  int   [B*h_kv]        combine arrival counters (zeroed by qrot)
 //   part float [W + B*h_kv][520] split-K partials (o'[4][128], m[4], l[4])
 //   cpart float [B*h_kv*S][520] combine chunk results (only when S > 1)
+//   wpart float [Ww + B*h_kv][520] window partials (BF16 windows only)
 // S, the combine CTAs per (sequence, KV head), is sized for ~32 partials
 // each when every sequence is max_pages long: a segment then overlaps about
 // W / (B*h_kv) + 2 warp ranges.
@@ -77,6 +78,21 @@ DecodePlan decode_plan(const optr_params* p, int B, int max_pages) {
   d.h_kv = p->cfg.h_kv;
   d.max_pages = max_pages;
   d.W = p->num_sms * kDecodeWarpsPerSm;
+  // BF16 windows: Uw units of 16 window tokens per (sequence, KV head);
+  // Ww window warps, each owning at least one unit: with the tensor-core
+  // partial kernel 4 per SM beside 12 INT2 warps (so W is 12 per SM), with
+  // the CUDA-core one every warp takes a share before its pages
+  d.Uw = (p->cfg.sink + p->cfg.recent + kWinUnit - 1) / kWinUnit;
+  const long long units = (long long)B * d.h_kv * d.Uw;
+  d.Ww = 0;
+  if (units > 0) {
+    if (p->cfg.decode_variant != OPTR_VARIANT_CUDA_CORE) {
+      d.W = p->num_sms * kWinIntWarps;
+      d.Ww = (int)std::min<long long>((long long)p->num_sms * (kDecodeWarpsPerSm - kWinIntWarps), units);
+    } else {
+      d.Ww = (int)std::min<long long>(d.W, units);
+    }
+  }
   size_t o = 0;
   d.off_qf = o;
   o = round_up(o + sizeof(float) * (size_t)B * d.h_q * kD, 256);
@@ -104,6 +120,10 @@ DecodePlan decode_plan(const optr_params* p, int B, int max_pages) {
   d.off_cpart = o;
   if (d.S > 1)
     o = round_up(o + sizeof(float) * kPartFloats * (size_t)B * d.h_kv * d.S, 256);
+  d.off_wpart = o;
+  if (d.Ww > 0)
+    o = round_up(o + sizeof(float) * kPartFloats *
+                         ((size_t)d.Ww + (size_t)B * d.h_kv), 256);
   d.total = o;
   return d;
 }
@@ -138,6 +158,9 @@ optr_status optr_params_create(const optr_config* cfg, const float* R_k,
       !(cfg->clip_v > 0.f && cfg->clip_v <= 1.f))
     return OPTR_ERR_INVALID_ARG;
   if (cfg->h_kv > 1024) return OPTR_ERR_OUT_OF_RANGE;
+  if (cfg->sink < 0 || cfg->recent < 0 || cfg->sink % kPage != 0)
+    return OPTR_ERR_INVALID_ARG;
+  if (cfg->sink > 1024 || cfg->recent > 1024) return OPTR_ERR_OUT_OF_RANGE;
 
   const int H = cfg->h_kv;
   const size_t mat = (size_t)kD * kD;
@@ -182,6 +205,7 @@ optr_status optr_params_create(const optr_config* cfg, const float* R_k,
   if (e == cudaSuccess) e = cudaMalloc(&p->R_v, sizeof(float) * H * mat);
   if (e == cudaSuccess) e = cudaMalloc(&p->R_vT, sizeof(float) * H * mat);
   if (e == cudaSuccess) e = cudaMalloc(&p->muR, sizeof(float) * H * kD);
+  if (e == cudaSuccess) e = cudaMalloc(&p->mu, sizeof(float) * H * kD);
   if (e == cudaSuccess) e = cudaMalloc(&p->err, sizeof(unsigned));
   std::vector<uint16_t> t5((size_t)H * kRT5Halves);
   if (e == cudaSuccess) e = cudaMalloc(&p->Rk_t5, sizeof(uint16_t) * t5.size());
@@ -208,6 +232,8 @@ optr_status optr_params_create(const optr_config* cfg, const float* R_k,
   if (e == cudaSuccess)
     e = cudaMemcpy(p->muR, muR.data(), sizeof(float) * H * kD,
                    cudaMemcpyHostToDevice);
+  if (e == cudaSuccess)
+    e = cudaMemcpy(p->mu, mu, sizeof(float) * H * kD, cudaMemcpyHostToDevice);
   if (e == cudaSuccess) e = cudaMemset(p->err, 0, sizeof(unsigned));
   if (e != cudaSuccess) {
     optr_params_destroy(p);
@@ -224,6 +250,7 @@ void optr_params_destroy(optr_params* p) {
   cudaFree(p->R_v);
   cudaFree(p->R_vT);
   cudaFree(p->muR);
+  cudaFree(p->mu);
   cudaFree(p->Rk_t5);
   cudaFree(p->Rv_t5);
   cudaFree(p->err);
@@ -234,13 +261,50 @@ size_t optr_page_bytes(const optr_params* p) {
   return p ? (size_t)p->cfg.h_kv * kChunk : 0;
 }
 
-optr_status optr_kv_append(const optr_params* p, const void* k, const void* v,
-                           int n_tok, const int32_t* cu_new,
-                           const int32_t* pos0, const int32_t* block_table,
-                           int B, int max_pages, uint8_t* pool, int num_pages,
-                           cudaStream_t stream) {
+namespace {
+
+bool windows_on(const optr_params* p) {
+  return p->cfg.sink > 0 || p->cfg.recent > 0;
+}
+
+// The window store of a _win call, validated: null when the windows are
+// off; *bad set when they are on and the store is missing or misaligned.
+const WinArgs* window_args(const optr_params* p, void* win,
+                           const int32_t* win_slot, int n_slots, WinArgs* buf,
+                           bool* bad) {
+  *bad = false;
+  if (!windows_on(p)) return nullptr;
+  if (!win || !win_slot || n_slots <= 0 || !aligned(win, 16)) {
+    *bad = true;
+    return nullptr;
+  }
+  buf->win = static_cast<__nv_bfloat16*>(win);
+  buf->slot = win_slot;
+  buf->n_slots = n_slots;
+  return buf;
+}
+
+}  // namespace
+
+size_t optr_window_bytes(const optr_params* p, int n_slots) {
+  if (!p || n_slots <= 0) return 0;
+  return (size_t)n_slots * p->cfg.h_kv * 2 * (p->cfg.sink + p->cfg.recent) *
+         kD * sizeof(uint16_t);
+}
+
+optr_status optr_kv_append_win(const optr_params* p, const void* k,
+                               const void* v, int n_tok, const int32_t* cu_new,
+                               const int32_t* pos0, const int32_t* block_table,
+                               int B, int max_pages, uint8_t* pool,
+                               int num_pages, void* win,
+                               const int32_t* win_slot, int n_slots,
+                               cudaStream_t stream) {
   if (!p || n_tok < 0 || B <= 0 || max_pages <= 0 || num_pages <= 0)
     return OPTR_ERR_INVALID_ARG;
+  WinArgs wbuf;
+  bool bad = false;
+  const WinArgs* wa = window_args(p, win, win_slot, n_slots, &wbuf, &bad);
+  if (bad) return OPTR_ERR_INVALID_ARG;
   if (n_tok == 0) return OPTR_OK;
   if (!k || !v || !cu_new || !pos0 || !block_table || !pool)
     return OPTR_ERR_INVALID_ARG;
@@ -264,8 +328,22 @@ optr_status optr_kv_append(const optr_params* p, const void* k, const void* v,
                              block_table, B, max_pages, pool, num_pages,
                              stream);
   prof_mark(p, 1, stream);
+  if (e == cudaSuccess && wa)
+    e = launch_window_copy(p, (const __nv_bfloat16*)k, (const __nv_bfloat16*)v,
+                           n_tok, cu_new, pos0, B, *wa, stream);
   if (p->prof) const_cast<optr_params*>(p)->ran[0] = 1;
   return cuda_status(e);
+}
+
+optr_status optr_kv_append(const optr_params* p, const void* k, const void* v,
+                           int n_tok, const int32_t* cu_new,
+                           const int32_t* pos0, const int32_t* block_table,
+                           int B, int max_pages, uint8_t* pool, int num_pages,
+                           cudaStream_t stream) {
+  if (p && windows_on(p)) return OPTR_ERR_INVALID_ARG;
+  return optr_kv_append_win(p, k, v, n_tok, cu_new, pos0, block_table, B,
+                            max_pages, pool, num_pages, nullptr, nullptr, 0,
+                            stream);
 }
 
 size_t optr_decode_workspace_size(const optr_params* p, int B, int max_pages) {
@@ -273,18 +351,25 @@ size_t optr_decode_workspace_size(const optr_params* p, int B, int max_pages) {
   return decode_plan(p, B, max_pages).total;
 }
 
-optr_status optr_decode_attention(const optr_params* p, const void* q,
-                                  const int32_t* block_table,
-                                  const int32_t* seq_lens, int B,
-                                  int max_pages, const uint8_t* pool,
-                                  int num_pages, float* out, void* workspace,
-                                  size_t ws_bytes, cudaStream_t stream) {
+optr_status optr_decode_attention_win(const optr_params* p, const void* q,
+                                      const int32_t* block_table,
+                                      const int32_t* seq_lens, int B,
+                                      int max_pages, const uint8_t* pool,
+                                      int num_pages, const void* win,
+                                      const int32_t* win_slot, int n_slots,
+                                      float* out, void* workspace,
+                                      size_t ws_bytes, cudaStream_t stream) {
   if (!p || B <= 0 || max_pages <= 0 || num_pages <= 0)
     return OPTR_ERR_INVALID_ARG;
   if (!q || !block_table || !seq_lens || !pool || !out)
     return OPTR_ERR_INVALID_ARG;
   if (!aligned(pool, 16) || !aligned(q, 16) || !aligned(out, 16))
     return OPTR_ERR_INVALID_ARG;
+  WinArgs wbuf;
+  bool bad = false;
+  const WinArgs* wa = window_args(p, const_cast<void*>(win), win_slot, n_slots,
+                                  &wbuf, &bad);
+  if (bad) return OPTR_ERR_INVALID_ARG;
   if ((long long)max_pages * kPage > (1LL << 30) || B > (1 << 24))
     return OPTR_ERR_OUT_OF_RANGE;
   // the split-K plan indexes (sequence, KV head, page) units with 32 bits
@@ -296,19 +381,33 @@ optr_status optr_decode_attention(const optr_params* p, const void* q,
   int variant = p->cfg.decode_variant;
   cudaError_t e = launch_decode(p, variant, (const __nv_bfloat16*)q,
                                 block_table, seq_lens, B, max_pages, pool,
-                                num_pages, out, workspace, plan, stream);
+                                num_pages, out, workspace, plan, stream,
+                                nullptr, wa);
   if (p->prof) const_cast<optr_params*>(p)->ran[1] = 1;
   return cuda_status(e);
 }
 
-optr_status optr_decode_step(const optr_params* p, const void* q,
-                             const void* k, const void* v, int n_tok,
-                             const int32_t* cu_new, const int32_t* pos0,
-                             const int32_t* block_table,
-                             const int32_t* seq_lens, int B, int max_pages,
-                             uint8_t* pool, int num_pages, float* out,
-                             void* workspace, size_t ws_bytes,
-                             cudaStream_t stream) {
+optr_status optr_decode_attention(const optr_params* p, const void* q,
+                                  const int32_t* block_table,
+                                  const int32_t* seq_lens, int B,
+                                  int max_pages, const uint8_t* pool,
+                                  int num_pages, float* out, void* workspace,
+                                  size_t ws_bytes, cudaStream_t stream) {
+  if (p && windows_on(p)) return OPTR_ERR_INVALID_ARG;
+  return optr_decode_attention_win(p, q, block_table, seq_lens, B, max_pages,
+                                   pool, num_pages, nullptr, nullptr, 0, out,
+                                   workspace, ws_bytes, stream);
+}
+
+optr_status optr_decode_step_win(const optr_params* p, const void* q,
+                                 const void* k, const void* v, int n_tok,
+                                 const int32_t* cu_new, const int32_t* pos0,
+                                 const int32_t* block_table,
+                                 const int32_t* seq_lens, int B, int max_pages,
+                                 uint8_t* pool, int num_pages, void* win,
+                                 const int32_t* win_slot, int n_slots,
+                                 float* out, void* workspace, size_t ws_bytes,
+                                 cudaStream_t stream) {
   if (!p || n_tok < 0 || B <= 0 || max_pages <= 0 || num_pages <= 0)
     return OPTR_ERR_INVALID_ARG;
   if (!q || !block_table || !seq_lens || !pool || !out)
@@ -317,6 +416,10 @@ optr_status optr_decode_step(const optr_params* p, const void* q,
   if (!aligned(pool, 16) || !aligned(q, 16) || !aligned(out, 16) ||
       (n_tok > 0 && (!aligned(k, 16) || !aligned(v, 16))))
     return OPTR_ERR_INVALID_ARG;
+  WinArgs wbuf;
+  bool bad = false;
+  const WinArgs* wa = window_args(p, win, win_slot, n_slots, &wbuf, &bad);
+  if (bad) return OPTR_ERR_INVALID_ARG;
   if ((long long)max_pages * kPage > (1LL << 30) || B > (1 << 24))
     return OPTR_ERR_OUT_OF_RANGE;
   if ((long long)B * max_pages * p->cfg.h_kv >= (1LL << 31))
@@ -328,19 +431,37 @@ optr_status optr_decode_step(const optr_params* p, const void* q,
   // anything else runs as the two calls
   if (n_tok == 0 || n_tok > 256 || p->cfg.decode_variant == OPTR_VARIANT_CUDA_CORE ||
       p->cfg.append_variant == OPTR_VARIANT_CUDA_CORE) {
-    optr_status st = optr_kv_append(p, k, v, n_tok, cu_new, pos0, block_table,
-                                    B, max_pages, pool, num_pages, stream);
+    optr_status st = optr_kv_append_win(p, k, v, n_tok, cu_new, pos0,
+                                        block_table, B, max_pages, pool,
+                                        num_pages, win, win_slot, n_slots,
+                                        stream);
     if (st != OPTR_OK) return st;
-    return optr_decode_attention(p, q, block_table, seq_lens, B, max_pages, pool,
-                                 num_pages, out, workspace, ws_bytes, stream);
+    return optr_decode_attention_win(p, q, block_table, seq_lens, B, max_pages,
+                                     pool, num_pages, win, win_slot, n_slots,
+                                     out, workspace, ws_bytes, stream);
   }
   StepAppend app{(const __nv_bfloat16*)k, (const __nv_bfloat16*)v, n_tok,
                  cu_new, pos0, pool};
   cudaError_t e = launch_decode(p, p->cfg.decode_variant, (const __nv_bfloat16*)q,
                                 block_table, seq_lens, B, max_pages, pool,
-                                num_pages, out, workspace, plan, stream, &app);
+                                num_pages, out, workspace, plan, stream, &app,
+                                wa);
   if (p->prof) const_cast<optr_params*>(p)->ran[0] = const_cast<optr_params*>(p)->ran[1] = 1;
   return cuda_status(e);
+}
+
+optr_status optr_decode_step(const optr_params* p, const void* q,
+                             const void* k, const void* v, int n_tok,
+                             const int32_t* cu_new, const int32_t* pos0,
+                             const int32_t* block_table,
+                             const int32_t* seq_lens, int B, int max_pages,
+                             uint8_t* pool, int num_pages, float* out,
+                             void* workspace, size_t ws_bytes,
+                             cudaStream_t stream) {
+  if (p && windows_on(p)) return OPTR_ERR_INVALID_ARG;
+  return optr_decode_step_win(p, q, k, v, n_tok, cu_new, pos0, block_table,
+                              seq_lens, B, max_pages, pool, num_pages, nullptr,
+                              nullptr, 0, out, workspace, ws_bytes, stream);
 }
 
 optr_status optr_profile_enable(optr_params* p, int on) {

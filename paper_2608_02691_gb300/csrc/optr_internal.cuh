@@ -21,6 +21,9 @@ constexpr int kMaxRatio = 8;             // largest supported h_q / h_kv
 // partial kernel; the workspace holds one partial slot per warp plus one per
 // (sequence, KV head), see DecodePlan.
 constexpr int kDecodeWarpsPerSm = 16;
+// with BF16 windows the tensor-core partial kernel keeps 12 of its 16 warps
+// per SM on the INT2 pages and gives 4 to the window units
+constexpr int kWinIntWarps = 12;
 constexpr int kCombineMaxSplit = 16;  // combine CTAs per (sequence, KV head)
 
 }  // namespace optr
@@ -35,6 +38,7 @@ struct optr_params {
   float* R_v;          // device [h_kv][D][D]
   float* R_vT;         // device [h_kv][D][D], R_vT[h][j][i] = R_v[h][i][j]
   float* muR;          // device [h_kv][D], mu R_k computed in fp64
+  float* mu;           // device [h_kv][D], the key mean (window logits)
   uint16_t* Rk_t5;     // device tcgen05 B operands of R_k (append_tc05.cu)
   uint16_t* Rv_t5;     // device tcgen05 B operands of R_v
   unsigned* err;       // device error word
@@ -97,14 +101,54 @@ namespace optr {
 struct DecodePlan {
   int B, h_q, h_kv, max_pages, W;  // W = partial-kernel warps
   int S;                           // combine CTAs per (sequence, KV head)
+  int Uw;   // BF16-window units (16 window tokens) per (sequence, KV head)
+  int Ww;   // warps that take window units: min(W, B * h_kv * Uw)
   size_t off_qf, off_qs, off_frag, off_koff, off_invs, off_pref, off_cnt,
-      off_part, off_cpart, total;
+      off_part, off_cpart, off_wpart, total;
 };
 DecodePlan decode_plan(const optr_params* p, int B, int max_pages);
 
 // One split-K partial (float32): the unnormalised rotated output o'[4][128]
 // of the 4 query heads of a GQA group, then their running maxima m[4]
 // (log2 domain) and sums l[4].
+// BF16 windows (Sec. 3.1 and 4.1; include/optr.h "BF16 windows"): of a
+// sequence holding n tokens, positions s < sink and s >= n - recent are
+// window positions; the INT2 positions are [sink, int2_end).  With
+// sink = recent = 0 every position is INT2.
+__host__ __device__ __forceinline__ int int2_end(int n, int sink, int recent) {
+  return n - recent > sink ? n - recent : sink;
+}
+// INT2 pages of the sequence: logical pages sink/16 .. ceil(int2_end/16)-1
+// (sink is a multiple of 16, so the first one is full).
+__host__ __device__ __forceinline__ int int2_pages(int n, int sink, int recent) {
+  const int e = int2_end(n, sink, recent);
+  return e > sink ? (e + kPage - 1) / kPage - sink / kPage : 0;
+}
+// Window positions of the sequence, listed sink part first: count, and the
+// position of list entry i.
+__host__ __device__ __forceinline__ int win_count(int n, int sink, int recent) {
+  const int ns = n < sink ? n : sink;
+  const int r0 = n - recent > sink ? n - recent : sink;
+  return ns + (n > r0 ? n - r0 : 0);
+}
+__host__ __device__ __forceinline__ int win_pos(int i, int n, int sink, int recent) {
+  const int ns = n < sink ? n : sink;
+  const int r0 = n - recent > sink ? n - recent : sink;
+  return i < ns ? i : r0 + (i - ns);
+}
+// Store row of window position s (recent > 0 whenever s >= sink).
+__host__ __device__ __forceinline__ int win_row(int s, int sink, int recent) {
+  return s < sink ? s : sink + (s - sink) % recent;
+}
+constexpr int kWinUnit = 16;  // window tokens per decode work unit
+
+// Window store arguments of one call (null when the windows are off).
+struct WinArgs {
+  __nv_bfloat16* win;     // [n_slots][h_kv][2][sink + recent][D]
+  const int32_t* slot;    // [B]
+  int n_slots;
+};
+
 constexpr int kPartFloats = 4 * kD + 8;
 constexpr int kPartM = 4 * kD;
 constexpr int kPartL = 4 * kD + 4;
@@ -140,6 +184,13 @@ cudaError_t launch_decode(const optr_params* p, int variant,
                           const int32_t* seq_lens, int B, int max_pages,
                           const uint8_t* pool, int num_pages, float* out,
                           void* ws, const DecodePlan& plan, cudaStream_t s,
-                          const StepAppend* app = nullptr);
+                          const StepAppend* app, const WinArgs* win);
+
+// Window part of a cache write (positions of the BF16 windows copied into
+// the store); a separate launch after the INT2 write.
+cudaError_t launch_window_copy(const optr_params* p, const __nv_bfloat16* k,
+                               const __nv_bfloat16* v, int n_tok,
+                               const int32_t* cu_new, const int32_t* pos0,
+                               int B, const WinArgs& win, cudaStream_t s);
 
 }  // namespace optr

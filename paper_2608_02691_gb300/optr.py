@@ -25,6 +25,14 @@ OPTR_VARIANT_CUDA_CORE = 1
 OPTR_VARIANT_TENSOR = 2
 PAGE_HEAD_BYTES = 1536
 HEAD_DIM = 128
+# device error bits (optr_device_error)
+OPTR_DEVERR_PAGE_ID = 1
+OPTR_DEVERR_POSITION = 2
+OPTR_DEVERR_SEQ_LEN = 4
+OPTR_DEVERR_CU_NEW = 8
+OPTR_DEVERR_FP16_RANGE = 16
+OPTR_DEVERR_TIMEOUT = 32
+OPTR_DEVERR_WIN_SLOT = 64
 
 
 class OptrError(RuntimeError):
@@ -38,7 +46,8 @@ class optr_config(ctypes.Structure):
                 ("head_dim", ctypes.c_int), ("group", ctypes.c_int),
                 ("page_size", ctypes.c_int), ("clip_k", ctypes.c_float),
                 ("clip_v", ctypes.c_float), ("append_variant", ctypes.c_int),
-                ("decode_variant", ctypes.c_int)]
+                ("decode_variant", ctypes.c_int), ("sink", ctypes.c_int),
+                ("recent", ctypes.c_int)]
 
 
 _V = ctypes.c_void_p
@@ -58,6 +67,14 @@ _SIG = {
                                            _V, _V]),
     "optr_decode_step": (_I, [_V, _V, _V, _V, _I, _V, _V, _V, _V, _I, _I, _V,
                               _I, _V, _V, ctypes.c_size_t, _V]),
+    "optr_window_bytes": (ctypes.c_size_t, [_V, _I]),
+    "optr_kv_append_win": (_I, [_V, _V, _V, _I, _V, _V, _V, _I, _I, _V, _I,
+                                _V, _V, _I, _V]),
+    "optr_decode_attention_win": (_I, [_V, _V, _V, _V, _I, _I, _V, _I, _V,
+                                       _V, _I, _V, _V, ctypes.c_size_t, _V]),
+    "optr_decode_step_win": (_I, [_V, _V, _V, _V, _I, _V, _V, _V, _V, _I, _I,
+                                  _V, _I, _V, _V, _I, _V, _V, ctypes.c_size_t,
+                                  _V]),
     "optr_profile_enable": (_I, [_V, _I]),
     "optr_profile_last": (_I, [_V, ctypes.POINTER(ctypes.c_float)]),
 }
@@ -135,10 +152,12 @@ class Params:
 def optr_params_create(R_k, R_v, mu, h_q: int, clip_k: float = 1.0,
                        clip_v: float = 1.0,
                        append_variant: int = OPTR_VARIANT_DEFAULT,
-                       decode_variant: int = OPTR_VARIANT_DEFAULT) -> Params:
+                       decode_variant: int = OPTR_VARIANT_DEFAULT,
+                       sink: int = 0, recent: int = 0) -> Params:
     """R_k, R_v float32 [h_kv][128][128] and mu float32 [h_kv][128] (host
     tensors); the library copies them to the current CUDA device.  R_v may be
-    None: the value rotation is folded into the model's W_V / W_O."""
+    None: the value rotation is folded into the model's W_V / W_O.  sink /
+    recent > 0 keep BF16 windows (the *_win calls)."""
     R_k = R_k.detach().to("cpu", torch.float32).contiguous()
     if R_v is not None:
         R_v = R_v.detach().to("cpu", torch.float32).contiguous()
@@ -148,7 +167,7 @@ def optr_params_create(R_k, R_v, mu, h_q: int, clip_k: float = 1.0,
             mu.shape != (h_kv, 128):
         raise ValueError("R_k, R_v must be [h_kv][128][128], mu [h_kv][128]")
     cfg = optr_config(h_q, h_kv, 128, 32, 16, clip_k, clip_v, append_variant,
-                      decode_variant)
+                      decode_variant, sink, recent)
     h = ctypes.c_void_p()
     _check(lib().optr_params_create(ctypes.byref(cfg), _ptr(R_k),
                                     None if R_v is None else _ptr(R_v),
@@ -219,6 +238,84 @@ def optr_decode_step(p: Params, q, k, v, cu_new, pos0, block_table, seq_lens,
         _ptr(pos0), _ptr(block_table), _ptr(seq_lens), B, max_pages,
         _ptr(pool), pool.shape[0], _ptr(out), _ptr(workspace),
         workspace.numel(), _stream(stream)), "optr_decode_step")
+
+
+def optr_window_bytes(p: Params, n_slots: int) -> int:
+    return int(lib().optr_window_bytes(p.handle, n_slots))
+
+
+def _win_args(p, win, win_slot):
+    if win is None:
+        return None, None, 0
+    _dev(win, torch.bfloat16, "win")
+    _dev(win_slot, torch.int32, "win_slot")
+    rows = p.cfg.sink + p.cfg.recent
+    if tuple(win.shape[1:]) != (p.h_kv, 2, rows, 128):
+        raise ValueError("win must be [n_slots][h_kv][2][sink + recent][128]")
+    return _ptr(win), _ptr(win_slot), win.shape[0]
+
+
+def optr_kv_append_win(p: Params, k, v, cu_new, pos0, block_table, pool, win,
+                       win_slot, stream=None) -> None:
+    """optr_kv_append plus the BF16-window copy: win bf16
+    [n_slots][h_kv][2][sink + recent][128], win_slot int32 [B]."""
+    for t, dt, nm in ((k, torch.bfloat16, "k"), (v, torch.bfloat16, "v"),
+                      (cu_new, torch.int32, "cu_new"), (pos0, torch.int32, "pos0"),
+                      (block_table, torch.int32, "block_table"),
+                      (pool, torch.uint8, "pool")):
+        _dev(t, dt, nm)
+    w, ws_, n_slots = _win_args(p, win, win_slot)
+    B, max_pages = block_table.shape
+    _check(lib().optr_kv_append_win(
+        p.handle, _ptr(k), _ptr(v), k.shape[0], _ptr(cu_new), _ptr(pos0),
+        _ptr(block_table), B, max_pages, _ptr(pool), pool.shape[0], w, ws_,
+        n_slots, _stream(stream)), "optr_kv_append_win")
+
+
+def optr_decode_attention_win(p: Params, q, block_table, seq_lens, pool, win,
+                              win_slot, out, workspace, stream=None) -> None:
+    """optr_decode_attention with the BF16 windows read from win."""
+    for t, dt, nm in ((q, torch.bfloat16, "q"),
+                      (block_table, torch.int32, "block_table"),
+                      (seq_lens, torch.int32, "seq_lens"),
+                      (pool, torch.uint8, "pool"), (out, torch.float32, "out"),
+                      (workspace, torch.uint8, "workspace")):
+        _dev(t, dt, nm)
+    w, ws_, n_slots = _win_args(p, win, win_slot)
+    B, max_pages = block_table.shape
+    _check(lib().optr_decode_attention_win(
+        p.handle, _ptr(q), _ptr(block_table), _ptr(seq_lens), B, max_pages,
+        _ptr(pool), pool.shape[0], w, ws_, n_slots, _ptr(out), _ptr(workspace),
+        workspace.numel(), _stream(stream)), "optr_decode_attention_win")
+
+
+def optr_decode_step_win(p: Params, q, k, v, cu_new, pos0, block_table,
+                         seq_lens, pool, win, win_slot, out, workspace,
+                         stream=None) -> None:
+    """optr_decode_step with BF16 windows: the step's window copies and the
+    windowed decode."""
+    for t, dt, nm in ((q, torch.bfloat16, "q"), (k, torch.bfloat16, "k"),
+                      (v, torch.bfloat16, "v"), (cu_new, torch.int32, "cu_new"),
+                      (pos0, torch.int32, "pos0"),
+                      (block_table, torch.int32, "block_table"),
+                      (seq_lens, torch.int32, "seq_lens"),
+                      (pool, torch.uint8, "pool"), (out, torch.float32, "out"),
+                      (workspace, torch.uint8, "workspace")):
+        _dev(t, dt, nm)
+    w, ws_, n_slots = _win_args(p, win, win_slot)
+    B, max_pages = block_table.shape
+    _check(lib().optr_decode_step_win(
+        p.handle, _ptr(q), _ptr(k), _ptr(v), k.shape[0], _ptr(cu_new),
+        _ptr(pos0), _ptr(block_table), _ptr(seq_lens), B, max_pages,
+        _ptr(pool), pool.shape[0], w, ws_, n_slots, _ptr(out), _ptr(workspace),
+        workspace.numel(), _stream(stream)), "optr_decode_step_win")
+
+
+def new_windows(p: Params, n_slots: int, device="cuda") -> torch.Tensor:
+    """A zero-filled window store [n_slots][h_kv][2][sink + recent][128]
+    (bf16)."""
+    return torch.zeros(n_slots, p.h_kv, 2, p.cfg.sink + p.cfg.recent, 128,
+                       dtype=torch.bfloat16, device=device)
 
 
 NOALLOC_SCRATCH_BYTES = 16 << 20
