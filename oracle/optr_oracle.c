@@ -185,15 +185,22 @@ static void rotate_back(const double* x, const float* R, double* y) {
   }
 }
 
-/* Q2 applied group by group to a rotated 128-vector; codes/scale/min and
- * (optionally) the pre-rounding values are returned. */
-static void quantize_vector(const double* z, float clip, uint8_t* codes,
+/* Q2 applied group by group to a rotated 128-vector, groups of G = 32 or
+ * 128 consecutive channels (Sec. 3.1, group size G; the paper's default is
+ * 128, Sec. 5); codes and (optionally) the pre-rounding values are
+ * returned, and scale/min per 32-channel block of the stored layout: with
+ * G = 128 the one group's pair is repeated in its four blocks. */
+static void quantize_vector(const double* z, float clip, int G, uint8_t* codes,
                             uint16_t* scale, uint16_t* mn, float* u) {
-  for (int g = 0; g < OR_D / OR_G; ++g) {
-    float zf[OR_G];
-    for (int i = 0; i < OR_G; ++i) zf[i] = (float)z[g * OR_G + i];
-    oracle_quantize_group(zf, OR_G, clip, codes + g * OR_G, scale + g, mn + g,
-                          u ? u + g * OR_G : NULL);
+  for (int g0 = 0; g0 < OR_D; g0 += G) {
+    float zf[OR_D];
+    uint16_t s, m;
+    for (int i = 0; i < G; ++i) zf[i] = (float)z[g0 + i];
+    oracle_quantize_group(zf, G, clip, codes + g0, &s, &m, u ? u + g0 : NULL);
+    for (int blk = g0 / OR_G; blk < (g0 + G) / OR_G; ++blk) {
+      scale[blk] = s;
+      mn[blk] = m;
+    }
   }
 }
 
@@ -215,16 +222,18 @@ int oracle_get_threads(void) { return g_threads; }
  * Arrays: k, v bf16 bits [n_tok][h_kv][128]; R_k, R_v float32
  * [h_kv][128][128]; mu float32 [h_kv][128].  u_out (optional, float32
  * [n_tok][h_kv][2][128]) receives the pre-rounding values of the key
- * (index 0) and value (index 1) codes.  Returns 0, or -1 when a table entry
- * or position is out of range (nothing is written for that token).
+ * (index 0) and value (index 1) codes.  group: Q2 group size, 32 or 128.
+ * Returns 0, or -1 when a table entry or position is out of range (nothing
+ * is written for that token) or the group size is not supported.
  */
 int oracle_kv_append(const uint16_t* k, const uint16_t* v, int n_tok,
                      const int32_t* cu_new, const int32_t* pos0,
                      const int32_t* block_table, int B, int max_pages,
                      uint8_t* pool, int num_pages, int h_kv, const float* R_k,
                      const float* R_v, const float* mu, float clip_k,
-                     float clip_v, float* u_out) {
+                     float clip_v, float* u_out, int group) {
   int bad = 0;
+  if (group != 32 && group != 128) return -1;
   if (cu_new[0] != 0 || cu_new[B] != n_tok) return -1;
 #pragma omp parallel for schedule(dynamic, 16) num_threads(g_threads) reduction(|: bad)
   for (int t = 0; t < n_tok; ++t) {
@@ -250,8 +259,8 @@ int oracle_kv_append(const uint16_t* k, const uint16_t* v, int n_tok,
       uint16_t sk[4], mk[4], sv[4], mv[4];
       float* uk = u_out ? u_out + (((size_t)t * h_kv + h) * 2 + 0) * OR_D : NULL;
       float* uv = u_out ? u_out + (((size_t)t * h_kv + h) * 2 + 1) * OR_D : NULL;
-      quantize_vector(zk, clip_k, ck, sk, mk, uk);
-      quantize_vector(zv, clip_v, cv, sv, mv, uv);
+      quantize_vector(zk, clip_k, group, ck, sk, mk, uk);
+      quantize_vector(zv, clip_v, group, cv, sv, mv, uv);
       uint8_t* c = chunk_of(pool, page, h_kv, h);
       store_slot(c, OR_KC, OR_KM, slot, ck, sk, mk);
       store_slot(c, OR_VC, OR_VM, slot, cv, sv, mv);
@@ -502,7 +511,7 @@ int oracle_attention_dense_win(const double* q, const double* K,
                                const float* R_v, const double* mu,
                                int quantize, float clip_k, float clip_v,
                                int sink, int recent, double* out,
-                               double* p_out) {
+                               double* p_out, int group) {
   if (n <= 0) {
     for (int i = 0; i < OR_D; ++i) out[i] = 0.0;
     return 0;
@@ -523,7 +532,7 @@ int oracle_attention_dense_win(const double* q, const double* K,
     if (quantize) {
       uint8_t c[OR_D];
       uint16_t sc[4], mn[4];
-      quantize_vector(z, clip_k, c, sc, mn, NULL);
+      quantize_vector(z, clip_k, group, c, sc, mn, NULL);
       for (int i = 0; i < OR_D; ++i) zq[i] = dequant(c[i], sc[i / OR_G], mn[i / OR_G]);
     } else {
       for (int i = 0; i < OR_D; ++i) zq[i] = z[i];
@@ -535,7 +544,7 @@ int oracle_attention_dense_win(const double* q, const double* K,
     if (quantize) {
       uint8_t c[OR_D];
       uint16_t sc[4], mn[4];
-      quantize_vector(z, clip_v, c, sc, mn, NULL);
+      quantize_vector(z, clip_v, group, c, sc, mn, NULL);
       for (int i = 0; i < OR_D; ++i) zq[i] = dequant(c[i], sc[i / OR_G], mn[i / OR_G]);
     } else {
       for (int i = 0; i < OR_D; ++i) zq[i] = z[i];
@@ -554,15 +563,22 @@ int oracle_attention_dense(const double* q, const double* K, const double* V,
                            const double* mu, int quantize, float clip_k,
                            float clip_v, double* out, double* p_out) {
   return oracle_attention_dense_win(q, K, V, n, R_k, R_v, mu, quantize, clip_k,
-                                    clip_v, 0, 0, out, p_out);
+                                    clip_v, 0, 0, out, p_out, OR_G);
 }
 
 /* Exported for tests: z = x R (fp64) and the group quantization of z, for
- * one 128-vector. */
+ * one 128-vector, groups of `group` (32 or 128) channels. */
+int oracle_rotate_quantize_g(const double* x, const float* R, float clip,
+                             double* z, uint8_t* codes, uint16_t* scale,
+                             uint16_t* mn, float* u, int group) {
+  if (group != 32 && group != 128) return -1;
+  rotate(x, R, z);
+  quantize_vector(z, clip, group, codes, scale, mn, u);
+  return 0;
+}
+
 int oracle_rotate_quantize(const double* x, const float* R, float clip,
                            double* z, uint8_t* codes, uint16_t* scale,
                            uint16_t* mn, float* u) {
-  rotate(x, R, z);
-  quantize_vector(z, clip, codes, scale, mn, u);
-  return 0;
+  return oracle_rotate_quantize_g(x, R, clip, z, codes, scale, mn, u, OR_G);
 }

@@ -60,7 +60,7 @@ def _declare(L):
     L.oracle_quantize_group.argtypes = [_P, i, f, _P, _P, _P, _P]
     L.oracle_quantize_group.restype = i
     L.oracle_kv_append.argtypes = [_P, _P, i, _P, _P, _P, i, i, _P, i, i, _P,
-                                   _P, _P, f, f, _P]
+                                   _P, _P, f, f, _P, i]
     L.oracle_kv_append.restype = i
     L.oracle_decode_attention.argtypes = [_P, _P, _P, i, i, _P, i, i, i, _P,
                                           _P, _P, _P, _P, i, _P]
@@ -72,13 +72,15 @@ def _declare(L):
     L.oracle_window_write.argtypes = [_P, _P, i, _P, _P, i, _P, i, i, i, i, _P]
     L.oracle_window_write.restype = i
     L.oracle_attention_dense_win.argtypes = [_P, _P, _P, i, _P, _P, _P, i, f,
-                                             f, i, i, _P, _P]
+                                             f, i, i, _P, _P, i]
     L.oracle_attention_dense_win.restype = i
     L.oracle_attention_dense.argtypes = [_P, _P, _P, i, _P, _P, _P, i, f, f,
                                          _P, _P]
     L.oracle_attention_dense.restype = i
     L.oracle_rotate_quantize.argtypes = [_P, _P, f, _P, _P, _P, _P, _P]
     L.oracle_rotate_quantize.restype = i
+    L.oracle_rotate_quantize_g.argtypes = [_P, _P, f, _P, _P, _P, _P, _P, i]
+    L.oracle_rotate_quantize_g.restype = i
     L.oracle_read_slot.argtypes = [_P, i, i, i, i, _P, _P]
     L.oracle_read_slot.restype = i
     L.oracle_code_byte.argtypes = [i]
@@ -122,8 +124,10 @@ def quantize_group(z, clip: float = 1.0):
     return codes, int(s[0]), int(m[0]), u, bool(deg)
 
 
-def rotate_quantize(x, R, clip: float = 1.0):
-    """z = x R (fp64) and its per-group quantization for one 128-vector."""
+def rotate_quantize(x, R, clip: float = 1.0, group: int = 32):
+    """z = x R (fp64) and its per-group quantization for one 128-vector
+    (groups of ``group`` = 32 or 128 channels; scale/min per 32-channel
+    block of the stored layout)."""
     x = _c(x, np.float64)
     R = _c(R, np.float32)
     z = np.zeros(D, np.float64)
@@ -131,13 +135,16 @@ def rotate_quantize(x, R, clip: float = 1.0):
     s = np.zeros(4, np.uint16)
     m = np.zeros(4, np.uint16)
     u = np.zeros(D, np.float32)
-    lib().oracle_rotate_quantize(_ptr(x), _ptr(R), float(clip), _ptr(z),
-                                 _ptr(codes), _ptr(s), _ptr(m), _ptr(u))
+    rc = lib().oracle_rotate_quantize_g(_ptr(x), _ptr(R), float(clip), _ptr(z),
+                                        _ptr(codes), _ptr(s), _ptr(m), _ptr(u),
+                                        int(group))
+    if rc != 0:
+        raise ValueError("group size must be 32 or 128")
     return z, codes, s, m, u
 
 
 def kv_append(k_bits, v_bits, cu_new, pos0, block_table, pool, R_k, R_v, mu,
-              clip_k=1.0, clip_v=1.0, want_u=False):
+              clip_k=1.0, clip_v=1.0, want_u=False, group=32):
     """Oracle cache write; ``pool`` (uint8 [num_pages][h_kv][1536]) is
     modified in place.  Returns the pre-rounding values when want_u."""
     k_bits = _c(k_bits, np.uint16)
@@ -155,9 +162,10 @@ def kv_append(k_bits, v_bits, cu_new, pos0, block_table, pool, R_k, R_v, mu,
         _ptr(k_bits), _ptr(v_bits), n_tok, _ptr(cu_new), _ptr(pos0), _ptr(bt),
         B, max_pages, _ptr(pool), num_pages, h_kv, _ptr(_c(R_k, np.float32)),
         _ptr(_c(R_v, np.float32)), _ptr(_c(mu, np.float32)), float(clip_k),
-        float(clip_v), _ptr(u))
+        float(clip_v), _ptr(u), int(group))
     if rc != 0:
-        raise ValueError("oracle_kv_append: table entry or position out of range")
+        raise ValueError("oracle_kv_append: table entry or position out of range"
+                         " (or group size not 32 / 128)")
     return u
 
 
@@ -229,7 +237,7 @@ def window_write(k_bits, v_bits, cu_new, pos0, win, win_slot, sink, recent):
 
 
 def attention_dense(q, K, V, R_k, R_v, mu, quantize=True, clip_k=1.0,
-                    clip_v=1.0, want_p=False, sink=0, recent=0):
+                    clip_v=1.0, want_p=False, sink=0, recent=0, group=32):
     """Single-head dense statement in the inverse-rotation form; positions
     s < sink or s >= n - recent are BF16 window positions."""
     q = _c(q, np.float64)
@@ -244,7 +252,7 @@ def attention_dense(q, K, V, R_k, R_v, mu, quantize=True, clip_k=1.0,
                                      _ptr(_c(mu, np.float64)),
                                      int(bool(quantize)), float(clip_k),
                                      float(clip_v), int(sink), int(recent),
-                                     _ptr(out), _ptr(p))
+                                     _ptr(out), _ptr(p), int(group))
     return (out, p[:n]) if want_p else out
 
 
