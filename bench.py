@@ -364,36 +364,43 @@ def extra_workloads(args, dev):
     hbm_peak, _ = peaks()
     flush = Flusher(dev)
     res = {}
-    # prefill append: 4 x 32768 tokens
-    wl = synth.workload("prefill", args.seed)
-    case = synth.build_case(wl, args.seed, device=dev)
-    p = optr.optr_params_create(case["R_k"], case["R_v"], case["mu"],
-                                case["h_q"], append_variant=args.append_variant)
-    pool = optr.new_pool(p, case["num_pages"], device=dev)
-    bt = case["block_table"].to(dev)
-    k, v = case["k_new"].to(dev), case["v_new"].to(dev)
-    cu, pos0 = case["cu_new"].to(dev), case["pos0_new"].to(dev)
-    for _ in range(3):
-        optr.optr_kv_append(p, k, v, cu, pos0, bt, pool)
-    optr.optr_profile_enable(p, True)
-    t = []
-    for _ in range(max(5, args.steps // 4)):
-        flush()
-        optr.optr_kv_append(p, k, v, cu, pos0, bt, pool)
-        t.append(optr.optr_profile_last(p)["append"])
-    optr.optr_profile_enable(p, False)
-    ms = float(np.mean(t))
-    n_tok = k.shape[0]
-    nb = append_bytes(n_tok, case["h_kv"])
-    res["prefill_append"] = {
-        "tokens": n_tok, "ms": round(ms, 4),
-        "tokens_per_s": round(n_tok / (ms * 1e-3), 1),
-        "gbs": round(nb / (ms * 1e-3) / 1e9, 1),
-        "frac": round(nb / (ms * 1e-3) / 1e9 / hbm_peak, 4)}
-    del pool, k, v, case
-    torch.cuda.empty_cache()
+    # prefill append: 4 x 32768 tokens (G = 32 on the tcgen05 cache write;
+    # G = 128, the paper's default, on the CUDA-core one)
+    for key, group in (("prefill_append", 32), ("prefill_append_g128", 128)):
+        wl = synth.workload("prefill", args.seed)
+        case = synth.build_case(wl, args.seed, device=dev)
+        p = optr.optr_params_create(case["R_k"], case["R_v"], case["mu"],
+                                    case["h_q"], append_variant=args.append_variant,
+                                    group=group)
+        pool = optr.new_pool(p, case["num_pages"], device=dev)
+        bt = case["block_table"].to(dev)
+        k, v = case["k_new"].to(dev), case["v_new"].to(dev)
+        cu, pos0 = case["cu_new"].to(dev), case["pos0_new"].to(dev)
+        for _ in range(3):
+            optr.optr_kv_append(p, k, v, cu, pos0, bt, pool)
+        optr.optr_profile_enable(p, True)
+        t = []
+        for _ in range(max(5, args.steps // 4)):
+            flush()
+            optr.optr_kv_append(p, k, v, cu, pos0, bt, pool)
+            t.append(optr.optr_profile_last(p)["append"])
+        optr.optr_profile_enable(p, False)
+        ms = float(np.mean(t))
+        n_tok = k.shape[0]
+        nb = append_bytes(n_tok, case["h_kv"])
+        res[key] = {
+            "tokens": n_tok, "group": group, "ms": round(ms, 4),
+            "tokens_per_s": round(n_tok / (ms * 1e-3), 1),
+            "gbs": round(nb / (ms * 1e-3) / 1e9, 1),
+            "frac": round(nb / (ms * 1e-3) / 1e9 / hbm_peak, 4)}
+        del pool, k, v, case
+        torch.cuda.empty_cache()
 
     res["decode8k_windows"] = windows_step(args, dev, flush, hbm_peak)
+    torch.cuda.empty_cache()
+    res["decode8k_paper_defaults"] = windows_step(args, dev, flush, hbm_peak,
+                                                  group=128, clip_k=0.96,
+                                                  clip_v=0.92)
     torch.cuda.empty_cache()
 
     for name in ("long128k", "ragged"):
@@ -432,16 +439,19 @@ def extra_workloads(args, dev):
     return res
 
 
-def windows_step(args, dev, flush, hbm_peak, sink=64, recent=256):
+def windows_step(args, dev, flush, hbm_peak, sink=64, recent=256, group=32,
+                 clip_k=1.0, clip_v=1.0):
     """The decode8k step with the paper's BF16 windows (64 sink, 256 recent
-    tokens; Sec. 5): optr_decode_step_win, L2 flushed before every step."""
+    tokens; Sec. 5), optionally with its G = 128 and clip ratios:
+    optr_decode_step_win, L2 flushed before every step."""
     from paper_2608_02691_gb300 import optr, synth
     wl = synth.workload("decode8k", args.seed)
     case = synth.build_case(wl, args.seed, device=dev)
     p = optr.optr_params_create(case["R_k"], case["R_v"], case["mu"],
                                 case["h_q"], decode_variant=args.variant,
                                 append_variant=args.append_variant, sink=sink,
-                                recent=recent)
+                                recent=recent, group=group, clip_k=clip_k,
+                                clip_v=clip_v)
     B, h_q, h_kv = case["B"], case["h_q"], case["h_kv"]
     pool = optr.new_pool(p, case["num_pages"], device=dev)
     win = optr.new_windows(p, B, device=dev)
@@ -492,7 +502,8 @@ def windows_step(args, dev, flush, hbm_peak, sink=64, recent=256):
     wt = sum(window_split(x, sink, recent)[1] for x in lens)
     pb = i2 * h_kv * 96 + wt * h_kv * 512  # what the partial kernel streams
     pm = float(np.mean(part))
-    return {"sink": sink, "recent": recent, "step_ms": round(ms, 4),
+    return {"sink": sink, "recent": recent, "group": group,
+            "clip_k": clip_k, "clip_v": clip_v, "step_ms": round(ms, 4),
             "bytes_per_step": nb, "gbs": round(nb / (ms * 1e-3) / 1e9, 1),
             "partial_ms": round(pm, 4),
             "partial_gbs": round(pb / (pm * 1e-3) / 1e9, 1),

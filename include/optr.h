@@ -20,14 +20,15 @@
  *  - GQA grouping is contiguous: query head j reads KV head j / (h_q / h_kv)
  *    (Sec. 3, "Preliminaries": the set G_h of query heads sharing KV head h).
  *  - Attention logits use the scale 1/sqrt(D) (Sec. 3, Eq. 1).
- *  - Supported shape: head_dim D = 128, group G = 32, page_size P = 16.
- *    Anything else returns OPTR_ERR_UNSUPPORTED.
+ *  - Supported shape: head_dim D = 128, group G = 32 or 128, page_size
+ *    P = 16.  Anything else returns OPTR_ERR_UNSUPPORTED.
  *
  * Quantizer Q2 (Sec. 3.1 "group-wise affine INT2 with clipping ratio c and
  * group size G"; Table "Default experimental settings").  The paper does not
  * write the formula out; this library fixes the following reading.  For one
- * token, one KV head and one group of G = 32 consecutive ROTATED channels
- * z_0..z_31, evaluated in IEEE float32 arithmetic:
+ * token, one KV head and one group of G consecutive ROTATED channels
+ * z_0..z_{G-1} (G = cfg.group: 32, or the paper's 128), evaluated in IEEE
+ * float32 arithmetic:
  *      mn = c * min_i z_i,  mx = c * max_i z_i          (c = clip ratio)
  *      r  = mx - mn
  *      degenerate group (r is not > 1e-30 or r is not finite):
@@ -71,6 +72,9 @@
  *      offset  512: V codes  [16 slots][32 bytes]
  *      offset 1024: K meta   [16 slots][4 groups] {fp16 scale, fp16 min}
  *      offset 1280: V meta   [16 slots][4 groups] {fp16 scale, fp16 min}
+ * The metadata has one {scale, min} entry per 32-channel block; with
+ * G = 128 the group's pair is stored in all four entries (the decode then
+ * reads the same layout for both group sizes).
  * Within a slot's 32 code bytes the groups are interleaved word-major:
  * channel ch = 32*g + 4*w + r  (group g in 0..3, w in 0..7, r in 0..3) is
  * stored in byte 4*w + g, bits [2r, 2r+1].  Byte 4*w + g therefore holds the
@@ -148,7 +152,7 @@ typedef struct {
   int h_q;            /* query heads; a positive multiple of h_kv          */
   int h_kv;           /* KV heads                                          */
   int head_dim;       /* must be 128                                       */
-  int group;          /* must be 32                                        */
+  int group;          /* Q2 group size: 32, or 128 (the paper's default)  */
   int page_size;      /* must be 16                                        */
   float clip_k;       /* key clip ratio c_K in (0, 1]; 1 = min-max          */
   float clip_v;       /* value clip ratio c_V in (0, 1]; 1 = min-max        */
@@ -203,9 +207,10 @@ size_t optr_page_bytes(const optr_params* p);
  *   pool        device bytes [num_pages][h_kv][1536], written in place.
  * Each written slot's codes and metadata are replaced entirely.  Two appends
  * that target the same slot concurrently race.  The tensor-core variant
- * (default for more than 256 new tokens) converts k and v to fp16: values of
- * magnitude 65504 or more set OPTR_DEVERR_FP16_RANGE (use the CUDA-core
- * variant for such inputs).  Out-of-range table entries
+ * (default for more than 256 new tokens with G = 32; G = 128 writes use the
+ * CUDA-core kernels) converts k and v to fp16: values of magnitude 65504 or
+ * more set OPTR_DEVERR_FP16_RANGE (use the CUDA-core variant for such
+ * inputs).  Out-of-range table entries
  * or positions skip that token and set a device error bit.
  */
 optr_status optr_kv_append(const optr_params* p, const void* k, const void* v,

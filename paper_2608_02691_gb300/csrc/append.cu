@@ -26,8 +26,9 @@ append_cuda_core_kernel(const __nv_bfloat16* __restrict__ k,
                         const float* __restrict__ R_k,
                         const float* __restrict__ R_v,
                         const float* __restrict__ muR, float clip_k,
-                        float clip_v, unsigned* err) {
+                        float clip_v, unsigned* err, int group128) {
   __shared__ float xs[2][T][kD];
+  __shared__ float2 grange[2][kGroups];  // G = 128: block ranges of a token
   __shared__ long long dst[T];
   __shared__ int dslot[T];
   const int h = blockIdx.y;
@@ -87,6 +88,15 @@ append_cuda_core_kernel(const __nv_bfloat16* __restrict__ k,
       lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, o));
       hi = fmaxf(hi, __shfl_xor_sync(0xffffffffu, hi, o));
     }
+    if (group128) {  // one range over the four warps (blocks) of this kind
+      if (lane == 0) grange[kind][g] = make_float2(lo, hi);
+      __syncthreads();
+      const float2 r0 = grange[kind][0], r1 = grange[kind][1];
+      const float2 r2 = grange[kind][2], r3 = grange[kind][3];
+      lo = fminf(fminf(r0.x, r1.x), fminf(r2.x, r3.x));
+      hi = fmaxf(fmaxf(r0.y, r1.y), fmaxf(r2.y, r3.y));
+      __syncthreads();  // grange is rewritten for the next token
+    }
     GroupQuant gq = group_quant_params(lo, hi, clip);
     unsigned bits = (unsigned)quant_code(z, gq) << (2 * (lane & 3));
     bits |= __shfl_xor_sync(0xffffffffu, bits, 1);
@@ -116,11 +126,12 @@ append_small_kernel(const __nv_bfloat16* __restrict__ k,
                     const float* __restrict__ R_k,
                     const float* __restrict__ R_v,
                     const float* __restrict__ muR, float clip_k, float clip_v,
-                    unsigned* err, int fold_v) {
+                    unsigned* err, int fold_v, int group128) {
   __shared__ AppendSmallSmemT<T> sm;
   append_small_body<T>(blockIdx.x, blockIdx.y, blockIdx.z, sm, k, v, n_tok,
                     cu_new, pos0, bt, B, max_pages, pool, num_pages, h_kv, R_k,
-                    R_v, muR, clip_k, clip_v, err, fold_v && blockIdx.z == 1);
+                    R_v, muR, clip_k, clip_v, err, fold_v && blockIdx.z == 1,
+                    group128 != 0);
 }
 
 }  // namespace
@@ -132,6 +143,7 @@ cudaError_t launch_append_cuda_core(const optr_params* p,
                                     const int32_t* bt, int B, int max_pages,
                                     uint8_t* pool, int num_pages,
                                     cudaStream_t s) {
+  const int g128 = p->cfg.group == 128 ? 1 : 0;
   // few tokens (decode steps): slice-parallel rotation
   if (n_tok <= 256) {
     const int T = small_tile(n_tok);
@@ -140,18 +152,18 @@ cudaError_t launch_append_cuda_core(const optr_params* p,
       return launch_pdl(append_small_kernel<kSmallTokFew>, grid, dim3(512), 0, s, k, v,
                         n_tok, cu_new, pos0, bt, B, max_pages, pool, num_pages,
                         p->cfg.h_kv, p->R_k, p->R_v, p->muR, p->cfg.clip_k,
-                        p->cfg.clip_v, p->err, p->fold_v);
+                        p->cfg.clip_v, p->err, p->fold_v, g128);
     return launch_pdl(append_small_kernel<kSmallTok>, grid, dim3(512), 0, s, k, v, n_tok,
                       cu_new, pos0, bt, B, max_pages, pool, num_pages,
                       p->cfg.h_kv, p->R_k, p->R_v, p->muR, p->cfg.clip_k,
-                      p->cfg.clip_v, p->err, p->fold_v);
+                      p->cfg.clip_v, p->err, p->fold_v, g128);
   } else {
     constexpr int T = 32;
     dim3 grid((n_tok + T - 1) / T, p->cfg.h_kv);
     return launch_pdl(append_cuda_core_kernel<T>, grid, dim3(256), 0, s, k, v,
                       n_tok, cu_new, pos0, bt, B, max_pages, pool, num_pages,
                       p->cfg.h_kv, p->R_k, p->R_v, p->muR, p->cfg.clip_k,
-                      p->cfg.clip_v, p->err);
+                      p->cfg.clip_v, p->err, g128);
   }
 }
 

@@ -45,9 +45,10 @@ __device__ __forceinline__ void append_small_body(
     int max_pages, uint8_t* __restrict__ pool, int num_pages, int h_kv,
     const float* __restrict__ R_k, const float* __restrict__ R_v,
     const float* __restrict__ muR, float clip_k, float clip_v, unsigned* err,
-    bool identity = false) {
+    bool identity = false, bool group128 = false) {
   // identity: z = x, no rotation (values with the rotation folded into the
-  // model's projections)
+  // model's projections); group128: Q2 groups of all 128 channels (the
+  // pair is stored in each of the four 32-channel metadata entries)
   static_assert(T <= 16, "one quantizing warp per token");
   float (&xs)[T][kD] = sm.xs;
   float (&zp)[4][T][kD] = sm.zp;
@@ -153,18 +154,40 @@ __device__ __forceinline__ void append_small_body(
   const int codes_off = kind ? OPTR_V_CODES_OFFSET : OPTR_K_CODES_OFFSET;
   const int meta_off = kind ? OPTR_V_META_OFFSET : OPTR_K_META_OFFSET;
   uint8_t* chunk = pool + woff;
+  float zv[kGroups];
 #pragma unroll
   for (int g = 0; g < kGroups; ++g) {
     const int jj = 32 * g + lane;
     const float zsum = ((zp[0][warp][jj] + zp[1][warp][jj]) + zp[2][warp][jj]) + zp[3][warp][jj];
-    const float z = __fsub_rn(zsum, musub[g]);
-    float lo = z, hi = z;
+    zv[g] = __fsub_rn(zsum, musub[g]);
+  }
+  // G = 128: one range over the four blocks of 32 channels
+  GroupQuant g128;
+  if (group128) {
+    float lo = fminf(fminf(zv[0], zv[1]), fminf(zv[2], zv[3]));
+    float hi = fmaxf(fmaxf(zv[0], zv[1]), fmaxf(zv[2], zv[3]));
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
       lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, o));
       hi = fmaxf(hi, __shfl_xor_sync(0xffffffffu, hi, o));
     }
-    GroupQuant gq = group_quant_params(lo, hi, clip);
+    g128 = group_quant_params(lo, hi, clip);
+  }
+#pragma unroll
+  for (int g = 0; g < kGroups; ++g) {
+    const float z = zv[g];
+    GroupQuant gq;
+    if (group128) {
+      gq = g128;
+    } else {
+      float lo = z, hi = z;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, o));
+        hi = fmaxf(hi, __shfl_xor_sync(0xffffffffu, hi, o));
+      }
+      gq = group_quant_params(lo, hi, clip);
+    }
     unsigned bits = (unsigned)quant_code(z, gq) << (2 * (lane & 3));
     bits |= __shfl_xor_sync(0xffffffffu, bits, 1);
     bits |= __shfl_xor_sync(0xffffffffu, bits, 2);

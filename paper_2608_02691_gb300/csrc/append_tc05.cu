@@ -91,8 +91,11 @@ struct Smem {
   int cu[kCuCache + 1];
   int p0[kCuCache];
   uint4 xchg[2][kRows][2];               // second-half code words per row
+  // G = 128: each half row's (min, max), per tile group, tile parity, half
+  float2 mmx[2][2][2 * kRows];
   uint64_t full[kStages], empty[kStages], aready[2][2], dready[2], dfree[2];
   uint64_t xready[2], xdone[2];  // the exchange slot of group g written / read
+  uint64_t rready[2];            // G = 128: both halves' ranges of the tile written
   uint32_t tmem;
   int abort;
 };
@@ -185,7 +188,7 @@ __device__ __forceinline__ void minmax32(const float (&x)[32], float& lo, float&
   hi = fmaxf(fmaxf(h[0], h[1]), fmaxf(h[2], h[3]));
 }
 
-template <bool kClamp>
+template <bool kClamp, bool kG128>
 __global__ void __launch_bounds__(kThreads, 1)
 append_tc05_kernel(const __grid_constant__ CUtensorMap tmap_k,
                    const __grid_constant__ CUtensorMap tmap_v, int n_tok,
@@ -228,6 +231,7 @@ append_tc05_kernel(const __grid_constant__ CUtensorMap tmap_k,
       tc05::bar_init(&S.dfree[g], kGroupThreads);
       tc05::bar_init(&S.xready[g], kGroupThreads / 2);
       tc05::bar_init(&S.xdone[g], kGroupThreads / 2);
+      tc05::bar_init(&S.rready[g], kGroupThreads);
     }
     // the 128-byte TMA swizzle wants 1024-byte aligned boxes
     S.abort = (tc05::smem_addr(S.stage[0]) & 1023u) != 0;
@@ -376,41 +380,89 @@ append_tc05_kernel(const __grid_constant__ CUtensorMap tmap_k,
         tc05::tmem_ld32(tD + 32u * G2, acc[0]);
         tc05::tmem_ld32(tD + 32u * (G2 + 1), acc[1]);
         tc05::tmem_wait_ld();
-        tc05::fence_before();
-        tc05::bar_arrive(&S.dfree[g]);  // D[g] read: the next MMA may start
+        if constexpr (!kG128) {
+          tc05::fence_before();
+          tc05::bar_arrive(&S.dfree[g]);  // D[g] read: the next MMA may start
+        }
         uint32_t bytes[2][8];
-#pragma unroll
-        for (int e = 0; e < 2; ++e) {
+        const float xs = kind ? 64.0f : 1.0f;  // x = xs * z
+        // x = z = acc / 64 - mu R (keys; acc / 64 is exact, so one
+        // rounding as fmul + fsub), or x = acc = 64 z (values, mu = 0: the
+        // group's range and codes are then taken in units of z / 64,
+        // exactly)
+        auto row_values = [&](int e, const uint32_t (&a)[32], float (&x)[32]) {
           const int G = G2 + e;
-          // x = z = acc / 64 - mu R (keys; acc / 64 is exact, so one
-          // rounding as fmul + fsub), or x = acc = 64 z (values, mu = 0:
-          // the group's range and codes are then taken in units of z / 64,
-          // exactly)
-          float x[32];
           if (kind == 0) {
             const float4* mu4 = reinterpret_cast<const float4*>(S.mu + 32 * G);
 #pragma unroll
             for (int j4 = 0; j4 < 8; ++j4) {
               const float4 m = mu4[j4];
-              x[4 * j4 + 0] = fmaf(__uint_as_float(acc[e][4 * j4 + 0]), 1.0f / 64.0f, -m.x);
-              x[4 * j4 + 1] = fmaf(__uint_as_float(acc[e][4 * j4 + 1]), 1.0f / 64.0f, -m.y);
-              x[4 * j4 + 2] = fmaf(__uint_as_float(acc[e][4 * j4 + 2]), 1.0f / 64.0f, -m.z);
-              x[4 * j4 + 3] = fmaf(__uint_as_float(acc[e][4 * j4 + 3]), 1.0f / 64.0f, -m.w);
+              x[4 * j4 + 0] = fmaf(__uint_as_float(a[4 * j4 + 0]), 1.0f / 64.0f, -m.x);
+              x[4 * j4 + 1] = fmaf(__uint_as_float(a[4 * j4 + 1]), 1.0f / 64.0f, -m.y);
+              x[4 * j4 + 2] = fmaf(__uint_as_float(a[4 * j4 + 2]), 1.0f / 64.0f, -m.z);
+              x[4 * j4 + 3] = fmaf(__uint_as_float(a[4 * j4 + 3]), 1.0f / 64.0f, -m.w);
             }
           } else {
 #pragma unroll
-            for (int j = 0; j < 32; ++j) x[j] = __uint_as_float(acc[e][j]);
+            for (int j = 0; j < 32; ++j) x[j] = __uint_as_float(a[j]);
           }
-          float lo, hi;
-          minmax32(x, lo, hi);
-          const float xs = kind ? 64.0f : 1.0f;  // x = xs * z
+        };
+        auto scaled_params = [&](float lo, float hi) {
           FastQuant q = fast_quant_params(lo * (1.0f / xs), hi * (1.0f / xs), clip);
           range_err |= q.degenerate && !(fabsf(hi - lo) <= 3.402823466e38f);
           q.mn *= xs;
           q.mx *= xs;
           q.inv4 *= 1.0f / xs;
-          code_bytes<kClamp>(x, q, bytes[e]);
-          meta[e] = q.meta;
+          return q;
+        };
+        if constexpr (kG128) {
+          // one range over the row's 128 channels: this half's two groups,
+          // then the partner half's through shared memory (double-buffered
+          // by tile parity; a buffer is rewritten two tiles later, after
+          // the partner's arrival for the tile in between, i.e. after its
+          // read)
+          // (the accumulator is read again from tensor memory after the
+          // exchange, so no registers hold it meanwhile; D[g] is released
+          // after that second read)
+          float lo, hi;
+          {
+            float x[32], l1, h1;
+            row_values(0, acc[0], x);
+            minmax32(x, lo, hi);
+            row_values(1, acc[1], x);
+            minmax32(x, l1, h1);
+            lo = fminf(lo, l1);
+            hi = fmaxf(hi, h1);
+          }
+          float2* mm = S.mmx[g][k & 1];
+          mm[hp * kRows + row] = make_float2(lo, hi);
+          tc05::bar_arrive(&S.rready[g]);
+          if (!__all_sync(0xffffffffu, tc05::bar_wait(&S.rready[g], k & 1, abort))) break;
+          const float2 o = mm[(1 - hp) * kRows + row];
+          const FastQuant q = scaled_params(fminf(lo, o.x), fmaxf(hi, o.y));
+#pragma unroll
+          for (int e = 0; e < 2; ++e) {
+            uint32_t a2[32];
+            tc05::tmem_ld32(tD + 32u * (G2 + e), a2);
+            tc05::tmem_wait_ld();
+            float x[32];
+            row_values(e, a2, x);
+            code_bytes<kClamp>(x, q, bytes[e]);
+            meta[e] = q.meta;
+          }
+          tc05::fence_before();
+          tc05::bar_arrive(&S.dfree[g]);  // D[g] read: the next MMA may start
+        } else {
+#pragma unroll
+          for (int e = 0; e < 2; ++e) {
+            float x[32];
+            row_values(e, acc[e], x);
+            float lo, hi;
+            minmax32(x, lo, hi);
+            const FastQuant q = scaled_params(lo, hi);
+            code_bytes<kClamp>(x, q, bytes[e]);
+            meta[e] = q.meta;
+          }
         }
         // byte 0 of bytes[0][w] / bytes[1][w] to bytes 2hp, 2hp + 1 of the
         // word (byte 1 of bytes[0][w] is zero)
@@ -496,9 +548,10 @@ cudaError_t launch_append_tc05(const optr_params* p, const __nv_bfloat16* k,
                                const int32_t* bt, int B, int max_pages,
                                uint8_t* pool, int num_pages, cudaStream_t s) {
   const bool clamp = !(p->cfg.clip_k == 1.0f && p->cfg.clip_v == 1.0f);
-  const void* fn = clamp ? reinterpret_cast<const void*>(&append_tc05_kernel<true>)
-                         : reinterpret_cast<const void*>(&append_tc05_kernel<false>);
-  cudaError_t e = ensure_dynamic_smem(fn, sizeof(Smem));
+  const bool g128 = p->cfg.group == 4 * kG;
+  auto fn = clamp ? (g128 ? append_tc05_kernel<true, true> : append_tc05_kernel<true, false>)
+                  : (g128 ? append_tc05_kernel<false, true> : append_tc05_kernel<false, false>);
+  cudaError_t e = ensure_dynamic_smem(reinterpret_cast<const void*>(fn), sizeof(Smem));
   if (e != cudaSuccess) return e;
   const int h_kv = p->cfg.h_kv;
   CUtensorMap mk, mv;
@@ -510,12 +563,7 @@ cudaError_t launch_append_tc05(const optr_params* p, const __nv_bfloat16* k,
   int per = max(1, p->num_sms / (2 * h_kv));
   per = min(per, tiles);
   dim3 grid(per, h_kv, 2);
-  if (clamp)
-    return launch_pdl(append_tc05_kernel<true>, grid, dim3(kThreads), sizeof(Smem), s,
-                      mk, mv, n_tok, cu_new, pos0, bt, B, max_pages, pool, num_pages,
-                      h_kv, (const uint16_t*)p->Rk_t5, (const uint16_t*)p->Rv_t5,
-                      (const float*)p->muR, p->cfg.clip_k, p->cfg.clip_v, p->err);
-  return launch_pdl(append_tc05_kernel<false>, grid, dim3(kThreads), sizeof(Smem), s,
+  return launch_pdl(fn, grid, dim3(kThreads), sizeof(Smem), s,
                     mk, mv, n_tok, cu_new, pos0, bt, B, max_pages, pool, num_pages,
                     h_kv, (const uint16_t*)p->Rk_t5, (const uint16_t*)p->Rv_t5,
                     (const float*)p->muR, p->cfg.clip_k, p->cfg.clip_v, p->err);

@@ -235,7 +235,8 @@ step_prologue_kernel(
     float* __restrict__ koff, float* __restrict__ invs, int* __restrict__ pref,
     int* __restrict__ nzpref, int* __restrict__ cnt_ws, unsigned* err, int fold_v,
     int n_wcp, __nv_bfloat16* __restrict__ win,
-    const int32_t* __restrict__ win_slot, int n_slots, int sink, int recent) {
+    const int32_t* __restrict__ win_slot, int n_slots, int sink, int recent,
+    int group128) {
   extern __shared__ __align__(16) unsigned char dsm_[];
   const int bid = blockIdx.x;
   if (bid < n_app) {
@@ -244,7 +245,7 @@ step_prologue_kernel(
     append_small_body<T>(tblk, hk, kind, *reinterpret_cast<AppendSmallSmemT<T>*>(dsm_),
                       k, v, n_tok, cu_new, pos0, bt, B, max_pages, pool,
                       num_pages, h_kv, R_k, R_v, muR, clip_k, clip_v, err,
-                      fold_v && kind == 1);
+                      fold_v && kind == 1, group128 != 0);
   } else if (bid < n_app + n_wcp) {
     window_copy_body(bid - n_app, *reinterpret_cast<WinCopySmem*>(dsm_), k, v,
                      n_tok, cu_new, pos0, B, win, win_slot, n_slots, h_kv,
@@ -810,7 +811,8 @@ cudaError_t launch_decode(const optr_params* p, int variant,
                    cnt_ws, p->err, p->fold_v, n_wcp,
                    windows ? win->win : (__nv_bfloat16*)nullptr,
                    windows ? win->slot : (const int32_t*)nullptr,
-                   windows ? win->n_slots : 0, sink, recent);
+                   windows ? win->n_slots : 0, sink, recent,
+                   p->cfg.group == 128 ? 1 : 0);
     if (e != cudaSuccess) return e;
     prof_mark(p, 1, s);  // the append stage covers the fused launch,
     prof_mark(p, 2, s);  // the query-rotation stage is empty

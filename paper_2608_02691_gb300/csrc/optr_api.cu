@@ -151,8 +151,8 @@ optr_status optr_params_create(const optr_config* cfg, const float* R_k,
   if (!cfg || !R_k || !mu || !out) return OPTR_ERR_INVALID_ARG;
   if (cfg->h_kv <= 0 || cfg->h_q <= 0 || cfg->h_q % cfg->h_kv != 0)
     return OPTR_ERR_INVALID_ARG;
-  if (cfg->head_dim != kD || cfg->group != kG || cfg->page_size != kPage ||
-      cfg->h_q / cfg->h_kv != 4)
+  if (cfg->head_dim != kD || (cfg->group != kG && cfg->group != 4 * kG) ||
+      cfg->page_size != kPage || cfg->h_q / cfg->h_kv != 4)
     return OPTR_ERR_UNSUPPORTED;
   if (!(cfg->clip_k > 0.f && cfg->clip_k <= 1.f) ||
       !(cfg->clip_v > 0.f && cfg->clip_v <= 1.f))

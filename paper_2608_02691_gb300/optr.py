@@ -153,11 +153,13 @@ def optr_params_create(R_k, R_v, mu, h_q: int, clip_k: float = 1.0,
                        clip_v: float = 1.0,
                        append_variant: int = OPTR_VARIANT_DEFAULT,
                        decode_variant: int = OPTR_VARIANT_DEFAULT,
-                       sink: int = 0, recent: int = 0) -> Params:
+                       sink: int = 0, recent: int = 0,
+                       group: int = 32) -> Params:
     """R_k, R_v float32 [h_kv][128][128] and mu float32 [h_kv][128] (host
     tensors); the library copies them to the current CUDA device.  R_v may be
     None: the value rotation is folded into the model's W_V / W_O.  sink /
-    recent > 0 keep BF16 windows (the *_win calls)."""
+    recent > 0 keep BF16 windows (the *_win calls); group is the Q2 group
+    size (32, or the paper's 128)."""
     R_k = R_k.detach().to("cpu", torch.float32).contiguous()
     if R_v is not None:
         R_v = R_v.detach().to("cpu", torch.float32).contiguous()
@@ -166,7 +168,7 @@ def optr_params_create(R_k, R_v, mu, h_q: int, clip_k: float = 1.0,
     if R_k.shape != (h_kv, 128, 128) or (R_v is not None and R_v.shape != R_k.shape) or \
             mu.shape != (h_kv, 128):
         raise ValueError("R_k, R_v must be [h_kv][128][128], mu [h_kv][128]")
-    cfg = optr_config(h_q, h_kv, 128, 32, 16, clip_k, clip_v, append_variant,
+    cfg = optr_config(h_q, h_kv, 128, group, 16, clip_k, clip_v, append_variant,
                       decode_variant, sink, recent)
     h = ctypes.c_void_p()
     _check(lib().optr_params_create(ctypes.byref(cfg), _ptr(R_k),

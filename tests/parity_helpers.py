@@ -154,7 +154,7 @@ def flipped_groups(case, stats_ctx, stats_new):
     return out
 
 
-def oracle_case(case, pool_init=None):
+def oracle_case(case, pool_init=None, group=32, clip_k=1.0, clip_v=1.0):
     """Oracle append of context and new tokens; returns (pool, u_ctx, u_new)."""
     pool = (np.zeros((case["num_pages"], case["h_kv"], 1536), np.uint8)
             if pool_init is None else pool_init.copy())
@@ -166,13 +166,15 @@ def oracle_case(case, pool_init=None):
                                  synth.bf16_bits(case["v_ctx"]),
                                  case["cu_ctx"].numpy(),
                                  case["pos0_ctx"].numpy(), bt, pool, *args,
-                                 want_u=True)
+                                 want_u=True, group=group, clip_k=clip_k,
+                                 clip_v=clip_v)
     if case["k_new"].shape[0]:
         u_new = oracle.kv_append(synth.bf16_bits(case["k_new"]),
                                  synth.bf16_bits(case["v_new"]),
                                  case["cu_new"].numpy(),
                                  case["pos0_new"].numpy(), bt, pool, *args,
-                                 want_u=True)
+                                 want_u=True, group=group, clip_k=clip_k,
+                                 clip_v=clip_v)
     return pool, u_ctx, u_new
 
 

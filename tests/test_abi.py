@@ -56,7 +56,7 @@ def test_host_argument_errors_launch_nothing(lib):
     assert lib.optr_params_create(ctypes.byref(cfg), None, f, f, ctypes.byref(h)) == -1
     assert lib.optr_params_create(None, f, f, f, ctypes.byref(h)) == -1
     # unsupported shapes: head_dim, group, page size, GQA ratio
-    for bad in (dict(head_dim=64), dict(group=128), dict(page_size=8),
+    for bad in (dict(head_dim=64), dict(group=64), dict(page_size=8),
                 dict(h_q=16)):
         c = optr.optr_config(32, 8, 128, 32, 16, 1.0, 1.0, 0, 0)
         for k, val in bad.items():
@@ -64,6 +64,11 @@ def test_host_argument_errors_launch_nothing(lib):
         assert lib.optr_params_create(ctypes.byref(c), f, f, f, ctypes.byref(h)) == -2
     c = optr.optr_config(32, 8, 128, 32, 16, 0.0, 1.0, 0, 0)
     assert lib.optr_params_create(ctypes.byref(c), f, f, f, ctypes.byref(h)) == -1
+    # BF16 windows: sink a multiple of 16, both windows at most 1024
+    for sink, recent, want in ((8, 0, -1), (-16, 0, -1), (0, -1, -1),
+                               (1040, 0, -3), (0, 1025, -3)):
+        c = optr.optr_config(32, 8, 128, 32, 16, 1.0, 1.0, 0, 0, sink, recent)
+        assert lib.optr_params_create(ctypes.byref(c), f, f, f, ctypes.byref(h)) == want
     assert not h.value
     # operations on a null handle
     assert lib.optr_kv_append(None, None, None, 1, None, None, None, 1, 1,

@@ -1,0 +1,138 @@
+"""The paper's default quantizer settings on the GPU (Sec. 5 and the
+default-settings table: group size G = 128, clipping ratios 0.96 for keys
+and 0.92 for values; with its 64 sink and 256 recent BF16 tokens), against
+the oracle:
+
+* cache write with G = 128 on every write path (single-token tiles of the
+  decode step, the CUDA-core kernel for larger writes, which G = 128 writes
+  use under every variant), codes and metadata as without;
+* decode over oracle-written G = 128 pools, both decode variants;
+* the whole paper-default configuration (G = 128, clips, windows) through
+  the fused decode step.
+"""
+import numpy as np
+import pytest
+import torch
+
+from oracle import oracle
+from paper_2608_02691_gb300 import optr, synth
+
+import parity_helpers as ph
+
+pytestmark = pytest.mark.gpu
+
+VARIANTS = [optr.OPTR_VARIANT_CUDA_CORE, optr.OPTR_VARIANT_TENSOR]
+CASES = [("tiny", 1.0), ("decode8k", 1 / 16), ("ragged", 1 / 32),
+         ("prefill", 1 / 128)]
+CK, CV = 0.96, 0.92
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _setup():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2608_02691_gb300 import build
+    build.build()
+    oracle.build()
+    oracle.set_threads(max(1, min(16, __import__("os").cpu_count() or 1)))
+    torch.cuda.set_device(0)
+
+
+_cache = {}
+
+
+def _case(name, scale):
+    if (name, scale) not in _cache:
+        c = synth.build_case(synth.workload(name, 0, scale), 0)
+        _cache[(name, scale)] = (c, *ph.oracle_case(c, group=128, clip_k=CK, clip_v=CV))
+    return _cache[(name, scale)]
+
+
+@pytest.mark.parametrize("name,scale", CASES)
+@pytest.mark.parametrize("avar", VARIANTS)
+def test_group128_cache_write(name, scale, avar):
+    c, pool_ref, u_ctx, u_new = _case(name, scale)
+    p = optr.optr_params_create(c["R_k"], c["R_v"], c["mu"], c["h_q"],
+                                clip_k=CK, clip_v=CV, append_variant=avar,
+                                group=128)
+    pool = optr.new_pool(p, c["num_pages"])
+    bt = c["block_table"].cuda()
+    for kk, vv, cu, pos0 in ((c["k_ctx"], c["v_ctx"], c["cu_ctx"], c["pos0_ctx"]),
+                             (c["k_new"], c["v_new"], c["cu_new"], c["pos0_new"])):
+        if kk.shape[0]:
+            optr.optr_kv_append(p, kk.cuda(), vv.cuda(), cu.cuda(), pos0.cuda(),
+                                bt, pool)
+    torch.cuda.synchronize()
+    assert optr.optr_device_error(p) == 0
+    pg = pool.cpu().numpy()
+    for cu, pos0, u in ((c["cu_ctx"], c["pos0_ctx"], u_ctx),
+                        (c["cu_new"], c["pos0_new"], u_new)):
+        if u is None:
+            continue
+        pages, slots = ph.token_slots(cu, pos0, c["block_table"])
+        st = ph.compare_append(pg, pool_ref, u, pages, slots)
+        # one (scale, min) pair per token and kind, in all four entries
+        for kind in (0, 1):
+            _, sc, mn = ph.slot_codes(pg, pages, slots, kind)
+            assert np.all(sc == sc[..., :1]) and np.all(mn == mn[..., :1])
+
+
+@pytest.mark.parametrize("name,scale", CASES[:3])
+@pytest.mark.parametrize("dvar", VARIANTS)
+def test_group128_decode(name, scale, dvar):
+    c, pool_ref, _, _ = _case(name, scale)
+    got = ph.gpu_decode(c, pool_ref, variant=dvar)
+    ref = ph.oracle_decode(c, pool_ref)
+    ph.assert_decode_close(got, ref, f"{name} G=128")
+
+
+@pytest.mark.parametrize("dvar", VARIANTS)
+def test_paper_default_configuration_step(dvar):
+    """G = 128, c_K = 0.96, c_V = 0.92, 64 sink and 256 recent BF16 tokens:
+    context written, then the fused step (new token, decode)."""
+    sink, recent = 64, 256
+    c, pool_ref, u_ctx, u_new = _case("decode8k", 1 / 16)
+    B = c["B"]
+    slots = np.arange(B, dtype=np.int32)
+    win_ref = oracle.new_windows(B, c["h_kv"], sink, recent)
+    for kk, vv, cu, pos0 in ((c["k_ctx"], c["v_ctx"], c["cu_ctx"], c["pos0_ctx"]),
+                             (c["k_new"], c["v_new"], c["cu_new"], c["pos0_new"])):
+        oracle.window_write(synth.bf16_bits(kk), synth.bf16_bits(vv), cu.numpy(),
+                            pos0.numpy(), win_ref, slots, sink, recent)
+    p = optr.optr_params_create(c["R_k"], c["R_v"], c["mu"], c["h_q"],
+                                clip_k=CK, clip_v=CV, decode_variant=dvar,
+                                sink=sink, recent=recent, group=128)
+    pool = optr.new_pool(p, c["num_pages"])
+    win = optr.new_windows(p, B)
+    ws_slot = torch.from_numpy(slots).cuda()
+    bt = c["block_table"].cuda()
+    optr.optr_kv_append_win(p, c["k_ctx"].cuda(), c["v_ctx"].cuda(),
+                            c["cu_ctx"].cuda(), c["pos0_ctx"].cuda(), bt, pool,
+                            win, ws_slot)
+    out = torch.empty(B, c["h_q"], 128, dtype=torch.float32, device="cuda")
+    ws = optr.new_workspace(p, B, bt.shape[1])
+    optr.optr_decode_step_win(p, c["q"].cuda(), c["k_new"].cuda(),
+                              c["v_new"].cuda(), c["cu_new"].cuda(),
+                              c["pos0_new"].cuda(), bt, c["seq_lens"].cuda(),
+                              pool, win, ws_slot, out, ws)
+    torch.cuda.synchronize()
+    assert optr.optr_device_error(p) == 0
+    assert np.array_equal(win.cpu().view(torch.int16).numpy().view(np.uint16), win_ref)
+    pg = pool.cpu().numpy()
+    sts = []
+    for cu, pos0, u in ((c["cu_ctx"], c["pos0_ctx"], u_ctx),
+                        (c["cu_new"], c["pos0_new"], u_new)):
+        pages, sl = ph.token_slots(cu, pos0, c["block_table"])
+        sts.append(ph.compare_append(pg, pool_ref, u, pages, sl))
+    skip = ph.flipped_groups(c, *sts)
+    ref = oracle.decode_attention(
+        synth.bf16_bits(c["q"]), c["block_table"].numpy(), c["seq_lens"].numpy(),
+        pool_ref, c["R_k"].numpy(), c["R_v"].numpy(), c["h_kv"], win=win_ref,
+        win_slot=slots, sink=sink, recent=recent, mu=c["mu"].numpy())
+    got = out.cpu().double().numpy()
+    keep = np.ones(got.shape[:2], bool)
+    for b, h in skip:
+        keep[b, 4 * h:4 * h + 4] = False
+    assert keep.any()
+    ph.assert_decode_close(got[keep], ref[keep], "paper defaults")
+    assert np.all(np.isfinite(got))
