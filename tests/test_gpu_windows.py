@@ -307,3 +307,78 @@ def test_plain_entry_points_reject_windows():
         optr.optr_kv_append(p, c["k_ctx"].cuda(), c["v_ctx"].cuda(),
                             c["cu_ctx"].cuda(), c["pos0_ctx"].cuda(),
                             c["block_table"].cuda(), pool)
+
+
+def test_window_step_replays_from_a_cuda_graph():
+    """The windowed decode step (window copy CTAs in the prologue launch,
+    window warps in the partial kernel, window merge in the combine)
+    captured once in a CUDA graph and replayed gives the bytes and output of
+    a direct call."""
+    sink, recent = 64, 256
+    c, _, _, _, win_ref, slots = _case("decode8k", 1 / 16, sink, recent)
+    dev = "cuda"
+    res = []
+    for use_graph in (False, True):
+        p = optr.optr_params_create(c["R_k"], c["R_v"], c["mu"], c["h_q"],
+                                    sink=sink, recent=recent)
+        pool = optr.new_pool(p, c["num_pages"], device=dev)
+        win = optr.new_windows(p, win_ref.shape[0], device=dev)
+        ws_slot = torch.from_numpy(slots).to(dev)
+        bt = c["block_table"].to(dev)
+        optr.optr_kv_append_win(p, c["k_ctx"].to(dev), c["v_ctx"].to(dev),
+                                c["cu_ctx"].to(dev), c["pos0_ctx"].to(dev), bt,
+                                pool, win, ws_slot)
+        args = [c["q"].to(dev), c["k_new"].to(dev), c["v_new"].to(dev),
+                c["cu_new"].to(dev), c["pos0_new"].to(dev), bt,
+                c["seq_lens"].to(dev), pool, win, ws_slot]
+        out = torch.empty(c["B"], c["h_q"], 128, dtype=torch.float32, device=dev)
+        ws = optr.new_workspace(p, c["B"], bt.shape[1], device=dev)
+        torch.cuda.synchronize()
+        if use_graph:
+            s = torch.cuda.Stream()
+            s.wait_stream(torch.cuda.current_stream())
+            with torch.cuda.stream(s):  # warm-up outside the capture
+                optr.optr_decode_step_win(p, *args, out, ws)
+            torch.cuda.current_stream().wait_stream(s)
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g):
+                optr.optr_decode_step_win(p, *args, out, ws)
+            out.zero_()
+            g.replay()
+        else:
+            optr.optr_decode_step_win(p, *args, out, ws)
+            optr.optr_decode_step_win(p, *args, out, ws)
+        torch.cuda.synchronize()
+        assert optr.optr_device_error(p) == 0
+        res.append((pool.cpu(), win.cpu(), out.cpu()))
+    for a, b in zip(*res):
+        assert torch.equal(a, b)
+
+
+def test_long_write_copies_only_window_rows():
+    """A write of several thousand tokens per sequence in one call (the
+    prefill case: tiles of 256 tokens with few window rows each) fills the
+    store exactly as the oracle's rule."""
+    sink, recent = 64, 256
+    lens = [3000, 64, 700, 1, 2500]
+    B, h_kv = len(lens), 8
+    k, v = synth.kv_tokens(sum(lens), h_kv, "t4", 5, 0)
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    pos0 = np.array([0, 10, 300, 5000, 40], np.int32)
+    slots = np.array([4, 0, 3, 1, 2], np.int32)
+    win_ref = oracle.new_windows(B, h_kv, sink, recent)
+    oracle.window_write(synth.bf16_bits(k), synth.bf16_bits(v), cu, pos0,
+                        win_ref, slots, sink, recent)
+    R_k, R_v = synth.rotations(h_kv, 5)
+    p = optr.optr_params_create(R_k, R_v, synth.key_mean(k), 32, sink=sink,
+                                recent=recent)
+    total = [int(a) + int(b) for a, b in zip(pos0, lens)]
+    bt, num_pages = synth.page_tables(total, True, 5)
+    pool = optr.new_pool(p, num_pages)
+    win = optr.new_windows(p, B)
+    optr.optr_kv_append_win(p, k.cuda(), v.cuda(), torch.from_numpy(cu).cuda(),
+                            torch.from_numpy(pos0).cuda(), bt.cuda(), pool, win,
+                            torch.from_numpy(slots).cuda())
+    torch.cuda.synchronize()
+    assert optr.optr_device_error(p) == 0
+    np.testing.assert_array_equal(_win_bits(win), win_ref)
