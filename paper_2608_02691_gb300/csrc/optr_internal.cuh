@@ -102,7 +102,7 @@ struct DecodePlan {
   int B, h_q, h_kv, max_pages, W;  // W = partial-kernel warps
   int S;                           // combine CTAs per (sequence, KV head)
   int Uw;   // BF16-window units (16 window tokens) per (sequence, KV head)
-  int Ww;   // warps that take window units: min(W, B * h_kv * Uw)
+  int Ww;   // window warps (tensor kernel: 4 per SM; CUDA-core: all W), at most B * h_kv * Uw
   size_t off_qf, off_qs, off_frag, off_koff, off_invs, off_pref, off_cnt,
       off_part, off_cpart, off_wpart, total;
 };
