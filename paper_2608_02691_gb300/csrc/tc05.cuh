@@ -32,11 +32,6 @@ __host__ __device__ constexpr uint32_t idesc_f16(int M, int N) {
   return (1u << 4) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
 }
 
-// As idesc_f16 with A and B bf16 (type 1 in bits [7,10) and [10,13)).
-__host__ __device__ constexpr uint32_t idesc_bf16(int M, int N) {
-  return idesc_f16(M, N) | (1u << 7) | (1u << 10);
-}
-
 __device__ __forceinline__ void bar_init(uint64_t* bar, uint32_t count) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_addr(bar)),
                "r"(count));
