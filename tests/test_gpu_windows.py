@@ -21,7 +21,10 @@ import parity_helpers as ph
 pytestmark = pytest.mark.gpu
 
 VARIANTS = [optr.OPTR_VARIANT_CUDA_CORE, optr.OPTR_VARIANT_TENSOR]
-CASES = [("tiny", 1.0), ("decode8k", 1 / 16), ("ragged", 1 / 32)]
+# long128k: one sequence, so the combine splits each (sequence, KV head)
+# over several CTAs (the last one merges the window partials)
+CASES = [("tiny", 1.0), ("decode8k", 1 / 16), ("ragged", 1 / 32),
+         ("long128k", 1 / 32)]
 WINDOWS = [(64, 256), (16, 32), (0, 48), (32, 0)]
 
 
@@ -296,6 +299,44 @@ def test_window_slot_out_of_range_is_flagged():
     keep = np.arange(c["B"]) != 3
     ph.assert_decode_close(got[keep], ref[keep], "other sequences")
     assert np.all(np.isfinite(got))
+
+
+@pytest.mark.parametrize("dvar", VARIANTS)
+def test_window_decode_many_sequences(dvar):
+    """300 sequences (more than the partial kernel caches page prefix sums
+    for, so it reads them after waiting), lengths from 1 to 700."""
+    sink, recent = 64, 256
+    g = np.random.default_rng(13)
+    lens = g.integers(1, 700, size=300).tolist()
+    B, h_kv, h_q = len(lens), 8, 32
+    k, v = synth.kv_tokens(sum(lens), h_kv, "t4", 13, 0)
+    mu = synth.key_mean(k)
+    R_k, R_v = synth.rotations(h_kv, 13)
+    q = synth.queries(B, h_q, 13)
+    cu = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    bt, num_pages = synth.page_tables(lens, True, 13)
+    pool_ref = np.zeros((num_pages, h_kv, 1536), np.uint8)
+    oracle.kv_append(synth.bf16_bits(k), synth.bf16_bits(v), cu,
+                     np.zeros(B, np.int32), bt.numpy(), pool_ref, R_k.numpy(),
+                     R_v.numpy(), mu.numpy())
+    slots = g.permutation(B + 7)[:B].astype(np.int32)
+    win_ref = oracle.new_windows(B + 7, h_kv, sink, recent)
+    oracle.window_write(synth.bf16_bits(k), synth.bf16_bits(v), cu,
+                        np.zeros(B, np.int32), win_ref, slots, sink, recent)
+    c = dict(q=q, block_table=bt, seq_lens=torch.tensor(lens, dtype=torch.int32),
+             R_k=R_k, R_v=R_v, mu=mu, h_kv=h_kv)
+    ref = _oracle_decode(c, pool_ref, win_ref, slots, sink, recent)
+    p = optr.optr_params_create(R_k, R_v, mu, h_q, decode_variant=dvar,
+                                sink=sink, recent=recent)
+    out = torch.full((B, h_q, 128), 7.0, dtype=torch.float32, device="cuda")
+    ws = optr.new_workspace(p, B, bt.shape[1], device="cuda")
+    optr.optr_decode_attention_win(p, q.cuda(), bt.cuda(), c["seq_lens"].cuda(),
+                                   torch.from_numpy(pool_ref).cuda(),
+                                   _win_tensor(win_ref),
+                                   torch.from_numpy(slots).cuda(), out, ws)
+    torch.cuda.synchronize()
+    assert optr.optr_device_error(p) == 0
+    ph.assert_decode_close(out.cpu().double().numpy(), ref, "300 sequences")
 
 
 def test_plain_entry_points_reject_windows():
