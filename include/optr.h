@@ -219,8 +219,10 @@ optr_status optr_kv_append(const optr_params* p, const void* k, const void* v,
                            int B, int max_pages, uint8_t* pool, int num_pages,
                            cudaStream_t stream);
 
-/* Workspace bytes optr_decode_attention needs for this batch shape on the
- * current device (split-K partials and the rotated queries). */
+/* Workspace bytes optr_decode_attention (and _win, optr_decode_step and
+ * _win) needs for this batch shape on the current device: split-K
+ * partials, the rotated queries and, when p has BF16 windows, the window
+ * partials. */
 size_t optr_decode_workspace_size(const optr_params* p, int B, int max_pages);
 
 /*
