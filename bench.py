@@ -669,7 +669,9 @@ def main():
 
     res = run_ours(args, rank, world, dev)
     m = res["main"]
-    extra = extra_workloads(args, dev) if (rank == 0 and not args.no_extra) else None
+    # the other workloads only at N = 1 (a multi-GPU run holds every GPU)
+    extra = (extra_workloads(args, dev)
+             if (rank == 0 and world == 1 and not args.no_extra) else None)
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu:
         case_cpu = {k: (v.cpu() if torch.is_tensor(v) else v)
