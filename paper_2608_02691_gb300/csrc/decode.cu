@@ -258,7 +258,7 @@ step_prologue_kernel(
   }
 }
 
-// Window part of a separate cache write (512 threads per 256 new tokens).
+// Window part of a separate cache write (512 threads per 16 new tokens).
 __global__ void __launch_bounds__(512)
 window_copy_kernel(const __nv_bfloat16* __restrict__ k,
                    const __nv_bfloat16* __restrict__ v, int n_tok,

@@ -15,21 +15,18 @@ namespace optr {
 
 // ------------------------------------------------------------ cache write
 
-constexpr int kWinCopyTok = 256;  // tokens per copy CTA (512 threads)
+constexpr int kWinCopyTok = 16;  // tokens per copy CTA (512 threads)
 
 struct WinCopySmem {
-  long long base[kWinCopyTok];  // store offset (elements) of a copied row in
-                                // plane (head 0, keys)
-  int tok[kWinCopyTok];         // its token
-  int cnt;                      // rows to copy
+  long long base[kWinCopyTok];  // store offset (elements) of the token's row
+                                // in plane (head 0, keys), or -1
 };
 
-// CTA `tile` looks at new tokens [256 tile, 256 tile + 256): token t of
-// sequence b (rows cu_new[b] .. cu_new[b+1]-1, positions from pos0[b], end =
-// pos0[b] + count) is a window position of the written cache when s < sink
-// or, with recent > 0, s >= end - recent; its K and V rows of every KV head
-// go to row win_row(s) of slot win_slot[b].  The window tokens of the tile
-// are listed first (most tokens of a long write are not), then copied.
+// CTA `tile` copies new tokens [16 tile, 16 tile + 16): token t of sequence
+// b (rows cu_new[b] .. cu_new[b+1]-1, positions from pos0[b], end = pos0[b]
+// + count) is a window position of the written cache when s < sink or, with
+// recent > 0, s >= end - recent; its K and V rows of every KV head go to
+// row win_row(s) of slot win_slot[b].
 __device__ __forceinline__ void window_copy_body(
     int tile, WinCopySmem& sm, const __nv_bfloat16* __restrict__ k,
     const __nv_bfloat16* __restrict__ v, int n_tok,
@@ -38,12 +35,11 @@ __device__ __forceinline__ void window_copy_body(
     int n_slots, int h_kv, int sink, int recent, unsigned* err) {
   const int tid = threadIdx.x;
   const int rows = sink + recent;
-  if (tid == 0) sm.cnt = 0;
   pdl_wait();  // inputs may come from earlier kernels
   pdl_trigger();
-  __syncthreads();
   if (tid < kWinCopyTok) {
     const int tok = tile * kWinCopyTok + tid;
+    long long base = -1;
     if (tok < n_tok) {
       int lo = 0, hi = B;  // largest b with cu_new[b] <= tok
       while (hi - lo > 1) {
@@ -61,25 +57,25 @@ __device__ __forceinline__ void window_copy_body(
           } else {
             // row in [0, sink + recent), in 64 bits for any int32 pos0
             const long long row = s < sink ? s : sink + (s - sink) % recent;
-            const int i = atomicAdd(&sm.cnt, 1);
-            sm.base[i] = (long long)slot * h_kv * 2 * rows * kD + row * kD;
-            sm.tok[i] = tok;
+            base = (long long)slot * h_kv * 2 * rows * kD + row * kD;
           }
         }
       }
     }
+    sm.base[tid] = base;
   }
   __syncthreads();
-  // 16-byte pieces: listed row tt, KV head hh, kind, piece c of the row
+  // 16-byte pieces: token tt, KV head hh, kind, piece c of the 256-byte row
   const int per_tok = 2 * h_kv * (kD / 8);
-  const int n = sm.cnt;
-  for (int idx = tid; idx < n * per_tok; idx += blockDim.x) {
+  for (int idx = tid; idx < kWinCopyTok * per_tok; idx += blockDim.x) {
     const int tt = idx / per_tok, r = idx - tt * per_tok;
+    const long long base = sm.base[tt];
+    if (base < 0) continue;
     const int kind = r / (h_kv * (kD / 8));
     const int hh = (r / (kD / 8)) % h_kv, c = r % (kD / 8);
-    const int tok = sm.tok[tt];
+    const int tok = tile * kWinCopyTok + tt;
     const __nv_bfloat16* src = (kind ? v : k) + ((size_t)tok * h_kv + hh) * kD + 8 * c;
-    __nv_bfloat16* dst = win + sm.base[tt] + (long long)(hh * 2 + kind) * rows * kD + 8 * c;
+    __nv_bfloat16* dst = win + base + (long long)(hh * 2 + kind) * rows * kD + 8 * c;
     *reinterpret_cast<uint4*>(dst) = __ldg(reinterpret_cast<const uint4*>(src));
   }
 }
