@@ -79,11 +79,48 @@ def test_host_argument_errors_launch_nothing(lib):
                                 None, 1, 1, None, 1, None, None, 0, None) == -1
     assert lib.optr_decode_workspace_size(None, 1, 1) == 0
     assert lib.optr_page_bytes(None) == 0
+    # the BF16-window entry points
+    assert lib.optr_window_bytes(None, 4) == 0
+    assert lib.optr_kv_append_win(None, None, None, 1, None, None, None, 1, 1,
+                                  None, 1, None, None, 0, None) == -1
+    assert lib.optr_decode_attention_win(None, None, None, None, 1, 1, None, 1,
+                                         None, None, 0, None, None, 0,
+                                         None) == -1
+    assert lib.optr_decode_step_win(None, None, None, None, 0, None, None, None,
+                                    None, 1, 1, None, 1, None, None, 0, None,
+                                    None, 0, None) == -1
     flags = ctypes.c_uint32()
     assert lib.optr_device_error(None, ctypes.byref(flags)) == -1
 
 
 # ---------------------------------------------------------- split-K plan
+
+def test_window_unit_partition_gives_each_window_warp_work():
+    """BF16-window units: Ww = min(window warps, units), contiguous ranges;
+    every window warp owns at least one unit, and the warps owning a
+    sequence's non-empty units form a gap-free run whose closed-form ends
+    (the combine's) are the first and last owner."""
+    import random
+    rng = random.Random(3)
+    for _ in range(300):
+        B, h_kv, Uw = rng.randint(1, 40), rng.choice([1, 8]), rng.choice([1, 4, 20])
+        U = B * h_kv * Uw
+        Ww = min(rng.choice([7, 64, 608]), U)
+        owner = {}
+        for w in range(Ww):
+            u0, u1 = w * U // Ww, (w + 1) * U // Ww
+            assert u1 > u0
+            for u in range(u0, u1):
+                owner[u] = w
+        for bh in range(B * h_kv):
+            nwu = rng.randint(0, Uw)
+            if nwu == 0:
+                continue
+            ws = [owner[bh * Uw + j] for j in range(nwu)]
+            assert ws == sorted(ws) and set(ws) == set(range(ws[0], ws[-1] + 1))
+            assert _warp_of(bh * Uw, U, Ww) == ws[0]
+            assert _warp_of(bh * Uw + nwu - 1, U, Ww) == ws[-1]
+
 
 def _ranges(F, W):
     return [(w * F // W, (w + 1) * F // W) for w in range(W)]
