@@ -364,8 +364,8 @@ def extra_workloads(args, dev):
     hbm_peak, _ = peaks()
     flush = Flusher(dev)
     res = {}
-    # prefill append: 4 x 32768 tokens (G = 32 on the tcgen05 cache write;
-    # G = 128, the paper's default, on the CUDA-core one)
+    # prefill append: 4 x 32768 tokens, G = 32 and the paper's G = 128, both
+    # on the tcgen05 cache write
     for key, group in (("prefill_append", 32), ("prefill_append_g128", 128)):
         wl = synth.workload("prefill", args.seed)
         case = synth.build_case(wl, args.seed, device=dev)

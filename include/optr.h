@@ -207,10 +207,10 @@ size_t optr_page_bytes(const optr_params* p);
  *   pool        device bytes [num_pages][h_kv][1536], written in place.
  * Each written slot's codes and metadata are replaced entirely.  Two appends
  * that target the same slot concurrently race.  The tensor-core variant
- * (default for more than 256 new tokens with G = 32; G = 128 writes use the
- * CUDA-core kernels) converts k and v to fp16: values of magnitude 65504 or
- * more set OPTR_DEVERR_FP16_RANGE (use the CUDA-core variant for such
- * inputs).  Out-of-range table entries
+ * (the default for more than 256 new tokens, with either group size)
+ * converts k and v to fp16: values of magnitude 65504 or more set
+ * OPTR_DEVERR_FP16_RANGE and leave their token's record unspecified (use
+ * the CUDA-core variant for such inputs).  Out-of-range table entries
  * or positions skip that token and set a device error bit.
  */
 optr_status optr_kv_append(const optr_params* p, const void* k, const void* v,
@@ -298,17 +298,22 @@ optr_status optr_profile_last(const optr_params* p, float ms[4]);
  * the device and can fail under memory pressure).
  *
  * Same arguments, result and errors as optr_decode_attention, minus the
- * workspace.  The scratch memory is a fixed array of
- * OPTR_NOALLOC_SCRATCH_BYTES (16 MiB) in the library's device image; every
- * GPU that loads the library holds it until the process exits.  A batch
- * whose workspace would exceed it (optr_decode_workspace_size(p, B,
- * max_pages) > OPTR_NOALLOC_SCRATCH_BYTES; about B > 230 at 8 KV heads on a
- * 152-SM GPU) is rejected with OPTR_ERR_WORKSPACE before any launch.
+ * workspace: the same argument and range checks run first, in the same
+ * order; params with BF16 windows (cfg.sink or cfg.recent > 0) are refused
+ * with OPTR_ERR_INVALID_ARG, as optr_decode_attention refuses them (there
+ * is no windowed variant of this call).  The scratch memory is a fixed
+ * array of OPTR_NOALLOC_SCRATCH_BYTES (16 MiB) in the library's device
+ * image; every GPU that loads the library holds it until the process
+ * exits.  A batch whose workspace would exceed it
+ * (optr_decode_workspace_size(p, B, max_pages) > OPTR_NOALLOC_SCRATCH_BYTES;
+ * about B > 230 at 8 KV heads on a 152-SM GPU) is rejected with
+ * OPTR_ERR_WORKSPACE before any launch.
  *
- * The first call on each device looks up the array's device address with
- * that device current (cudaGetSymbolAddress); make that first call before
- * any stream capture.  Nothing in the scratch needs to start at zero.  All
- * calls on a device share the one array, so calls that overlap on the GPU
+ * optr_params_create looks up the array's device address on its device
+ * (with that device current) and keeps it in the params, so this call does
+ * no set-up of its own; params created after a cudaDeviceReset carry the
+ * new address.  Nothing in the scratch needs to start at zero.  All calls
+ * on a device share the one array, so calls that overlap on the GPU
  * (different streams, or different threads without ordering) race and
  * corrupt each other's results; serialise them.  This call allocates
  * nothing and never calls cudaMalloc or cudaFree.
@@ -321,7 +326,6 @@ optr_status optr_decode_attention_noalloc(const optr_params* p, const void* q,
                                           int num_pages, float* out,
                                           cudaStream_t stream);
 
-/* Static description of a status code. */
 /*
  * BF16 windows (Sec. 3.1, opening paragraph: the long history is INT2 while
  * a small BF16 window is kept; Sec. 4.1: sink and recent tokens stay in
@@ -384,6 +388,7 @@ optr_status optr_decode_step_win(const optr_params* p, const void* q,
                                  float* out, void* workspace, size_t ws_bytes,
                                  cudaStream_t stream);
 
+/* Static description of a status code. */
 const char* optr_strerror(optr_status s);
 
 #ifdef __cplusplus

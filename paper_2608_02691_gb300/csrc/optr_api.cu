@@ -130,6 +130,29 @@ DecodePlan decode_plan(const optr_params* p, int B, int max_pages) {
 
 }  // namespace optr
 
+namespace optr {
+
+optr_status decode_args_status(const optr_params* p, const void* q,
+                               const int32_t* block_table,
+                               const int32_t* seq_lens, int B, int max_pages,
+                               const uint8_t* pool, int num_pages,
+                               const float* out) {
+  if (!p || B <= 0 || max_pages <= 0 || num_pages <= 0)
+    return OPTR_ERR_INVALID_ARG;
+  if (!q || !block_table || !seq_lens || !pool || !out)
+    return OPTR_ERR_INVALID_ARG;
+  if (!aligned(pool, 16) || !aligned(q, 16) || !aligned(out, 16))
+    return OPTR_ERR_INVALID_ARG;
+  if ((long long)max_pages * kPage > (1LL << 30) || B > (1 << 24))
+    return OPTR_ERR_OUT_OF_RANGE;
+  // the split-K plan indexes (sequence, KV head, page) units with 32 bits
+  if ((long long)B * max_pages * p->cfg.h_kv >= (1LL << 31))
+    return OPTR_ERR_OUT_OF_RANGE;
+  return OPTR_OK;
+}
+
+}  // namespace optr
+
 extern "C" {
 
 const char* optr_strerror(optr_status s) {
@@ -235,6 +258,7 @@ optr_status optr_params_create(const optr_config* cfg, const float* R_k,
   if (e == cudaSuccess)
     e = cudaMemcpy(p->mu, mu, sizeof(float) * H * kD, cudaMemcpyHostToDevice);
   if (e == cudaSuccess) e = cudaMemset(p->err, 0, sizeof(unsigned));
+  if (e == cudaSuccess) e = noalloc_scratch_address(&p->noalloc_ws);
   if (e != cudaSuccess) {
     optr_params_destroy(p);
     return OPTR_ERR_CUDA;
@@ -351,6 +375,7 @@ size_t optr_decode_workspace_size(const optr_params* p, int B, int max_pages) {
   return decode_plan(p, B, max_pages).total;
 }
 
+
 optr_status optr_decode_attention_win(const optr_params* p, const void* q,
                                       const int32_t* block_table,
                                       const int32_t* seq_lens, int B,
@@ -359,22 +384,14 @@ optr_status optr_decode_attention_win(const optr_params* p, const void* q,
                                       const int32_t* win_slot, int n_slots,
                                       float* out, void* workspace,
                                       size_t ws_bytes, cudaStream_t stream) {
-  if (!p || B <= 0 || max_pages <= 0 || num_pages <= 0)
-    return OPTR_ERR_INVALID_ARG;
-  if (!q || !block_table || !seq_lens || !pool || !out)
-    return OPTR_ERR_INVALID_ARG;
-  if (!aligned(pool, 16) || !aligned(q, 16) || !aligned(out, 16))
-    return OPTR_ERR_INVALID_ARG;
+  const optr_status st = decode_args_status(p, q, block_table, seq_lens, B,
+                                            max_pages, pool, num_pages, out);
+  if (st != OPTR_OK) return st;
   WinArgs wbuf;
   bool bad = false;
   const WinArgs* wa = window_args(p, const_cast<void*>(win), win_slot, n_slots,
                                   &wbuf, &bad);
   if (bad) return OPTR_ERR_INVALID_ARG;
-  if ((long long)max_pages * kPage > (1LL << 30) || B > (1 << 24))
-    return OPTR_ERR_OUT_OF_RANGE;
-  // the split-K plan indexes (sequence, KV head, page) units with 32 bits
-  if ((long long)B * max_pages * p->cfg.h_kv >= (1LL << 31))
-    return OPTR_ERR_OUT_OF_RANGE;
   DecodePlan plan = decode_plan(p, B, max_pages);
   if (!workspace || ws_bytes < plan.total || !aligned(workspace, 256))
     return OPTR_ERR_WORKSPACE;

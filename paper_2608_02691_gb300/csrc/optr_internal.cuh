@@ -42,6 +42,10 @@ struct optr_params {
   uint16_t* Rk_t5;     // device tcgen05 B operands of R_k (append_tc05.cu)
   uint16_t* Rv_t5;     // device tcgen05 B operands of R_v
   unsigned* err;       // device error word
+  // device address of the fixed scratch array of
+  // optr_decode_attention_noalloc on this params' device (noalloc.cu),
+  // looked up once at create with that device current
+  void* noalloc_ws;
   // stage timing (optr_profile_enable): ev[0..1] bracket the append kernel,
   // ev[2..5] the decode stages (before qrot, partial, combine, after).
   int prof;
@@ -50,6 +54,16 @@ struct optr_params {
 };
 
 namespace optr {
+// Argument and range checks shared by every decode entry point (null or
+// misaligned pointers, sizes): OPTR_OK or the status the call returns.
+optr_status decode_args_status(const optr_params* p, const void* q,
+                               const int32_t* block_table,
+                               const int32_t* seq_lens, int B, int max_pages,
+                               const uint8_t* pool, int num_pages,
+                               const float* out);
+// Device address of the no-allocation scratch array on the current device.
+cudaError_t noalloc_scratch_address(void** out);
+
 // Raise a kernel's dynamic shared memory limit on the current device to at
 // least `bytes` (static plus dynamic shared memory may exceed 48 KB only
 // after this opt-in).  Cached per (kernel, device) under a lock, so the
@@ -136,9 +150,11 @@ __host__ __device__ __forceinline__ int win_pos(int i, int n, int sink, int rece
   const int r0 = n - recent > sink ? n - recent : sink;
   return i < ns ? i : r0 + (i - ns);
 }
-// Store row of window position s (recent > 0 whenever s >= sink).
-__host__ __device__ __forceinline__ int win_row(int s, int sink, int recent) {
-  return s < sink ? s : sink + (s - sink) % recent;
+// Store row of window position s (recent > 0 whenever s >= sink), in 64
+// bits so that positions computed from any int32 pos0 stay exact; the row
+// itself lies in [0, sink + recent).
+__host__ __device__ __forceinline__ int win_row(long long s, int sink, int recent) {
+  return (int)(s < sink ? s : sink + (s - sink) % recent);
 }
 constexpr int kWinUnit = 16;  // window tokens per decode work unit
 

@@ -55,8 +55,7 @@ __device__ __forceinline__ void window_copy_body(
           if (slot < 0 || slot >= n_slots) {
             atomicOr(err, OPTR_DEVERR_WIN_SLOT);
           } else {
-            // row in [0, sink + recent), in 64 bits for any int32 pos0
-            const long long row = s < sink ? s : sink + (s - sink) % recent;
+            const long long row = win_row(s, sink, recent);
             base = (long long)slot * h_kv * 2 * rows * kD + row * kD;
           }
         }

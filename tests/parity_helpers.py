@@ -141,19 +141,6 @@ def gpu_decode(case, pool_np, variant=optr.OPTR_VARIANT_DEFAULT,
     return out.cpu().double().numpy()
 
 
-def flipped_groups(case, stats_ctx, stats_new):
-    """(b, h) groups whose cached codes differ in the tie band somewhere."""
-    out = set()
-    for st, cu in ((stats_ctx, case["cu_ctx"]), (stats_new, case["cu_new"])):
-        if st is None:
-            continue
-        cu = np.asarray(cu)
-        for t, h in np.argwhere(st["flipped"]):
-            b = int(np.searchsorted(cu, t, side="right") - 1)
-            out.add((b, int(h)))
-    return out
-
-
 def oracle_case(case, pool_init=None, group=32, clip_k=1.0, clip_v=1.0):
     """Oracle append of context and new tokens; returns (pool, u_ctx, u_new)."""
     pool = (np.zeros((case["num_pages"], case["h_kv"], 1536), np.uint8)
@@ -184,3 +171,110 @@ def oracle_decode(case, pool, rows=None, seq_lens=None, q=None):
         case["block_table"].numpy(),
         (case["seq_lens"] if seq_lens is None else seq_lens).numpy(), pool,
         case["R_k"].numpy(), case["R_v"].numpy(), case["h_kv"], rows=rows)
+
+
+def dequant_records(pool, pages, slots, h, kind):
+    """Dequantized rotated vectors code * scale + min (float64 [n][128]) of
+    KV head h at the given (page, slot) records of a pool; kind 0 = keys,
+    1 = values.  G = 128 records hold their pair in all four entries, so the
+    same 32-channel reading serves both group sizes."""
+    codes, sc, mn = slot_codes(pool, pages, slots, kind)
+    grp = _CH // 32
+    return codes[:, h, :] * sc[:, h, grp] + mn[:, h, grp]
+
+
+def e2e_row_bounds(case, pool_ref, pool_gpu, diffs, win=None, win_slot=None,
+                   sink=0, recent=0):
+    """Per output row, how far exact attention over the GPU-written cache may
+    lie from exact attention over the oracle-written one, given where the
+    two caches differ (in-band codes, an fp16 ulp of scale or min: both
+    within the append tolerance).  ``diffs`` is a list of (cu, pos0,
+    mask[n_tok][h_kv]) marking the differing token records of each write.
+    With BF16 windows (``win``: the oracle's store, bf16 bits
+    [n_slots][h_kv][2][sink + recent][128]; ``win_slot`` [B]) window
+    positions are read from the store, so their pool records never count.
+
+    For a row (b, j) of KV head h let D be the INT2 positions whose records
+    differ, p the oracle's softmax weights over the oracle cache, delta_s =
+    q'_j . (k'_s - k_s) / sqrt(d) the logit change (Sec. 3 Eq. 1 in the
+    rotated basis, Appendix "Rotated-query implementation") and
+    dv_s = v'_s - v_s.  The weights over the GPU cache are
+    p'_s = p_s e^{delta_s} / Z with Z = 1 + sum_D p_s (e^{delta_s} - 1), so,
+    with every value taken in the output basis (v R_v^T for INT2 positions,
+    the stored bf16 value for window positions),
+
+      |o' - o|_2 <= sum_D p'_s |dv_s|_2
+                    + (sum_s |p'_s - p_s|) * max_s |v_s - o|_2,
+      sum_s |p'_s - p_s| = ((1 - P_D)|1 - Z| + sum_D p_s |e^{delta_s} - Z|) / Z,
+
+    exactly (Sec. 3 Eq. 2; the sum of p' - p is zero, so any centre may be
+    subtracted from v; R_v is orthogonal, so |dv R_v^T|_2 = |dv|_2), and
+    |x|_inf <= |x|_2 bounds every element of the row.  Rows of groups with
+    no differing record get 0."""
+    B, h_q, h_kv = case["B"], case["h_q"], case["h_kv"]
+    ratio = h_q // h_kv
+    bt = case["block_table"].numpy()
+    lens = case["seq_lens"].numpy()
+    R_k = case["R_k"].numpy().astype(np.float64)
+    R_v = case["R_v"].numpy().astype(np.float64)
+    q = case["q"].float().numpy().astype(np.float64)
+    windows = sink > 0 or recent > 0
+    where = {}
+    for cu, pos0, mask in diffs:
+        cu = np.asarray(cu)
+        pos0 = np.asarray(pos0)
+        for t, h in np.argwhere(mask):
+            b = int(np.searchsorted(cu, t, side="right") - 1)
+            where.setdefault((b, int(h)), set()).add(int(pos0[b] + t - cu[b]))
+    bound = np.zeros((B, h_q))
+    for (b, h), poss in sorted(where.items()):
+        n = int(lens[b])
+        allp = np.arange(n)
+        in_win = (allp < sink) | (allp >= n - recent) if windows else np.zeros(n, bool)
+        d = np.array(sorted(s for s in poss if s < n and not in_win[s]), np.int64)
+        if n == 0 or d.size == 0:
+            continue
+        kr = dequant_records(pool_ref, bt[b, allp // 16], allp % 16, h, 0)
+        vr = dequant_records(pool_ref, bt[b, allp // 16], allp % 16, h, 1)
+        dk = dequant_records(pool_gpu, bt[b, d // 16], d % 16, h, 0) - kr[d]
+        dv = dequant_records(pool_gpu, bt[b, d // 16], d % 16, h, 1) - vr[d]
+        dvn = np.linalg.norm(dv, axis=1)
+        vout = vr @ R_v[h].T  # output basis
+        if windows:
+            wp = allp[in_win]
+            rows = np.where(wp < sink, wp, sink + (wp - sink) % max(recent, 1))
+            bits = np.asarray(win)[int(win_slot[b]), h, 1, rows, :]
+            vout[in_win] = (bits.astype(np.uint32) << 16).view(np.float32)
+        for r in range(ratio):
+            j = ratio * h + r
+            _, p = oracle.decode_attention(
+                synth.bf16_bits(case["q"]), bt, lens, pool_ref,
+                case["R_k"].numpy(), case["R_v"].numpy(), h_kv,
+                rows=[(b, j)], want_p=True, win=win, win_slot=win_slot,
+                sink=sink, recent=recent,
+                mu=case["mu"].numpy() if windows else None)
+            qp = (q[b, j] @ R_k[h]) / np.sqrt(128.0)
+            a = np.exp(dk @ qp)
+            pd = p[d]
+            Z = 1.0 + float(np.sum(pd * (a - 1.0)))
+            term_v = float(np.sum(pd * a / Z * dvn))
+            o = p @ vout
+            spread = float(np.max(np.linalg.norm(vout - o, axis=1)))
+            dp = ((1.0 - pd.sum()) * abs(1.0 - Z) +
+                  float(np.sum(pd * np.abs(a - Z)))) / Z
+            bound[b, j] = term_v + dp * spread
+    return bound
+
+
+def assert_rows_within_bar(got, ref, bound, what=""):
+    """Every row: max |gpu - oracle| <= OUT_TOL * RMS(oracle) + bound(row).
+    Returns (share of rows checked at the strict bar, mean bar / strict)."""
+    rms = float(np.sqrt(np.mean(ref ** 2)))
+    assert np.all(np.isfinite(got)), f"{what}: non-finite output"
+    bar = OUT_TOL * rms + bound
+    err = np.abs(got - ref).max(axis=2)
+    worst = np.unravel_index(np.argmax(err / bar), err.shape)
+    assert np.all(err <= bar * (1 + 1e-9)), (
+        f"{what}: row {worst} err {err[worst]:.3e} > bar {bar[worst]:.3e} "
+        f"(bound {bound[worst]:.3e}, strict {OUT_TOL * rms:.3e})")
+    return float((bound == 0).mean()), float(bar.mean() / (OUT_TOL * rms))

@@ -77,6 +77,8 @@ def test_host_argument_errors_launch_nothing(lib):
                                      None, None, 0, None) == -1
     assert lib.optr_decode_step(None, None, None, None, 0, None, None, None,
                                 None, 1, 1, None, 1, None, None, 0, None) == -1
+    assert lib.optr_decode_attention_noalloc(None, None, None, None, 1, 1,
+                                             None, 1, None, None) == -1
     assert lib.optr_decode_workspace_size(None, 1, 1) == 0
     assert lib.optr_page_bytes(None) == 0
     # the BF16-window entry points

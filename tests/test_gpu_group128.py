@@ -119,20 +119,18 @@ def test_paper_default_configuration_step(dvar):
     assert optr.optr_device_error(p) == 0
     assert np.array_equal(win.cpu().view(torch.int16).numpy().view(np.uint16), win_ref)
     pg = pool.cpu().numpy()
-    sts = []
+    diffs = []
     for cu, pos0, u in ((c["cu_ctx"], c["pos0_ctx"], u_ctx),
                         (c["cu_new"], c["pos0_new"], u_new)):
         pages, sl = ph.token_slots(cu, pos0, c["block_table"])
-        sts.append(ph.compare_append(pg, pool_ref, u, pages, sl))
-    skip = ph.flipped_groups(c, *sts)
+        st = ph.compare_append(pg, pool_ref, u, pages, sl)
+        diffs.append((cu.numpy(), pos0.numpy(), st["flipped"]))
     ref = oracle.decode_attention(
         synth.bf16_bits(c["q"]), c["block_table"].numpy(), c["seq_lens"].numpy(),
         pool_ref, c["R_k"].numpy(), c["R_v"].numpy(), c["h_kv"], win=win_ref,
         win_slot=slots, sink=sink, recent=recent, mu=c["mu"].numpy())
     got = out.cpu().double().numpy()
-    keep = np.ones(got.shape[:2], bool)
-    for b, h in skip:
-        keep[b, 4 * h:4 * h + 4] = False
-    assert keep.any()
-    ph.assert_decode_close(got[keep], ref[keep], "paper defaults")
-    assert np.all(np.isfinite(got))
+    bound = ph.e2e_row_bounds(c, pool_ref, pg, diffs, win=win_ref,
+                              win_slot=slots, sink=sink, recent=recent)
+    strict, mean_bar = ph.assert_rows_within_bar(got, ref, bound, "paper defaults")
+    print(f"paper defaults: strict rows {strict:.2f}, mean bar {mean_bar:.3f} x strict")

@@ -78,60 +78,61 @@ def test_decode_matches_oracle(name, scale, variant):
     print(f"{name} variant {variant}: err/rms {r:.2e}")
 
 
-@pytest.mark.parametrize("name,scale", CASES)
-@pytest.mark.parametrize("variant", VARIANTS)
-def test_end_to_end_matches_oracle(name, scale, variant):
-    """GPU append + GPU decode against oracle append + oracle decode.  Rows of
-    (sequence, KV head) groups whose cached records agree bit for bit must
-    meet the decode tolerance.  Other groups hold an in-band code or an fp16
-    ulp of scale/min (both allowed by the append tolerance); such a record
-    moves the output by up to a quantization step times its softmax weight,
-    so those rows are only reported (the append and decode tests check each
-    half strictly)."""
+def _end_to_end(name, scale, variant=optr.OPTR_VARIANT_DEFAULT):
+    """GPU append + GPU decode, the oracle's append + decode, and the bar of
+    every output row: OUT_TOL * RMS for rows of (sequence, KV head) groups
+    whose cached records agree bit for bit, plus ph.e2e_row_bounds for the
+    others (records that differ within the append tolerance: an in-band
+    code or an fp16 ulp of scale or min)."""
     c, pool_ref, u_ctx, u_new = _case(name, scale)
     p, pool, out = ph.gpu_case(c, variant=variant)
     pg = pool.cpu().numpy()
-    sts = []
+    diffs = []
     for cu, pos0, u in ((c["cu_ctx"], c["pos0_ctx"], u_ctx),
                         (c["cu_new"], c["pos0_new"], u_new)):
         if u is None:
-            sts.append(None)
             continue
         pages, slots = ph.token_slots(cu, pos0, c["block_table"])
-        sts.append(ph.compare_append(pg, pool_ref, u, pages, slots))
-    skip = ph.flipped_groups(c, *sts)
+        st = ph.compare_append(pg, pool_ref, u, pages, slots)
+        diffs.append((cu.numpy(), pos0.numpy(), st["flipped"]))
     got = out.cpu().double().numpy()
     ref = ph.oracle_decode(c, pool_ref)
-    keep = np.ones(got.shape[:2], bool)
-    for b, h in skip:
-        keep[b, 4 * h:4 * h + 4] = False
-    if keep.any():
-        ph.assert_decode_close(got[keep], ref[keep], f"{name} end-to-end")
-    assert np.all(np.isfinite(got))
     rms = float(np.sqrt(np.mean(ref ** 2)))
+    bound = ph.e2e_row_bounds(c, pool_ref, pg, diffs)
+    bar = ph.OUT_TOL * rms + bound
+    return got, ref, rms, bound, bar
+
+
+@pytest.mark.parametrize("name,scale", CASES)
+@pytest.mark.parametrize("variant", VARIANTS)
+def test_end_to_end_every_row_within_its_bar(name, scale, variant):
+    """GPU append + GPU decode against oracle append + oracle decode, every
+    row asserted: |gpu - oracle| <= OUT_TOL * RMS + bound(row), where bound
+    is 0 for rows whose cached records match the oracle's bit for bit and
+    the exact perturbation bound of ph.e2e_row_bounds otherwise.  (The
+    decode-alone tests bound the GPU decode of a given cache by
+    OUT_TOL * RMS; the bound covers the move from the oracle's cache to the
+    GPU's, both inside the append tolerance.)"""
+    got, ref, rms, bound, bar = _end_to_end(name, scale, variant)
+    strict, mean_bar = ph.assert_rows_within_bar(got, ref, bound, f"{name} end-to-end")
     err = float(np.abs(got - ref).max())
-    print(f"{name}: strict over {int(keep.sum())} rows ({len(skip)} groups "
-          f"with in-tolerance record differences); all rows err/rms {err / rms:.2e}")
+    print(f"{name} variant {variant}: strict rows {strict:.2f}, mean bar "
+          f"{mean_bar:.3f} x strict, all rows max err/rms {err / rms:.2e}")
 
 
-def test_end_to_end_strict_rows_are_the_majority():
-    """Across the multi-sequence workloads a good share of (sequence, KV head)
-    groups have bit-identical cached records (10-30% at these sizes), so
-    the strict end-to-end comparison is never vacuous."""
-    total = strict = 0
+def test_end_to_end_bar_stays_tight():
+    """The per-row bound is not a loophole: on the multi-sequence workloads
+    the average bar stays within 1.5x the strict decode tolerance, so every
+    end-to-end row is checked at nearly the decode bar (the differing
+    records are rare in-band codes and fp16 ulps; their perturbation bound
+    is small)."""
     for name, scale in (("decode8k", 1 / 16), ("ragged", 1 / 32)):
-        c, pool_ref, u_ctx, u_new = _case(name, scale)
-        p, pool, _ = ph.gpu_case(c)
-        pg = pool.cpu().numpy()
-        sts = []
-        for cu, pos0, u in ((c["cu_ctx"], c["pos0_ctx"], u_ctx),
-                            (c["cu_new"], c["pos0_new"], u_new)):
-            pages, slots = ph.token_slots(cu, pos0, c["block_table"])
-            sts.append(ph.compare_append(pg, pool_ref, u, pages, slots))
-        skip = ph.flipped_groups(c, *sts)
-        total += c["B"] * c["h_kv"]
-        strict += c["B"] * c["h_kv"] - len(skip)
-    assert strict >= total // 16, (strict, total)
+        _, _, rms, bound, bar = _end_to_end(name, scale)
+        ratio = float(bar.mean() / (ph.OUT_TOL * rms))
+        print(f"{name}: mean bar {ratio:.3f} x strict, strict rows "
+              f"{float((bound == 0).mean()):.2f}, max bound/strict "
+              f"{float(bound.max() / (ph.OUT_TOL * rms)):.3f}")
+        assert ratio <= 1.5, (name, ratio)
 
 
 @pytest.mark.parametrize("variant", VARIANTS)

@@ -202,31 +202,31 @@ def test_window_decode_short_and_empty_sequences(dvar):
 @pytest.mark.parametrize("name,scale", CASES)
 @pytest.mark.parametrize("dvar", VARIANTS)
 def test_window_step_end_to_end(name, scale, dvar):
-    """GPU cache write and decode step with windows against the oracle's
-    (rows of groups with in-tolerance record differences only reported)."""
+    """GPU cache write and decode step with windows against the oracle's,
+    every row asserted at OUT_TOL * RMS plus the perturbation bound of the
+    INT2 records that differ within the append tolerance (0 when none)."""
     sink, recent = 64, 256
     c, pool_ref, u_ctx, u_new, win_ref, slots = _case(name, scale, sink, recent)
     _, pool, win, out = _gpu_run(c, sink, recent, slots, win_ref.shape[0],
                                  dvar=dvar, step=True)
     np.testing.assert_array_equal(_win_bits(win), win_ref)
     pg = pool.cpu().numpy()
-    sts = []
+    diffs = []
     for cu, pos0, u in ((c["cu_ctx"], c["pos0_ctx"], u_ctx),
                         (c["cu_new"], c["pos0_new"], u_new)):
         if u is None:
-            sts.append(None)
             continue
         pages, slots_ = ph.token_slots(cu, pos0, c["block_table"])
-        sts.append(ph.compare_append(pg, pool_ref, u, pages, slots_))
-    skip = ph.flipped_groups(c, *sts)
+        st = ph.compare_append(pg, pool_ref, u, pages, slots_)
+        diffs.append((cu.numpy(), pos0.numpy(), st["flipped"]))
     got = out.cpu().double().numpy()
     ref = _oracle_decode(c, pool_ref, win_ref, slots, sink, recent)
-    keep = np.ones(got.shape[:2], bool)
-    for b, h in skip:
-        keep[b, 4 * h:4 * h + 4] = False
-    if keep.any():
-        ph.assert_decode_close(got[keep], ref[keep], f"{name} step windows")
-    assert np.all(np.isfinite(got))
+    bound = ph.e2e_row_bounds(c, pool_ref, pg, diffs, win=win_ref,
+                              win_slot=slots, sink=sink, recent=recent)
+    strict, mean_bar = ph.assert_rows_within_bar(got, ref, bound,
+                                                 f"{name} step windows")
+    print(f"{name} windows variant {dvar}: strict rows {strict:.2f}, mean bar "
+          f"{mean_bar:.3f} x strict")
 
 
 def test_window_step_equals_append_then_decode():

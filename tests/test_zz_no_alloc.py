@@ -9,12 +9,12 @@ calls in a row (the second call reuses the scratch the first one left), and
 that a batch too large for the scratch is refused.  The file name makes
 pytest collect it last.
 """
+import ctypes
+
 import pytest
 import torch
 
 from paper_2608_02691_gb300 import optr, synth
-
-import parity_helpers as ph
 
 pytestmark = pytest.mark.gpu
 
@@ -45,9 +45,9 @@ def test_noalloc_matches_workspace_entry_point(dev, name, scale):
         out = torch.full_like(ref, float("nan"))
         optr.optr_decode_attention_noalloc(p, q, bt, lens, pool, out)
         torch.cuda.synchronize()
-        ph.assert_decode_close(out.cpu().double().numpy(),
-                               ref.cpu().double().numpy(),
-                               f"{name} noalloc call {call}")
+        # the same kernels with the same plan: bit-identical to the
+        # workspace call
+        assert torch.equal(out, ref), f"{name} noalloc call {call}"
     assert optr.optr_device_error(p) == 0
 
 
@@ -64,3 +64,30 @@ def test_noalloc_rejects_batches_beyond_the_scratch(dev):
     with pytest.raises(optr.OptrError) as e:
         optr.optr_decode_attention_noalloc(p, q, bt, lens, pool, out)
     assert e.value.status == -4
+
+
+def test_noalloc_errors_follow_the_workspace_entry_point(dev):
+    """Argument and range errors come out as optr_decode_attention returns
+    them, before the scratch-size check: an oversized batch is out of range
+    (not a workspace error), a null query with a batch too large for the
+    scratch is an invalid argument, and params with BF16 windows are
+    refused.  Every case returns before any launch, so the (aligned,
+    non-null) device pointers below are never dereferenced."""
+    lib = optr.lib()
+    c = synth.build_case(synth.workload("tiny", 0, 1 / 64), 0)
+    p = optr.optr_params_create(c["R_k"], c["R_v"], c["mu"], c["h_q"])
+    buf = torch.zeros(1 << 16, dtype=torch.uint8, device=dev)
+    a = ctypes.c_void_p(buf.data_ptr())
+    ws = ctypes.c_void_p(buf.data_ptr())
+    for B, max_pages, q, want in (((1 << 24) + 1, 1, a, -3),
+                                  (64, (1 << 26) + 1, a, -3),
+                                  (4096, 64, None, -1)):
+        got_ws = lib.optr_decode_attention(p.handle, q, a, a, B, max_pages, a, 1,
+                                           a, ws, 1 << 16, None)
+        got_na = lib.optr_decode_attention_noalloc(p.handle, q, a, a, B,
+                                                   max_pages, a, 1, a, None)
+        assert got_ws == want and got_na == want, (B, max_pages, got_ws, got_na)
+    pw = optr.optr_params_create(c["R_k"], c["R_v"], c["mu"], c["h_q"],
+                                 sink=64, recent=256)
+    assert lib.optr_decode_attention_noalloc(pw.handle, a, a, a, 1, 1, a, 1, a,
+                                             None) == -1
