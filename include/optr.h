@@ -234,12 +234,8 @@ size_t optr_decode_workspace_size(const optr_params* p, int B, int max_pages);
  *   pool        device bytes [num_pages][h_kv][1536] (read only).
  *   out         device float32 [B][h_q][D]: attention output o = o' R_v^T.
  *   workspace   device, at least optr_decode_workspace_size(p, B, max_pages)
- *               bytes, 256-byte aligned, zero-filled once before its first
- *               use (cudaMemset / torch.zeros): its first bytes hold
- *               arrival counters that must start at zero, and every call
- *               leaves them at zero, so the same workspace serves later
- *               calls of any batch shape it is large enough for.  The rest
- *               is scratch between calls (concurrent calls need distinct
+ *               bytes, 256-byte aligned; contents need no initialisation and
+ *               are scratch between calls (concurrent calls need distinct
  *               workspaces).
  */
 optr_status optr_decode_attention(const optr_params* p, const void* q,
@@ -316,10 +312,8 @@ optr_status optr_profile_last(const optr_params* p, float ms[4]);
  * optr_params_create looks up the array's device address on its device
  * (with that device current) and keeps it in the params, so this call does
  * no set-up of its own; params created after a cudaDeviceReset carry the
- * new address.  The array keeps whatever the previous call left; each
- * call clears the part that must start at zero (the workspace's arrival
- * counters) with a cudaMemsetAsync on its stream before the decode.  All
- * calls on a device share the one array, so calls that overlap on the GPU
+ * new address.  Nothing in the scratch needs to start at zero.  All calls
+ * on a device share the one array, so calls that overlap on the GPU
  * (different streams, or different threads without ordering) race and
  * corrupt each other's results; serialise them.  This call allocates
  * nothing and never calls cudaMalloc or cudaFree.

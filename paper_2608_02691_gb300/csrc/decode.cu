@@ -786,43 +786,6 @@ cudaError_t launch_decode(const optr_params* p, int variant,
 
   int* cnt_ws = reinterpret_cast<int*>(w + plan.off_cnt);
   cudaError_t e;
-  if (variant != OPTR_VARIANT_CUDA_CORE && !windows) {
-    // one launch for the decode (decode_fused.cu); a step's cache write
-    // runs first, as the prologue's append CTAs only
-    if (app) {
-      prof_mark(p, 0, s);
-      const int T = small_tile(app->n_tok);
-      const int tiles = (app->n_tok + T - 1) / T;
-      const int n_app = tiles * h_kv * 2;
-      const size_t sm_app = T == kSmallTokFew ? sizeof(AppendSmallSmemT<kSmallTokFew>)
-                                              : sizeof(AppendSmallSmemT<kSmallTok>);
-      auto fn = T == kSmallTokFew ? step_prologue_kernel<kSmallTokFew>
-                                  : step_prologue_kernel<kSmallTok>;
-      e = ensure_dynamic_smem(reinterpret_cast<const void*>(fn), sm_app);
-      if (e != cudaSuccess) return e;
-      e = launch_pdl(fn, dim3(n_app), dim3(512), sm_app, s, n_app, tiles, app->k,
-                     app->v, app->n_tok, app->cu_new, app->pos0, bt, app->pool,
-                     num_pages, (const float*)p->R_v, (const float*)p->muR,
-                     p->cfg.clip_k, p->cfg.clip_v, q, (const float*)p->R_k, B,
-                     h_q, h_kv, qscale, seq_lens, max_pages, qf, qs, frag, koff,
-                     invs, pref, nzpref, cnt_ws, p->err, p->fold_v, 0,
-                     (__nv_bfloat16*)nullptr, (const int32_t*)nullptr, 0, sink,
-                     recent, p->cfg.group == 128 ? 1 : 0);
-      if (e != cudaSuccess) return e;
-      prof_mark(p, 1, s);
-    }
-    prof_mark(p, 2, s);
-    prof_mark(p, 3, s);
-    e = launch_decode_fused(p, q, bt, seq_lens, B, max_pages, pool, num_pages,
-                            out, pref, nzpref, part,
-                            reinterpret_cast<float*>(w + plan.off_ctap),
-                            reinterpret_cast<int*>(w + plan.off_ccnt),
-                            w + plan.off_qtab, app != nullptr, s);
-    if (e != cudaSuccess) return e;
-    prof_mark(p, 4, s);
-    prof_mark(p, 5, s);
-    return cudaSuccess;
-  }
   if (app) {
     // the cache write of the step (INT2 records and window copies) and the
     // query rotation in one launch

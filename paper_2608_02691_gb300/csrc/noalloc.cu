@@ -36,13 +36,6 @@ extern "C" optr_status optr_decode_attention_noalloc(
   const size_t need = optr_decode_workspace_size(p, B, max_pages);
   if (need == 0 || need > OPTR_NOALLOC_SCRATCH_BYTES) return OPTR_ERR_WORKSPACE;
   if (!p->noalloc_ws) return OPTR_ERR_CUDA;
-  // the arrival counters at the start of the workspace must be zero when
-  // the decode begins; the array keeps whatever the previous call (on any
-  // stream) left, so they are cleared here, in stream order (a memset, no
-  // allocation)
-  const size_t zero_bytes = optr::decode_plan(p, B, max_pages).off_qf;
-  if (cudaMemsetAsync(p->noalloc_ws, 0, zero_bytes, stream) != cudaSuccess)
-    return OPTR_ERR_CUDA;
   return optr_decode_attention(p, q, block_table, seq_lens, B, max_pages,
                                pool, num_pages, out, p->noalloc_ws,
                                OPTR_NOALLOC_SCRATCH_BYTES, stream);

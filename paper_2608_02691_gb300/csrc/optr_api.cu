@@ -57,10 +57,6 @@ cudaError_t ensure_dynamic_smem(const void* kernel, size_t bytes) {
 }
 
 // Workspace of one decode call (all offsets 256-byte aligned):
-//   ccnt int   [SMs]           arrival counters of the one-launch decode, at
-//                               offset 0 whatever the batch: zero before
-//                               the first call, and every call leaves them
-//                               at zero
 //   qf   float [B][h_q][128]   rotated, pre-scaled queries
 //   qs   float [B][h_q][4]     per-group sums of qf
 //   frag u32   [B][h_kv][32][16] tensor-core B fragments of qf (hi/lo f16)
@@ -68,16 +64,10 @@ cudaError_t ensure_dynamic_smem(const void* kernel, size_t bytes) {
 //                               [query head][group][hi/lo] (decode_tc.cu)
 //   invs float [B][h_q]         1 / (power-of-two prescale of frag)
 //   pref int   [2][B+1]        page prefix sums / non-empty prefix counts
-//   cnt  int   [B*h_kv]        arrival counters: zero between calls (the
-//                               workspace starts zeroed; every call resets
-//                               the ones it counts with)
+//   cnt  int   [B*h_kv]        combine arrival counters (zeroed by qrot)
 //   part float [W + B*h_kv][520] split-K partials (o'[4][128], m[4], l[4])
 //   cpart float [B*h_kv*S][520] combine chunk results (only when S > 1)
 //   wpart float [Ww + B*h_kv][520] window partials (BF16 windows only)
-//   ctap float [SMs + B*h_kv][520]  per-CTA merged partials of segments that
-//                               span CTAs (one-launch decode)
-//   qtab       [B*h_kv]        query data of segments beyond a CTA's shared
-//                               table (one-launch decode, many short segments)
 // S, the combine CTAs per (sequence, KV head), is sized for ~32 partials
 // each when every sequence is max_pages long: a segment then overlaps about
 // W / (B*h_kv) + 2 warp ranges.
@@ -104,8 +94,6 @@ DecodePlan decode_plan(const optr_params* p, int B, int max_pages) {
     }
   }
   size_t o = 0;
-  d.off_ccnt = o;
-  o = round_up(o + sizeof(int) * (size_t)p->num_sms, 256);
   d.off_qf = o;
   o = round_up(o + sizeof(float) * (size_t)B * d.h_q * kD, 256);
   d.off_qs = o;
@@ -136,11 +124,6 @@ DecodePlan decode_plan(const optr_params* p, int B, int max_pages) {
   if (d.Ww > 0)
     o = round_up(o + sizeof(float) * kPartFloats *
                          ((size_t)d.Ww + (size_t)B * d.h_kv), 256);
-  d.off_ctap = o;
-  o = round_up(o + sizeof(float) * kPartFloats *
-                       ((size_t)p->num_sms + (size_t)B * d.h_kv), 256);
-  d.off_qtab = o;
-  o = round_up(o + fused_qtab_entry_bytes() * (size_t)B * d.h_kv, 256);
   d.total = o;
   return d;
 }
@@ -250,14 +233,6 @@ optr_status optr_params_create(const optr_config* cfg, const float* R_k,
   std::vector<uint16_t> t5((size_t)H * kRT5Halves);
   if (e == cudaSuccess) e = cudaMalloc(&p->Rk_t5, sizeof(uint16_t) * t5.size());
   if (e == cudaSuccess) e = cudaMalloc(&p->Rv_t5, sizeof(uint16_t) * t5.size());
-  if (e == cudaSuccess) e = cudaMalloc(&p->Rk_l3, sizeof(uint16_t) * (size_t)H * kRL3Halves);
-  if (e == cudaSuccess) {
-    std::vector<uint16_t> l3((size_t)H * kRL3Halves);
-    for (int h = 0; h < H; ++h)
-      build_rotation_l3(R_k + h * mat, l3.data() + (size_t)h * kRL3Halves);
-    e = cudaMemcpy(p->Rk_l3, l3.data(), sizeof(uint16_t) * l3.size(),
-                   cudaMemcpyHostToDevice);
-  }
   if (e == cudaSuccess) {
     for (int h = 0; h < H; ++h)
       build_rotation_tc05(R_k + h * mat, t5.data() + (size_t)h * kRT5Halves);
@@ -301,7 +276,6 @@ void optr_params_destroy(optr_params* p) {
   cudaFree(p->muR);
   cudaFree(p->mu);
   cudaFree(p->Rk_t5);
-  cudaFree(p->Rk_l3);
   cudaFree(p->Rv_t5);
   cudaFree(p->err);
   free(p);

@@ -40,8 +40,6 @@ struct optr_params {
   float* muR;          // device [h_kv][D], mu R_k computed in fp64
   float* mu;           // device [h_kv][D], the key mean (window logits)
   uint16_t* Rk_t5;     // device tcgen05 B operands of R_k (append_tc05.cu)
-  uint16_t* Rk_l3;     // device R_k^T in three bf16 limbs, [h][limb][j][i],
-                       // 16-byte chunks of a row swizzled (decode_fused.cu)
   uint16_t* Rv_t5;     // device tcgen05 B operands of R_v
   unsigned* err;       // device error word
   // device address of the fixed scratch array of
@@ -119,8 +117,8 @@ struct DecodePlan {
   int S;                           // combine CTAs per (sequence, KV head)
   int Uw;   // BF16-window units (16 window tokens) per (sequence, KV head)
   int Ww;   // window warps (tensor kernel: 4 per SM; CUDA-core: all W), at most B * h_kv * Uw
-  size_t off_ccnt, off_qf, off_qs, off_frag, off_koff, off_invs, off_pref,
-      off_cnt, off_part, off_cpart, off_wpart, off_ctap, off_qtab, total;
+  size_t off_qf, off_qs, off_frag, off_koff, off_invs, off_pref, off_cnt,
+      off_part, off_cpart, off_wpart, total;
 };
 DecodePlan decode_plan(const optr_params* p, int B, int max_pages);
 
@@ -178,11 +176,6 @@ cudaError_t launch_append_cuda_core(const optr_params* p, const __nv_bfloat16* k
                                     const int32_t* bt, int B, int max_pages,
                                     uint8_t* pool, int num_pages,
                                     cudaStream_t s);
-// The one-launch decode's query-rotation operand: R^T[j][i] = R[i][j] split
-// into bf16 limbs hi + mid + lo (24 significant bits), [3][128][128] per
-// head, the 8-element chunk c of row j stored at chunk c ^ (j % 8).
-constexpr int kRL3Halves = 3 * kD * kD;
-void build_rotation_l3(const float* R /*[D][D]*/, uint16_t* out);
 // tcgen05 append operand: [hi, lo][128 x 128] fp16 per head, see append_tc05.cu.
 constexpr int kRT5Halves = 2 * kD * kD;
 void build_rotation_tc05(const float* R /*[D][D]*/, uint16_t* out);
@@ -208,18 +201,6 @@ cudaError_t launch_decode(const optr_params* p, int variant,
                           const uint8_t* pool, int num_pages, float* out,
                           void* ws, const DecodePlan& plan, cudaStream_t s,
                           const StepAppend* app, const WinArgs* win);
-
-// The one-launch decode (decode_fused.cu): tensor-core variant without
-// BF16 windows.  inputs_ready: the previous launch in the stream is the
-// step's cache write, which waited for the caller's kernels.
-cudaError_t launch_decode_fused(const optr_params* p, const __nv_bfloat16* q,
-                                const int32_t* bt, const int32_t* seq_lens,
-                                int B, int max_pages, const uint8_t* pool,
-                                int num_pages, float* out, int* pref, int* nz,
-                                float* part, float* cpart, int* cnt, void* qtab,
-                                bool inputs_ready, cudaStream_t s);
-// bytes of one segment's query data in the one-launch decode's table
-size_t fused_qtab_entry_bytes();
 
 // Window part of a cache write (positions of the BF16 windows copied into
 // the store); a separate launch after the INT2 write.

@@ -367,5 +367,4 @@ def new_pool(p: Params, num_pages: int, device="cuda") -> torch.Tensor:
 
 def new_workspace(p: Params, B: int, max_pages: int, device="cuda"):
     n = optr_decode_workspace_size(p, B, max_pages)
-    # zero-filled before first use; every decode call leaves it so
-    return torch.zeros(n, dtype=torch.uint8, device=device)
+    return torch.empty(n, dtype=torch.uint8, device=device)
