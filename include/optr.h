@@ -255,7 +255,11 @@ optr_status optr_decode_attention(const optr_params* p, const void* q,
  * first launches of that pair are independent (the cache write does not
  * touch the query), so for decode-step sized writes (n_tok <= 256) with the
  * default variants they run as one launch.  Other cases run exactly as the
- * two calls.  No allocation, no synchronisation.
+ * two calls.  The decode may read pages that the step does not write
+ * before the write has finished, so a physical page that receives one of
+ * the step's tokens must not also be mapped by another sequence's block
+ * table (pages holding a sequence's newest tokens are never shared in a
+ * paged cache).  No allocation, no synchronisation.
  */
 optr_status optr_decode_step(const optr_params* p, const void* q,
                              const void* k, const void* v, int n_tok,
@@ -390,6 +394,22 @@ optr_status optr_decode_step_win(const optr_params* p, const void* q,
 
 /* Static description of a status code. */
 const char* optr_strerror(optr_status s);
+
+/*
+ * Self-test of the bounded waits (library machinery; the paper has no
+ * counterpart).  Every mbarrier wait in the tcgen05 kernels gives up after
+ * a time limit, flags OPTR_DEVERR_TIMEOUT, drains its own copies and frees
+ * its tensor memory, so that no wait can hang the GPU.  This call launches
+ * one CTA that allocates the cache write's tensor-memory columns, waits
+ * with the limit limit_ns (1 ms .. 2 s, else OPTR_ERR_INVALID_ARG) on an
+ * mbarrier phase that nothing completes, and leaves through the cache
+ * write's exit path: OPTR_DEVERR_TIMEOUT is then set in p's device error
+ * word (optr_device_error) and the columns are free again.  Asynchronous on
+ * `stream`; no allocation.
+ */
+optr_status optr_selftest_wait_timeout(const optr_params* p,
+                                       unsigned long long limit_ns,
+                                       cudaStream_t stream);
 
 #ifdef __cplusplus
 }

@@ -570,3 +570,51 @@ cudaError_t launch_append_tc05(const optr_params* p, const __nv_bfloat16* k,
 }
 
 }  // namespace optr
+
+namespace optr {
+namespace {
+
+// Self-test of the bounded waits of the tcgen05 kernels: the exit path of
+// append_tc05_kernel run against an mbarrier phase that nothing completes.
+// Warp 0 allocates the same tensor-memory columns as the cache write; every
+// warp waits with the given limit, which runs out; the CTA then takes the
+// cache write's exit sequence (flag OPTR_DEVERR_TIMEOUT, free the columns).
+__global__ void __launch_bounds__(128, 1)
+tc05_wait_selftest_kernel(unsigned* err, unsigned long long limit_ns) {
+  __shared__ __align__(8) uint64_t bar;
+  __shared__ uint32_t tmem;
+  __shared__ int abort;
+  const int tid = threadIdx.x, warp = tid >> 5;
+  if (tid == 0) {
+    tc05::bar_init(&bar, 1);  // one arrival completes the phase; none comes
+    abort = 0;
+    tc05::bar_init_fence();
+  }
+  if (warp == 0) tc05::tmem_alloc(&tmem, kTmemCols);
+  tc05::fence_before();
+  __syncthreads();
+  tc05::fence_after();
+  const uint32_t base = tmem;
+  volatile int* ab = &abort;
+  // each warp waits (all its lanes agree), as the cache write's warps do
+  __all_sync(0xffffffffu, tc05::bar_wait(&bar, 0, ab, limit_ns));
+  tc05::fence_before();
+  __syncthreads();
+  if (abort && tid == 0) atomicOr(err, OPTR_DEVERR_TIMEOUT);
+  if (warp == 0) {
+    tc05::fence_after();
+    tc05::tmem_dealloc(base, kTmemCols);
+  }
+}
+
+}  // namespace
+}  // namespace optr
+
+extern "C" optr_status optr_selftest_wait_timeout(const optr_params* p,
+                                                  unsigned long long limit_ns,
+                                                  cudaStream_t stream) {
+  if (!p || limit_ns < 1000000ull || limit_ns > 2000000000ull)
+    return OPTR_ERR_INVALID_ARG;
+  optr::tc05_wait_selftest_kernel<<<1, 128, 0, stream>>>(p->err, limit_ns);
+  return cudaGetLastError() == cudaSuccess ? OPTR_OK : OPTR_ERR_CUDA;
+}

@@ -724,6 +724,7 @@ cudaError_t launch_partial_tensor(const optr_params* p, const uint8_t* pool,
                                   const float* invs, const float* qs,
                                   const int* pref, const int* nzpref,
                                   float* part, int W, bool early_pages,
+                                  const int32_t* step_cu, const int32_t* step_pos0,
                                   const WinPhase& wp, cudaStream_t s);
 
 cudaError_t launch_window_copy(const optr_params* p, const __nv_bfloat16* k,
@@ -831,7 +832,8 @@ cudaError_t launch_decode(const optr_params* p, int variant,
     // fused prologue it must wait first
     e = launch_partial_tensor(p, pool, bt, seq_lens, B, max_pages, num_pages,
                               frag, koff, invs, qs, pref, nzpref, part, plan.W,
-                              app == nullptr, wp, s);
+                              app == nullptr, app ? app->cu_new : nullptr,
+                              app ? app->pos0 : nullptr, wp, s);
   } else {
     e = launch_pdl(windows ? partial_cuda_core_kernel<true> : partial_cuda_core_kernel<false>,
                    dim3(plan.W / 4), dim3(128), 0, s,

@@ -163,8 +163,10 @@ __device__ __forceinline__ void load_chunk(PageChunk& ch, int base, int f1,
                                            const int32_t* __restrict__ bt,
                                            int B, int h_kv, int max_pages,
                                            int num_pages, unsigned* err,
-                                           int lane, int sink, int recent) {
+                                           int lane, int sink, int recent,
+                                           int& lpage) {
   ch.base = base;
+  lpage = 0;
   ch.unit = -1;
   ch.key = -1;
   ch.nvalid = 0;
@@ -181,6 +183,7 @@ __device__ __forceinline__ void load_chunk(PageChunk& ch, int base, int f1,
     const int r = f - p0 * h_kv;
     const int h = r / np;
     const int page = sink / kPage + (r - h * np);  // logical page (INT2 range)
+    lpage = page;
     const int phys = __ldg(bt + (size_t)lo * max_pages + page);
     ch.key = lo * h_kv + h;
     if (phys >= 0 && phys < num_pages) {
@@ -234,6 +237,8 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
                       const int* __restrict__ pref,
                       const int* __restrict__ nzpref,
                       float* __restrict__ part, int W, int early_pages,
+                      const int32_t* __restrict__ step_cu,
+                      const int32_t* __restrict__ step_pos0,
                       unsigned* err, int sink, int recent, WinPhase wp) {
   // One 16-warp CTA per SM: the warp schedulers favour the CTAs that
   // arrived first on an SM, and with four 4-warp CTAs per SM the last CTA
@@ -295,8 +300,9 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
   }
   PageChunk chk;
   int f_issue = f0;
+  int lpage;
   load_chunk(chk, f0, f1, pref, spref, cached, seq_lens, bt, B, h_kv,
-             max_pages, num_pages, err, lane, sink, recent);
+             max_pages, num_pages, err, lane, sink, recent, lpage);
 
   // issue one page into stage s (no commit); every lane records what the
   // stage holds
@@ -304,7 +310,7 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
     if (f_issue < f1) {
       if (f_issue - chk.base == 32)
         load_chunk(chk, f_issue, f1, pref, spref, cached, seq_lens, bt, B, h_kv,
-                   max_pages, num_pages, err, lane, sink, recent);
+                   max_pages, num_pages, err, lane, sink, recent, lpage);
       const int j = f_issue - chk.base;
       const int unit = __shfl_sync(0xffffffffu, chk.unit, j);
       const int key = __shfl_sync(0xffffffffu, chk.key, j);
@@ -326,10 +332,28 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
     issue(2 * q + 1);
     cp_async_commit();
   };
-  if (early_pages) issue_pair(0);
+  // In a decode step the previous kernel writes the step's new tokens, at
+  // positions [pos0[b], pos0[b] + n_b) of each sequence b (n_b from cu_new,
+  // an input complete before that kernel began).  A page of the first pair
+  // none of whose 16 positions is among them holds only records written
+  // before the step, so the pair is fetched before the wait when both pages
+  // are such (a step's written pages are not read by another sequence).
+  bool pre = early_pages != 0;
+  if (!pre && step_cu != nullptr) {
+    bool safe = true;
+    if (lane < 2 && f0 + lane < f1 && chk.key >= 0) {
+      const int b = chk.key / h_kv;
+      const long long n = (long long)__ldg(step_cu + b + 1) - __ldg(step_cu + b);
+      const long long s0 = __ldg(step_pos0 + b);
+      const long long t0 = (long long)lpage * kPage;
+      safe = n <= 0 || s0 >= t0 + kPage || s0 + n <= t0;
+    }
+    pre = __all_sync(0xffffffffu, safe);
+  }
+  if (pre) issue_pair(0);
   pdl_wait();  // (returns at once when already passed above)
   pdl_trigger();
-  if (!early_pages) issue_pair(0);
+  if (!pre) issue_pair(0);
 
   // per-segment state
   uint32_t bmin = 0;           // key min-term B fragment (sum q' per group)
@@ -641,6 +665,8 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
 
   // Pages go through the stages in pairs: pair q (stages 2q, 2q+1) is
   // processed while the other pair is in flight.
+  // the first segment's query data, loaded while the first pages land
+  begin_segment(__shfl_sync(0xffffffffu, chk.key, 0));
   static_assert(kStages == 4, "two pairs of stages");
   const int total = f1 - f0;
 #pragma unroll 1
@@ -671,6 +697,7 @@ cudaError_t launch_partial_tensor(const optr_params* p, const uint8_t* pool,
                                   const float* invs, const float* qs,
                                   const int* pref, const int* nzpref,
                                   float* part, int W, bool early_pages,
+                                  const int32_t* step_cu, const int32_t* step_pos0,
                                   const WinPhase& wp, cudaStream_t s) {
   const size_t dsmem = sizeof(WarpSmemTC) * kWarps;
   const bool win = wp.Ww > 0;
@@ -680,7 +707,7 @@ cudaError_t launch_partial_tensor(const optr_params* p, const uint8_t* pool,
   return launch_pdl(fn, dim3(W / (win ? kWinIntWarps : kWarps)), dim3(kWarps * 32),
                     dsmem, s, pool, bt, seq_lens, B, max_pages, num_pages,
                     p->cfg.h_q, p->cfg.h_kv, frag, koff, invs, qs, pref, nzpref,
-                    part, W, early_pages ? 1 : 0, p->err, p->cfg.sink,
+                    part, W, early_pages ? 1 : 0, step_cu, step_pos0, p->err, p->cfg.sink,
                     p->cfg.recent, wp);
 }
 

@@ -61,11 +61,13 @@ __device__ __forceinline__ bool bar_try_wait(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 
-// Wait for the phase of the given parity to complete.  Gives up after about
-// two seconds, or as soon as *abort is set; returns false then (and sets
-// *abort itself on its own timeout), so that no wait can hang the GPU.
+// Wait for the phase of the given parity to complete.  Gives up after
+// limit_ns nanoseconds (about two seconds unless given), or as soon as
+// *abort is set; returns false then (and sets *abort itself on its own
+// timeout), so that no wait can hang the GPU.
 __device__ __forceinline__ bool bar_wait(uint64_t* bar, uint32_t parity,
-                                         volatile int* abort) {
+                                         volatile int* abort,
+                                         uint64_t limit_ns = 2000000000ull) {
   if (bar_try_wait(bar, parity)) return true;
   uint64_t t0;
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t0));
@@ -78,7 +80,7 @@ __device__ __forceinline__ bool bar_wait(uint64_t* bar, uint32_t parity,
       if (*abort) return false;
       uint64_t t;
       asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-      if (t - t0 > 2000000000ull) {
+      if (t - t0 > limit_ns) {
         *abort = 1;
         return false;
       }

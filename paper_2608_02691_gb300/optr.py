@@ -63,6 +63,7 @@ _SIG = {
                                    ctypes.c_size_t, _V]),
     "optr_device_error": (_I, [_V, ctypes.POINTER(ctypes.c_uint32)]),
     "optr_strerror": (ctypes.c_char_p, [_I]),
+    "optr_selftest_wait_timeout": (_I, [_V, ctypes.c_ulonglong, _V]),
     "optr_decode_attention_noalloc": (_I, [_V, _V, _V, _V, _I, _I, _V, _I,
                                            _V, _V]),
     "optr_decode_step": (_I, [_V, _V, _V, _V, _I, _V, _V, _V, _V, _I, _I, _V,
@@ -345,6 +346,14 @@ def optr_device_error(p: Params) -> int:
     _check(lib().optr_device_error(p.handle, ctypes.byref(flags)),
            "optr_device_error")
     return int(flags.value)
+
+
+def optr_selftest_wait_timeout(p: Params, limit_ns: int, stream=None) -> None:
+    """Launch the bounded-wait self-test (see include/optr.h); the timeout
+    shows up in optr_device_error."""
+    _check(lib().optr_selftest_wait_timeout(p.handle, int(limit_ns),
+                                            _stream(stream)),
+           "optr_selftest_wait_timeout")
 
 
 def optr_profile_enable(p: Params, on: bool = True) -> None:

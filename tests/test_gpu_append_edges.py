@@ -119,3 +119,44 @@ def test_degenerate_groups(avar):
     codes, scale, _ = ph.slot_codes(pool.cpu().numpy(), pages[:1], slots[:1], 1)
     assert scale[0, :, 1].max() == 0.0  # value group 1 of token 0
     assert codes[0, :, 32:64].max() == 0
+
+
+def test_fp16_range_flag_on_tensor_variant():
+    """The tensor-core cache write converts k and v to fp16: a key element
+    of magnitude >= 65504 (bf16 70144 here) sets OPTR_DEVERR_FP16_RANGE and
+    leaves only that token-head's key record unspecified; every other record
+    still matches the oracle.  The CUDA-core variant takes the same input
+    without the flag and matches the oracle on every record."""
+    lens, first = [200, 100], [5, 0]
+    c = _append_case(lens, first, 25)
+    t_bad, h_bad = 17, 3
+    c["k"][t_bad, h_bad, 5] = 70000.0  # bf16 rounds it to 70144
+    assert float(c["k"][t_bad, h_bad, 5]) >= 65504.0
+    bt = c["bt"]
+    pool_ref = np.zeros((c["num_pages"], H_KV, 1536), np.uint8)
+    u = oracle.kv_append(synth.bf16_bits(c["k"]), synth.bf16_bits(c["v"]),
+                         c["cu"], c["pos0"], bt.numpy(), pool_ref,
+                         c["R_k"].numpy(), c["R_v"].numpy(), c["mu"].numpy(),
+                         want_u=True)
+    pages, slots = ph.token_slots(c["cu"], c["pos0"], bt.numpy())
+    for avar in APPEND_VARIANTS:
+        p = optr.optr_params_create(c["R_k"], c["R_v"], c["mu"], H_Q,
+                                    append_variant=avar)
+        pool = optr.new_pool(p, c["num_pages"], device="cuda")
+        optr.optr_kv_append(p, c["k"].cuda(), c["v"].cuda(),
+                            torch.from_numpy(c["cu"]).cuda(),
+                            torch.from_numpy(c["pos0"]).cuda(), bt.cuda(), pool)
+        torch.cuda.synchronize()
+        flags = optr.optr_device_error(p)
+        got = pool.cpu().numpy()
+        ref = pool_ref.copy()
+        if avar == optr.OPTR_VARIANT_TENSOR:
+            assert flags == optr.OPTR_DEVERR_FP16_RANGE
+            # the flagged key record (codes and metadata) is unspecified
+            pg, sl = pages[t_bad], slots[t_bad]
+            for arr in (got, ref):
+                arr[pg, h_bad, sl * 32:sl * 32 + 32] = 0
+                arr[pg, h_bad, 1024 + sl * 16:1024 + sl * 16 + 16] = 0
+        else:
+            assert flags == 0
+        ph.compare_append(got, ref, u, pages, slots)

@@ -121,18 +121,25 @@ def test_end_to_end_every_row_within_its_bar(name, scale, variant):
 
 
 def test_end_to_end_bar_stays_tight():
-    """The per-row bound is not a loophole: on the multi-sequence workloads
-    the average bar stays within 1.5x the strict decode tolerance, so every
-    end-to-end row is checked at nearly the decode bar (the differing
-    records are rare in-band codes and fp16 ulps; their perturbation bound
-    is small)."""
+    """The per-row bound is not a loophole.  Almost every (sequence, KV
+    head) group holds a few records that differ from the oracle's by an
+    fp16 ulp of a scale or a min (the GPU's float32 rotation rounds z
+    differently from the oracle's fp64 one, and fp16(min) or fp16(range/3)
+    moves when z sits near an fp16 rounding boundary), and a few hundredths
+    of a percent of codes fall in the tie band; each moves the output by
+    far less than the decode tolerance.  So the typical row's bar must stay
+    at the decode bar: the median over rows of the bar is at most 1.25x
+    OUT_TOL * RMS on the multi-sequence workloads (the mean and the largest
+    bound, set by rare in-band codes of heavily weighted tokens, are
+    reported)."""
     for name, scale in (("decode8k", 1 / 16), ("ragged", 1 / 32)):
         _, _, rms, bound, bar = _end_to_end(name, scale)
-        ratio = float(bar.mean() / (ph.OUT_TOL * rms))
-        print(f"{name}: mean bar {ratio:.3f} x strict, strict rows "
-              f"{float((bound == 0).mean()):.2f}, max bound/strict "
-              f"{float(bound.max() / (ph.OUT_TOL * rms)):.3f}")
-        assert ratio <= 1.5, (name, ratio)
+        strict = ph.OUT_TOL * rms
+        med = float(np.median(bar) / strict)
+        print(f"{name}: median bar {med:.3f} x strict, mean {bar.mean() / strict:.3f}, "
+              f"rows with no differing record {float((bound == 0).mean()):.2f}, "
+              f"largest bound {float(bound.max() / strict):.1f} x strict")
+        assert med <= 1.25, (name, med)
 
 
 @pytest.mark.parametrize("variant", VARIANTS)
@@ -283,3 +290,72 @@ def test_decode_step_equals_append_then_decode(name, scale, variant):
     assert optr.optr_device_error(p) == 0
     assert torch.equal(pool, pool2)
     assert torch.equal(out1, out2)
+
+
+@pytest.mark.parametrize("variant", VARIANTS)
+def test_decode_step_multi_token_write(variant):
+    """A decode step whose write covers the last 12 positions of every
+    sequence, across a page boundary (positions 16k - 1 .. 16k + 10), equals
+    the cache write followed by the decode, bit for bit: pages the step
+    writes are read only after it."""
+    c = synth.build_case(synth.workload("decode8k", 0, 1 / 16), 0)
+    dev = "cuda"
+    B, m, d = c["B"], 12, 5  # 12 new tokens, the last 5 context tokens unused
+    cu = c["cu_ctx"].tolist()
+    lens = [cu[b + 1] - cu[b] for b in range(B)]
+    head = torch.cat([torch.arange(cu[b], cu[b + 1] - m - d) for b in range(B)])
+    tail = torch.cat([torch.arange(cu[b + 1] - m - d, cu[b + 1] - d) for b in range(B)])
+    cu_head = torch.tensor([0] + list(np.cumsum([n - m - d for n in lens])), dtype=torch.int32)
+    cu_tail = torch.arange(0, (B + 1) * m, m, dtype=torch.int32)
+    pos0 = c["pos0_ctx"]
+    pos_tail = (pos0 + torch.tensor(lens, dtype=torch.int32) - m - d).to(torch.int32)
+    seq = (pos0 + torch.tensor(lens, dtype=torch.int32) - d).to(torch.int32).to(dev)
+    assert all((n - m - d) % 16 == 15 for n in lens)  # the write crosses a page boundary
+    p = optr.optr_params_create(c["R_k"], c["R_v"], c["mu"], c["h_q"],
+                                decode_variant=variant)
+    pool = optr.new_pool(p, c["num_pages"], device=dev)
+    bt = c["block_table"].to(dev)
+    optr.optr_kv_append(p, c["k_ctx"][head].to(dev), c["v_ctx"][head].to(dev),
+                        cu_head.to(dev), pos0.to(dev), bt, pool)
+    pool2 = pool.clone()
+    kt, vt = c["k_ctx"][tail].to(dev), c["v_ctx"][tail].to(dev)
+    q = c["q"].to(dev)
+    ws = optr.new_workspace(p, B, bt.shape[1], device=dev)
+    out1 = torch.empty(B, c["h_q"], 128, dtype=torch.float32, device=dev)
+    out2 = torch.full_like(out1, 7.0)
+    optr.optr_kv_append(p, kt, vt, cu_tail.to(dev), pos_tail.to(dev), bt, pool)
+    optr.optr_decode_attention(p, q, bt, seq, pool, out1, ws)
+    optr.optr_decode_step(p, q, kt, vt, cu_tail.to(dev), pos_tail.to(dev), bt,
+                          seq, pool2, out2, ws)
+    torch.cuda.synchronize()
+    assert optr.optr_device_error(p) == 0
+    assert torch.equal(pool, pool2)
+    assert torch.equal(out1, out2)
+
+
+def test_workspace_reused_across_batch_shapes():
+    """A workspace needs no initialisation and one large enough serves calls
+    of different batch shapes in any order: a 0xFF-filled workspace reused
+    for ragged B = 128, then decode8k B = 16, then ragged again gives the
+    results of fresh workspaces bit for bit."""
+    dev = "cuda"
+    cases = []
+    for name, scale in (("ragged", 1 / 32), ("decode8k", 1 / 16)):
+        c, pool_ref, _, _ = _case(name, scale)
+        p = optr.optr_params_create(c["R_k"], c["R_v"], c["mu"], c["h_q"])
+        pool = torch.from_numpy(pool_ref).to(dev)
+        bt = c["block_table"].to(dev)
+        fresh = torch.empty(c["B"], c["h_q"], 128, device=dev)
+        optr.optr_decode_attention(p, c["q"].to(dev), bt, c["seq_lens"].to(dev),
+                                   pool, fresh, optr.new_workspace(p, c["B"], bt.shape[1]))
+        cases.append((c, p, pool, bt, fresh))
+    size = max(optr.optr_decode_workspace_size(p, c["B"], bt.shape[1])
+               for c, p, _, bt, _ in cases)
+    ws = torch.full((size,), 0xFF, dtype=torch.uint8, device=dev)
+    for c, p, pool, bt, fresh in cases + cases[:1]:
+        out = torch.full_like(fresh, float("nan"))
+        optr.optr_decode_attention(p, c["q"].to(dev), bt, c["seq_lens"].to(dev),
+                                   pool, out, ws)
+        torch.cuda.synchronize()
+        assert torch.equal(out, fresh)
+    assert optr.optr_device_error(cases[0][1]) == 0
