@@ -54,7 +54,12 @@ def rotation(R0: torch.Tensor, A: torch.Tensor) -> torch.Tensor:
 
 
 def _f16(x: torch.Tensor) -> torch.Tensor:
-    return x.to(torch.float16).to(F64)
+    """The stored fp16 value of a float64 scale or min: rounded to float32,
+    then to fp16 (both round-to-nearest-even), as the cache's quantizer
+    stores the fp16 value of its float32 range.  Spelled out because a
+    direct float64 -> fp16 conversion rounds once and can differ by an
+    fp16 ulp."""
+    return x.to(torch.float32).to(torch.float16).to(F64)
 
 
 class Q2STE(torch.autograd.Function):
