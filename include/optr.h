@@ -140,6 +140,7 @@ typedef enum {
 #define OPTR_DEVERR_FP16_RANGE 16u /* tensor-core append: |k| or |v| >= 65504 */
 #define OPTR_DEVERR_TIMEOUT 32u  /* internal: a kernel's bounded wait gave up */
 #define OPTR_DEVERR_WIN_SLOT 64u /* window slot of a sequence < 0 or >= n_slots */
+#define OPTR_DEVERR_CALIB_RANGE 128u /* calibration: generator norm past exp's scaling range */
 
 /* Kernel variants (for measurement; 0 picks the library default). */
 #define OPTR_VARIANT_DEFAULT 0
@@ -394,6 +395,85 @@ optr_status optr_decode_step_win(const optr_params* p, const void* q,
 
 /* Static description of a status code. */
 const char* optr_strerror(optr_status s);
+
+/*
+ * Offline rotation calibration of one KV head (Sec. 4.2 "Orthogonal
+ * Rotation Refinement", Sec. 4.3 output-aware key objective, Sec. 4.4 value
+ * objective, Sec. 4.5 INT2-aware calibration with the straight-through
+ * estimator; Appendix, "OptR Algorithm"; Sec. 5: 80 Adam steps, lr 0.02,
+ * held-out selection every 20 steps).  It produces the R_k[h], R_v[h] and
+ * mu[h] that optr_params_create takes.  With d = 128, scale = 1/sqrt(d):
+ *   mu      = mean over the calibration trace's keys
+ *   R_K     = R0_K exp(A_K - A_K^T),  R_V = R0_V exp(A_V - A_V^T)
+ *   keys    kt_s = Q2((k_s - mu) R_K, clip_k) R_K^T   (window pairs: k_s - mu)
+ *   values  vt_s = Q2(v_s R_V, clip_v) R_V^T          (window pairs: v_s)
+ *   p_t     = softmax_{s <= t}(scale q_t . k_s),  p^K_t the same on kt
+ *   L_K     = mean_{t,j} [KL(p_t || p^K_t)
+ *                         + lam |((p^K_t - p_t) V) W_O[j]^T|^2 / d_model]
+ *   L_V     = mean_{t,j} |(phat_t (Vt - V)) W_O[j]^T|^2 / d_model,
+ *             phat the key attention under the selected R_K
+ * with Q2 the cache's quantizer (group cfg.group, fp16 scale and min taken
+ * from the float32 rounding of the float64 values) and its gradient the
+ * indicator of the clipped range [c min, c max] of the value's group.  A
+ * position s is a BF16-window position for query position t when
+ * s < sink or s > t - recent.  Adam (b1 0.9, b2 0.999, eps 1e-8) runs
+ * `steps` steps on A_K from 0, scoring R_K on the held-out trace at step
+ * 0, every select_every steps and after the last step and keeping the best;
+ * then the same for A_V under the selected R_K.  Float64 throughout, on the
+ * GPU; the gradient is written out (Frechet derivative of the matrix
+ * exponential from a Taylor series with scaling and squaring).
+ *
+ * All arrays are device float64 (int32 positions), row-major:
+ *   q [nt][g][128] (the g query heads of the KV head at query positions
+ *   t_pos[nt], each in 0 .. T-1), K, V [T][128], W_O [g][d_model][128]
+ *   (W_O[j] maps query head j's output to the model); the held-out trace
+ *   likewise with T_held / nt_held (T_held = 0: scored on the calibration
+ *   trace, pointers may be NULL); R0_K, R0_V [128][128] or NULL for the
+ *   normalised Hadamard matrix.  Outputs R_K, R_V [128][128], mu [128],
+ *   hist_k, hist_v [steps] (the training loss before each step).
+ * The workspace (optr_calib_workspace_size bytes, 256-byte aligned) is
+ * scratch.  The call enqueues its kernels on `stream` and synchronises it
+ * before returning; OPTR_ERR_OUT_OF_RANGE reports a generator whose norm
+ * left the exponential's scaling range (|A - A^T| above 2^15).
+ */
+typedef struct {
+  int g;              /* query heads of the KV head (1 .. 64)                */
+  int d_model;        /* rows of each W_O[j]                                 */
+  int T, nt;          /* calibration trace: tokens, query positions          */
+  int T_held, nt_held;/* held-out trace; T_held = 0: none                    */
+  int steps;          /* Adam steps per rotation (paper: 80)                 */
+  int select_every;   /* held-out selection period (paper: 20)               */
+  int group;          /* Q2 group size: 32 or 128                            */
+  int sink, recent;   /* BF16 windows (0, 0: none)                           */
+  double lr, lam;     /* Adam learning rate (0.02), key-loss lambda          */
+  double clip_k, clip_v; /* Q2 clipping ratios in (0, 1]                     */
+} optr_calib_config;
+
+/* Workspace bytes of optr_calibrate_head / optr_calib_loss_grad for this
+ * configuration, or 0 when the configuration is invalid. */
+size_t optr_calib_workspace_size(const optr_calib_config* c);
+
+optr_status optr_calibrate_head(
+    const optr_calib_config* c, const double* q, const double* K,
+    const double* V, const int32_t* t_pos, const double* W_O,
+    const double* q_held, const double* K_held, const double* V_held,
+    const int32_t* t_pos_held, const double* R0_K, const double* R0_V,
+    double* R_K, double* R_V, double* mu, double* hist_k, double* hist_v,
+    void* workspace, size_t ws_bytes, cudaStream_t stream);
+
+/* One evaluation of the objective on the calibration trace (held-out
+ * fields unused): which = 0, L_K at R_K = R0 exp(A - A^T); which = 1, L_V at
+ * R_V = R0 exp(A - A^T) under the key rotation R_K.  mu is given.  Writes
+ * the loss (device double) and, when dA is not NULL, its gradient with
+ * respect to A (device [128][128]).  Synchronises the stream. */
+optr_status optr_calib_loss_grad(const optr_calib_config* c, int which,
+                                 const double* q, const double* K,
+                                 const double* V, const int32_t* t_pos,
+                                 const double* W_O, const double* mu,
+                                 const double* R_K, const double* R0,
+                                 const double* A, double* loss, double* dA,
+                                 void* workspace, size_t ws_bytes,
+                                 cudaStream_t stream);
 
 /*
  * Self-test of the bounded waits (library machinery; the paper has no

@@ -50,6 +50,17 @@ class optr_config(ctypes.Structure):
                 ("recent", ctypes.c_int)]
 
 
+class optr_calib_config(ctypes.Structure):
+    _fields_ = [("g", ctypes.c_int), ("d_model", ctypes.c_int),
+                ("T", ctypes.c_int), ("nt", ctypes.c_int),
+                ("T_held", ctypes.c_int), ("nt_held", ctypes.c_int),
+                ("steps", ctypes.c_int), ("select_every", ctypes.c_int),
+                ("group", ctypes.c_int), ("sink", ctypes.c_int),
+                ("recent", ctypes.c_int), ("lr", ctypes.c_double),
+                ("lam", ctypes.c_double), ("clip_k", ctypes.c_double),
+                ("clip_v", ctypes.c_double)]
+
+
 _V = ctypes.c_void_p
 _I = ctypes.c_int
 _SIG = {
@@ -64,6 +75,11 @@ _SIG = {
     "optr_device_error": (_I, [_V, ctypes.POINTER(ctypes.c_uint32)]),
     "optr_strerror": (ctypes.c_char_p, [_I]),
     "optr_selftest_wait_timeout": (_I, [_V, ctypes.c_ulonglong, _V]),
+    "optr_calib_workspace_size": (ctypes.c_size_t, [ctypes.POINTER(optr_calib_config)]),
+    "optr_calibrate_head": (_I, [ctypes.POINTER(optr_calib_config)] + [_V] * 17
+                            + [ctypes.c_size_t, _V]),
+    "optr_calib_loss_grad": (_I, [ctypes.POINTER(optr_calib_config), _I] + [_V] * 12
+                             + [ctypes.c_size_t, _V]),
     "optr_decode_attention_noalloc": (_I, [_V, _V, _V, _V, _I, _I, _V, _I,
                                            _V, _V]),
     "optr_decode_step": (_I, [_V, _V, _V, _V, _I, _V, _V, _V, _V, _I, _I, _V,
@@ -377,3 +393,62 @@ def new_pool(p: Params, num_pages: int, device="cuda") -> torch.Tensor:
 def new_workspace(p: Params, B: int, max_pages: int, device="cuda"):
     n = optr_decode_workspace_size(p, B, max_pages)
     return torch.empty(n, dtype=torch.uint8, device=device)
+
+
+# ------------------------------------------------------------ calibration
+
+def calib_config(g, d_model, T, nt, T_held=0, nt_held=0, steps=80,
+                 select_every=20, group=32, sink=0, recent=0, lr=0.02, lam=1.0,
+                 clip_k=1.0, clip_v=1.0) -> optr_calib_config:
+    return optr_calib_config(g, d_model, T, nt, T_held, nt_held, steps,
+                             select_every, group, sink, recent, lr, lam, clip_k,
+                             clip_v)
+
+
+def optr_calib_workspace_size(cfg: optr_calib_config) -> int:
+    return int(lib().optr_calib_workspace_size(ctypes.byref(cfg)))
+
+
+def _calib_ws(cfg, device):
+    n = optr_calib_workspace_size(cfg)
+    if n == 0:
+        raise OptrError(-1, "optr_calib_workspace_size")
+    return torch.empty(n, dtype=torch.uint8, device=device)
+
+
+def optr_calibrate_head(cfg: optr_calib_config, q, K, V, t_pos, W_O,
+                        held=None, R0_K=None, R0_V=None, stream=None):
+    """One KV head's calibration (see include/optr.h).  q [nt][g][128],
+    K, V [T][128], W_O [g][d_model][128] float64 CUDA tensors, t_pos int32;
+    held = (q, K, V, t_pos) of the held-out trace or None.  Returns R_K,
+    R_V, mu, hist_k, hist_v (CUDA float64)."""
+    dev = K.device
+    d = 128
+    R_K = torch.empty(d, d, dtype=torch.float64, device=dev)
+    R_V = torch.empty_like(R_K)
+    mu = torch.empty(d, dtype=torch.float64, device=dev)
+    hk = torch.empty(max(cfg.steps, 1), dtype=torch.float64, device=dev)
+    hv = torch.empty_like(hk)
+    ws = _calib_ws(cfg, dev)
+    h = held if held is not None else (None, None, None, None)
+    _check(lib().optr_calibrate_head(
+        ctypes.byref(cfg), _ptr(q), _ptr(K), _ptr(V), _ptr(t_pos), _ptr(W_O),
+        _ptr(h[0]), _ptr(h[1]), _ptr(h[2]), _ptr(h[3]), _ptr(R0_K), _ptr(R0_V),
+        _ptr(R_K), _ptr(R_V), _ptr(mu), _ptr(hk), _ptr(hv), _ptr(ws),
+        ws.numel(), _stream(stream)), "optr_calibrate_head")
+    return R_K, R_V, mu, hk[:cfg.steps], hv[:cfg.steps]
+
+
+def optr_calib_loss_grad(cfg: optr_calib_config, which: int, q, K, V, t_pos,
+                         W_O, mu, R0, A, R_K=None, grad=True, stream=None):
+    """L_K (which 0) or L_V (which 1) at R = R0 exp(A - A^T) and its
+    gradient with respect to A (None when grad is False)."""
+    dev = K.device
+    loss = torch.empty(1, dtype=torch.float64, device=dev)
+    dA = torch.empty(128, 128, dtype=torch.float64, device=dev) if grad else None
+    ws = _calib_ws(cfg, dev)
+    _check(lib().optr_calib_loss_grad(
+        ctypes.byref(cfg), int(which), _ptr(q), _ptr(K), _ptr(V), _ptr(t_pos),
+        _ptr(W_O), _ptr(mu), _ptr(R_K), _ptr(R0), _ptr(A), _ptr(loss), _ptr(dA),
+        _ptr(ws), ws.numel(), _stream(stream)), "optr_calib_loss_grad")
+    return loss, dA

@@ -25,6 +25,7 @@ matrix, with column signs fixed so that diag(R_qr) > 0.
 """
 from __future__ import annotations
 
+import math
 from dataclasses import dataclass, field
 
 import torch
@@ -247,3 +248,22 @@ def build_case(wl: Workload, seed: int = 0, device="cpu") -> dict:
 def bf16_bits(t: torch.Tensor):
     """Raw uint16 bit patterns of a bf16 tensor as a numpy array (CPU)."""
     return t.detach().cpu().contiguous().view(torch.int16).numpy().view("uint16")
+
+
+def calib_trace(seed: int, T: int, nt: int, g: int = 4, d_model: int = 64,
+                device="cpu"):
+    """A synthetic calibration trace of one KV head, float64 (stands in for
+    the paper's BF16 GPQA Q/K/V traces): keys Student-t(4) with the 4
+    offset channels of key_offsets() (head 0 of ``seed``), values
+    Student-t(4), the g query heads ~ N(0, 1) at the last nt positions, and
+    a random output projection W_O [g][d_model][128] ~ N(0, 1/(g*128)).
+    Returns q [nt][g][128], K, V [T][128], W_O, t_pos int32 [nt]."""
+    gen = _gen(seed * 7919 + 17, "cpu")
+    K = _draw(T * D, "t4", gen, "cpu").view(T, D).to(torch.float64)
+    K += key_offsets(1, seed)[0].to(torch.float64)
+    V = _draw(T * D, "t4", gen, "cpu").view(T, D).to(torch.float64)
+    q = torch.randn(nt, g, D, generator=gen, dtype=torch.float64)
+    W_O = torch.randn(g, d_model, D, generator=gen, dtype=torch.float64) / math.sqrt(g * D)
+    t_pos = torch.arange(T - nt, T, dtype=torch.int32)
+    return (q.to(device), K.to(device), V.to(device), W_O.to(device),
+            t_pos.to(device))
