@@ -436,6 +436,81 @@ def extra_workloads(args, dev):
                      "partial_frac": round(sb / (part * 1e-3) / 1e9 / hbm_peak, 4)}
         del pool, case
         torch.cuda.empty_cache()
+    res["calibration"] = calibration_workload(args, dev)
+    return res
+
+
+def calib_flops(T, nt, g, dm, steps, every, held=True):
+    """Float64 FLOPs of optr_calibrate_head counted from its GEMM shapes
+    (2 M N K each): per Adam step the forward and backward GEMMs of the
+    objective, the rotation's exp (18 Horner products) and the Frechet
+    derivative (3 per Horner step); squarings, whose count the device
+    decides, are left out, so this is a lower bound."""
+    d = 128
+    key_f = 4 * T * d * d + 4 * g * nt * T * d + 2 * g * nt * d * dm
+    key_b = 2 * g * nt * dm * d + 4 * g * nt * T * d + 6 * T * d * d
+    val_f = 4 * T * d * d + 2 * g * nt * T * d + 2 * g * nt * d * dm
+    val_b = 2 * g * nt * dm * d + 2 * g * nt * T * d + 6 * T * d * d
+    rot = 19 * 2 * d ** 3
+    grad = (3 * 18 + 1) * 2 * d ** 3
+    n_sel = steps // every + (1 if steps % every else 0) + 1
+    setup = 2 * (2 * g * nt * T * d) + 2 * key_f
+    return (setup + steps * (key_f + key_b + val_f + val_b + 2 * (rot + grad))
+            + n_sel * (key_f + val_f) + 2 * (steps + 1) * rot)
+
+
+def calibration_workload(args, dev):
+    """One KV head's calibration at the paper's scale (Sec. 5 and the
+    appendix: ~2.7k-token traces, the objective over the final 64 query
+    positions, 80 Adam steps, selection every 20 steps): a 2048-token
+    synthetic trace and a held-out one of the same size, 4 query heads,
+    d_model 4096 (Qwen3-8B), G = 128, clips 0.96 / 0.92, windows 64 / 256.
+    The oracle is timed on one forward + backward of L_K at the same size."""
+    from paper_2608_02691_gb300 import optr, synth
+    T, nt, g, dm, steps, every = 2048, 64, 4, 4096, 80, 20
+    tr = synth.calib_trace(args.seed, T, nt, g, dm)
+    ho = synth.calib_trace(args.seed + 1, T, nt, g, dm)
+    cfg = optr.calib_config(g, dm, T, nt, T, nt, steps=steps, select_every=every,
+                            group=128, sink=64, recent=256, lr=0.02, lam=1.0,
+                            clip_k=0.96, clip_v=0.92)
+    q, K, V, W, tp = [x.to(dev) for x in tr]
+    hd = tuple(x.to(dev) for x in (ho[0], ho[1], ho[2], ho[4]))
+    optr.optr_calibrate_head(cfg, q, K, V, tp, W, held=hd)  # warm-up
+    t = []
+    for _ in range(2):
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record()
+        optr.optr_calibrate_head(cfg, q, K, V, tp, W, held=hd)
+        e1.record()
+        torch.cuda.synchronize()
+        t.append(e0.elapsed_time(e1) * 1e-3)
+    sec = float(np.mean(t))
+    flops = calib_flops(T, nt, g, dm, steps, every)
+    gf = flops / sec / 1e9
+    res = {"trace_tokens": T, "query_positions": nt, "query_heads": g,
+           "d_model": dm, "steps": steps, "s_per_head": round(sec, 4),
+           "qwen3_8b_all_heads_s": round(sec * 36 * 8, 1),
+           "roofline": {"bound": "alu", "unit": "GFLOP/s", "dtype": "f64",
+                        "achieved_lower_bound": round(gf, 1), "peak": 1250.0,
+                        "peak_source": "nominal GB300 FP64 (not measured)",
+                        "frac": round(gf / 1250.0, 4)}}
+    if not args.no_cpu:
+        import time
+        from oracle import calibration as cal
+        qc, Kc, Vc, Wc, tc = tr
+        mu = Kc.mean(0)
+        A = torch.zeros(128, 128, dtype=torch.float64, requires_grad=True)
+        t0 = time.perf_counter()
+        L = cal.key_loss(qc, Kc, Vc, mu, cal.rotation(cal.hadamard(128), A), Wc,
+                         tc.long(), 1.0, 0.96, 128, 64, 256)
+        torch.autograd.grad(L, A)
+        st = time.perf_counter() - t0
+        res["oracle"] = {"s_per_key_step": round(st, 3),
+                         "cores": torch.get_num_threads(),
+                         "s_per_head_est": round(st * 2 * steps, 1),
+                         "sample": "one L_K forward + backward at the same size; "
+                                   "per-head estimate = 160 such steps"}
     return res
 
 

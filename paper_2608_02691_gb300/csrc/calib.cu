@@ -26,6 +26,7 @@
 #include <math.h>
 #include <string.h>
 
+#include <algorithm>
 #include <vector>
 
 #include "optr_internal.cuh"
@@ -58,19 +59,26 @@ struct Gemm {
   const double* pass;
 };
 
-constexpr int kTM = 64, kTN = 64, kTK = 16;
+constexpr int kTK = 16;
 
-__global__ void __launch_bounds__(256) gemm_f64_kernel(Gemm g) {
-  __shared__ double As[kTK][kTM + 1];
-  __shared__ double Bs[kTK][kTN + 1];
-  const int b = blockIdx.z;
-  const int m0 = blockIdx.y * kTM, n0 = blockIdx.x * kTN;
+// TILE x TILE outputs per CTA of 256 threads ((TILE / 16)^2 outputs each).
+// The host picks the largest tile, then a split of K into kc chunks, so that
+// a call covers about two CTAs per SM (float64 runs at a few FMAs per clock
+// per SM on this GPU).  With kc > 1 chunk z of a product writes its raw sum
+// to P[z][b] and gemm_f64_reduce_kernel adds the chunks in a fixed order.
+template <int TILE>
+__global__ void __launch_bounds__(256) gemm_f64_kernel(Gemm g, int kc, double* P) {
+  constexpr int R = TILE / 16;  // outputs per thread per dimension
+  __shared__ double As[kTK][TILE + 1];
+  __shared__ double Bs[kTK][TILE + 1];
+  const int b = blockIdx.z / kc, z = blockIdx.z % kc;
+  const int m0 = blockIdx.y * TILE, n0 = blockIdx.x * TILE;
   const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
   double* C = g.C + (long long)b * g.sC;
   if (g.gate != nullptr && g.gate_idx >= *g.gate) {
-    if (g.pass != nullptr) {
-      for (int i = tid; i < kTM * kTN; i += 256) {
-        const int r = m0 + i / kTN, c = n0 + i % kTN;
+    if (g.pass != nullptr && kc == 1) {
+      for (int i = tid; i < TILE * TILE; i += 256) {
+        const int r = m0 + i / TILE, c = n0 + i % TILE;
         if (r < g.M && c < g.N) C[r * g.ldc + c] = g.pass[r * g.ldc + c];
       }
     }
@@ -78,56 +86,91 @@ __global__ void __launch_bounds__(256) gemm_f64_kernel(Gemm g) {
   }
   const double* A = g.A + (long long)b * g.sA;
   const double* B = g.B + (long long)b * g.sB;
-  double acc[4][4];
+  // this CTA's K range: chunk z of kc, in whole kTK slices
+  const int nsl = (g.K + kTK - 1) / kTK;
+  const int kb = (int)((long long)z * nsl / kc) * kTK;
+  const int ke = min(g.K, (int)((long long)(z + 1) * nsl / kc) * kTK);
+  double acc[R][R];
 #pragma unroll
-  for (int i = 0; i < 4; ++i)
+  for (int i = 0; i < R; ++i)
 #pragma unroll
-    for (int j = 0; j < 4; ++j) acc[i][j] = 0.0;
-  for (int k0 = 0; k0 < g.K; k0 += kTK) {
-    for (int i = tid; i < kTM * kTK; i += 256) {
+    for (int j = 0; j < R; ++j) acc[i][j] = 0.0;
+  for (int k0 = kb; k0 < ke; k0 += kTK) {
+    for (int i = tid; i < TILE * kTK; i += 256) {
       int mm, kk;
-      if (g.tA) { kk = i / kTM; mm = i % kTM; } else { mm = i / kTK; kk = i % kTK; }
+      if (g.tA) { kk = i / TILE; mm = i % TILE; } else { mm = i / kTK; kk = i % kTK; }
       const int gm = m0 + mm, gk = k0 + kk;
       double x = 0.0;
-      if (gm < g.M && gk < g.K) x = g.tA ? A[gk * g.lda + gm] : A[gm * g.lda + gk];
+      if (gm < g.M && gk < ke) x = g.tA ? A[gk * g.lda + gm] : A[gm * g.lda + gk];
       As[kk][mm] = x;
     }
-    for (int i = tid; i < kTK * kTN; i += 256) {
+    for (int i = tid; i < kTK * TILE; i += 256) {
       int kk, nn;
-      if (g.tB) { nn = i / kTK; kk = i % kTK; } else { kk = i / kTN; nn = i % kTN; }
+      if (g.tB) { nn = i / kTK; kk = i % kTK; } else { kk = i / TILE; nn = i % TILE; }
       const int gk = k0 + kk, gn = n0 + nn;
       double x = 0.0;
-      if (gk < g.K && gn < g.N) x = g.tB ? B[gn * g.ldb + gk] : B[gk * g.ldb + gn];
+      if (gk < ke && gn < g.N) x = g.tB ? B[gn * g.ldb + gk] : B[gk * g.ldb + gn];
       Bs[kk][nn] = x;
     }
     __syncthreads();
 #pragma unroll
     for (int kk = 0; kk < kTK; ++kk) {
-      double a[4], bb[4];
+      double a[R], bb[R];
 #pragma unroll
-      for (int i = 0; i < 4; ++i) a[i] = As[kk][ty * 4 + i];
+      for (int i = 0; i < R; ++i) a[i] = As[kk][ty * R + i];
 #pragma unroll
-      for (int j = 0; j < 4; ++j) bb[j] = Bs[kk][tx * 4 + j];
+      for (int j = 0; j < R; ++j) bb[j] = Bs[kk][tx * R + j];
 #pragma unroll
-      for (int i = 0; i < 4; ++i)
+      for (int i = 0; i < R; ++i)
 #pragma unroll
-        for (int j = 0; j < 4; ++j) acc[i][j] = fma(a[i], bb[j], acc[i][j]);
+        for (int j = 0; j < R; ++j) acc[i][j] = fma(a[i], bb[j], acc[i][j]);
     }
     __syncthreads();
   }
 #pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const int r = m0 + ty * 4 + i;
+  for (int i = 0; i < R; ++i) {
+    const int r = m0 + ty * R + i;
     if (r >= g.M) continue;
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const int c = n0 + tx * 4 + j;
+    for (int j = 0; j < R; ++j) {
+      const int c = n0 + tx * R + j;
       if (c >= g.N) continue;
+      if (kc > 1) {
+        P[(((long long)z * gridDim.z / kc + b) * g.M + r) * g.N + c] = acc[i][j];
+        continue;
+      }
       double x = g.alpha * acc[i][j];
       if (g.beta != 0.0) x += g.beta * C[r * g.ldc + c];
       if (r == c) x += g.diag;
       C[r * g.ldc + c] = x;
     }
+  }
+}
+
+// C[b] = alpha sum_z P[z][b] + beta C[b] + diag I (the chunks in order).
+__global__ void gemm_f64_reduce_kernel(Gemm g, int kc, int batch, const double* P) {
+  const long long mn = (long long)g.M * g.N;
+  if (g.gate != nullptr && g.gate_idx >= *g.gate) {
+    if (g.pass == nullptr) return;
+    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < mn * batch;
+         i += (long long)gridDim.x * blockDim.x) {
+      const long long b = i / mn, e = i % mn;
+      const int r = (int)(e / g.N), c = (int)(e % g.N);
+      g.C[b * g.sC + r * g.ldc + c] = g.pass[r * g.ldc + c];
+    }
+    return;
+  }
+  for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < mn * batch;
+       i += (long long)gridDim.x * blockDim.x) {
+    const long long b = i / mn, e = i % mn;
+    const int r = (int)(e / g.N), c = (int)(e % g.N);
+    double s = 0.0;
+    for (int z = 0; z < kc; ++z) s += P[((long long)z * batch + b) * mn + e];
+    double* C = g.C + b * g.sC + r * g.ldc + c;
+    double x = g.alpha * s;
+    if (g.beta != 0.0) x += g.beta * *C;
+    if (r == c) x += g.diag;
+    *C = x;
   }
 }
 
@@ -250,18 +293,32 @@ __global__ void q2_kernel(const double* __restrict__ Z, int rows, int G,
 // Row (j, t) of [g][nt][T]: logits scale * x (x = the row of X, or of Xc
 // at the BF16-window pairs when windows), masked to s <= t_pos[t]; the
 // softmax goes to P.  When Pref is given, rowv[row] = KL(Pref || P) =
-// sum_s pref (logpref - log max(p, 1e-300)).  One warp per row.
-__global__ void softmax_rows_kernel(const double* __restrict__ X,
-                                    const double* __restrict__ Xc, int rows,
-                                    int nt, int T, const int32_t* __restrict__ t_pos,
-                                    double scale, int sink, int recent,
-                                    double* __restrict__ P,
-                                    const double* __restrict__ Pref,
-                                    const double* __restrict__ logPref,
-                                    double* __restrict__ rowv) {
-  const int lane = threadIdx.x & 31;
-  const long long row = (blockIdx.x * (long long)blockDim.x + threadIdx.x) >> 5;
-  if (row >= rows) return;
+// sum_s pref (logpref - log max(p, 1e-300)), with log p = l - m - log(sum)
+// (p = 0 entries: log 1e-300; below 1e-300 the clamp).  One block of 256
+// threads per row; exp(l - m) is stored in the sum pass and normalised in
+// the last.
+__device__ __forceinline__ double block_reduce(double v, bool is_max, double* sh) {
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const double u = __shfl_xor_sync(0xffffffffu, v, o);
+    v = is_max ? fmax(v, u) : v + u;
+  }
+  __syncthreads();  // sh free from an earlier reduction
+  if (lane == 0) sh[w] = v;
+  __syncthreads();
+  double r = sh[0];
+  for (int i = 1; i < 8; ++i) r = is_max ? fmax(r, sh[i]) : r + sh[i];
+  return r;
+}
+
+__global__ void __launch_bounds__(256) softmax_rows_kernel(
+    const double* __restrict__ X, const double* __restrict__ Xc, int rows, int nt,
+    int T, const int32_t* __restrict__ t_pos, double scale, int sink, int recent,
+    double* __restrict__ P, const double* __restrict__ Pref,
+    const double* __restrict__ logPref, double* __restrict__ rowv) {
+  __shared__ double sh[8];
+  const long long row = blockIdx.x;
   const int t = t_pos[row % nt];
   const bool win = Xc != nullptr;
   const double* x = X + row * (long long)T;
@@ -271,29 +328,30 @@ __global__ void softmax_rows_kernel(const double* __restrict__ X,
     return v * scale;
   };
   double m = -INFINITY;
-  for (int s = lane; s < T; s += 32)
+  for (int s = threadIdx.x; s < T; s += 256)
     if (s <= t) m = fmax(m, logit(s));
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) m = fmax(m, __shfl_xor_sync(0xffffffffu, m, o));
-  double sum = 0.0;
-  for (int s = lane; s < T; s += 32)
-    if (s <= t) sum += exp(logit(s) - m);
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+  m = block_reduce(m, true, sh);
   double* p = P + row * (long long)T;
+  double sum = 0.0;
+  for (int s = threadIdx.x; s < T; s += 256) {
+    const double e = s <= t ? exp(logit(s) - m) : 0.0;
+    p[s] = e;
+    sum += e;
+  }
+  sum = block_reduce(sum, false, sh);
+  const double lsum = Pref != nullptr ? log(sum) : 0.0;
   double kl = 0.0;
-  for (int s = lane; s < T; s += 32) {
-    const double v = s <= t ? exp(logit(s) - m) / sum : 0.0;
+  for (int s = threadIdx.x; s < T; s += 256) {
+    const double v = p[s] / sum;
     p[s] = v;
     if (Pref != nullptr) {
-      const double pr = Pref[row * (long long)T + s];
-      kl += pr * (logPref[row * (long long)T + s] - log(fmax(v, 1e-300)));
+      const double lp = v > 1e-300 ? (logit(s) - m) - lsum : log(1e-300);
+      kl += Pref[row * (long long)T + s] * (logPref[row * (long long)T + s] - lp);
     }
   }
   if (Pref != nullptr) {
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) kl += __shfl_xor_sync(0xffffffffu, kl, o);
-    if (lane == 0) rowv[row] = kl;
+    kl = block_reduce(kl, false, sh);
+    if (threadIdx.x == 0) rowv[row] = kl;
   }
 }
 
@@ -467,8 +525,12 @@ inline int nblk(long long n, int t = 256) {
   return (int)(b < 4096 ? (b > 0 ? b : 1) : 4096);
 }
 
+constexpr long long kGemmScratch = 1 << 21;  // split-K doubles (16 MiB)
+
 struct GemmCall {
   cudaStream_t s;
+  double* scratch;        // split-K partial sums
+  long long scratch_len;  // doubles
   void operator()(int M, int N, int K, const double* A, long long lda, bool tA,
                   const double* B, long long ldb, bool tB, double* C, long long ldc,
                   double alpha = 1.0, double beta = 0.0, int batch = 1,
@@ -477,8 +539,24 @@ struct GemmCall {
                   const double* pass = nullptr) const {
     Gemm g{M, N, K, A, lda, sA, tA ? 1 : 0, B, ldb, sB, tB ? 1 : 0, C, ldc, sC,
            alpha, beta, diag, gate, gate_idx, pass};
-    dim3 grid((N + kTN - 1) / kTN, (M + kTM - 1) / kTM, batch);
-    gemm_f64_kernel<<<grid, 256, 0, s>>>(g);
+    auto ctas = [&](int t) {
+      return (long long)((N + t - 1) / t) * ((M + t - 1) / t) * batch;
+    };
+    const int tile = ctas(64) >= 300 ? 64 : (ctas(32) >= 300 ? 32 : 16);
+    // split K when the output alone gives too few CTAs (chunks of >= 64)
+    int kc = 1;
+    while (kc < 64 && ctas(tile) * kc < 300 && K / (2 * kc) >= 64 &&
+           (long long)(2 * kc) * batch * M * N <= scratch_len)
+      kc *= 2;
+    const dim3 grid((N + tile - 1) / tile, (M + tile - 1) / tile, batch * kc);
+    if (tile == 64) gemm_f64_kernel<64><<<grid, 256, 0, s>>>(g, kc, scratch);
+    else if (tile == 32) gemm_f64_kernel<32><<<grid, 256, 0, s>>>(g, kc, scratch);
+    else gemm_f64_kernel<16><<<grid, 256, 0, s>>>(g, kc, scratch);
+    if (kc > 1) {
+      const long long n = (long long)batch * M * N;
+      const int blocks = (int)std::min<long long>((n + 255) / 256, 4096);
+      gemm_f64_reduce_kernel<<<blocks, 256, 0, s>>>(g, kc, batch, scratch);
+    }
   }
 };
 
@@ -511,7 +589,9 @@ struct Calib {
   int* s_dev;
   unsigned* err;
   const double* W;  // [g][d_model][d]
+  double* gsc;      // split-K scratch of the GEMMs
   cudaStream_t st;
+  GemmCall gemm() const { return GemmCall{st, gsc, kGemmScratch}; }
 };
 
 struct Layout {
@@ -558,6 +638,7 @@ size_t carve(Calib& C, char* base) {
   C.DV = L.take<double>(g * nm * D);
   C.U = L.take<double>(g * nm * D);
   C.E = L.take<double>(g * nm * c.d_model);
+  C.gsc = L.take<double>(kGemmScratch);
   double** dd[] = {&C.R0[0], &C.R0[1], &C.A, &C.m, &C.v, &C.dA, &C.S, &C.Xs,
                    &C.Hs, &C.T1[0], &C.T1[1], &C.T2[0], &C.T2[1], &C.R, &C.dR,
                    &C.dE, &C.best};
@@ -572,7 +653,7 @@ size_t carve(Calib& C, char* base) {
 // squarings ([[E, L], [0, E]]^2 = [[E E, E L + L E], [0, E E]]), s decided
 // on the device.
 int expm(Calib& C, const double* S, double sign, const double* H) {
-  GemmCall gm{C.st};
+  GemmCall gm = C.gemm();
   expm_prep_kernel<<<1, kCD, 0, C.st>>>(S, sign, H, C.Xs, C.Hs, C.s_dev, C.err);
   int cur = 0;
   eye_kernel<<<kCD, kCD, 0, C.st>>>(C.T1[0]);
@@ -607,12 +688,12 @@ int expm(Calib& C, const double* S, double sign, const double* H) {
 void rotation(Calib& C, const double* R0) {
   skew_kernel<<<kCD, kCD, 0, C.st>>>(C.A, C.S);
   const int e = expm(C, C.S, 1.0, nullptr);
-  GemmCall{C.st}(kCD, kCD, kCD, R0, kCD, false, C.T1[e], kCD, false, C.R, kCD);
+  C.gemm()(kCD, kCD, kCD, R0, kCD, false, C.T1[e], kCD, false, C.R, kCD);
 }
 
 // dA = dS - dS^T with dS = L_exp(S^T, R0^T dR) (S^T = -S)
 void generator_grad(Calib& C, const double* R0) {
-  GemmCall{C.st}(kCD, kCD, kCD, R0, kCD, true, C.dR, kCD, false, C.dE, kCD);
+  C.gemm()(kCD, kCD, kCD, R0, kCD, true, C.dR, kCD, false, C.dE, kCD);
   const int e = expm(C, C.S, -1.0, C.dE);
   skew_kernel<<<kCD, kCD, 0, C.st>>>(C.T2[e], C.dA);
 }
@@ -624,14 +705,14 @@ namespace {
 // Inputs that stay fixed over the steps: K - mu, the BF16 reference
 // attention p (and log p), the raw window logits.
 void trace_setup(Calib& C, Trace& t, const double* mu) {
-  GemmCall gm{C.st};
+  GemmCall gm = C.gemm();
   const int g = C.c.g, D = kCD;
   const long long nT = (long long)t.T * D, r = (long long)g * t.nt;
   center_kernel<<<nblk(nT), 256, 0, C.st>>>(t.K, mu, nT, t.Kc);
   // raw BF16 logits q_j K^T into L, softmax into Pref
   gm(t.nt, t.T, D, t.q, (long long)g * D, false, t.K, D, true, C.L, t.T, 1.0, 0.0,
      g, D, 0, (long long)t.nt * t.T);
-  softmax_rows_kernel<<<nwarp_blocks(r), 256, 0, C.st>>>(
+  softmax_rows_kernel<<<(unsigned)r, 256, 0, C.st>>>(
       C.L, nullptr, (int)r, t.nt, t.T, t.tpos, C.scale, 0, 0, t.Pref, nullptr,
       nullptr, nullptr);
   logclamp_kernel<<<nblk(r * t.T), 256, 0, C.st>>>(t.Pref, r * t.T, t.logPref);
@@ -642,7 +723,7 @@ void trace_setup(Calib& C, Trace& t, const double* mu) {
 
 // Effective rotated-and-back rows Q2(X R) R^T into C.Kt (Zh, inside kept).
 void q2_roundtrip(Calib& C, const double* X, int T, double clip) {
-  GemmCall gm{C.st};
+  GemmCall gm = C.gemm();
   gm(T, kCD, kCD, X, kCD, false, C.R, kCD, false, C.Z, kCD);
   const long long warps = (long long)T * (kCD / C.c.group);
   q2_kernel<<<nwarp_blocks(warps), 256, 0, C.st>>>(C.Z, T, C.c.group, clip, C.Zh, C.inside);
@@ -651,13 +732,13 @@ void q2_roundtrip(Calib& C, const double* X, int T, double clip) {
 
 // L_K of trace t under C.R into *out; leaves PK, E for the backward.
 void key_forward(Calib& C, Trace& t, double* out) {
-  GemmCall gm{C.st};
+  GemmCall gm = C.gemm();
   const int g = C.c.g, D = kCD, dm = C.c.d_model;
   const long long r = (long long)g * t.nt, nTT = (long long)t.nt * t.T;
   q2_roundtrip(C, t.Kc, t.T, C.c.clip_k);
   gm(t.nt, t.T, D, t.q, (long long)g * D, false, C.Kt, D, true, C.L, t.T, 1.0, 0.0,
      g, D, 0, nTT);
-  softmax_rows_kernel<<<nwarp_blocks(r), 256, 0, C.st>>>(
+  softmax_rows_kernel<<<(unsigned)r, 256, 0, C.st>>>(
       C.L, C.windows ? t.Lc : nullptr, (int)r, t.nt, t.T, t.tpos, C.scale,
       C.c.sink, C.c.recent, C.PK, t.Pref, t.logPref, C.rowv);
   // e_j = ((pk - p) V) W_j^T
@@ -676,7 +757,7 @@ namespace {
 
 // dR of L_K (after key_forward on the same trace and rotation).
 void key_backward(Calib& C, Trace& t) {
-  GemmCall gm{C.st};
+  GemmCall gm = C.gemm();
   const int g = C.c.g, D = kCD, dm = C.c.d_model;
   const long long r = (long long)g * t.nt, nTT = (long long)t.nt * t.T;
   // U_j = (2 lambda / d_model) e_j W_j;  GV_j = U_j V^T
@@ -712,7 +793,7 @@ void value_setup(Calib& C, Trace& t) {
 
 // L_V of trace t under C.R (the value rotation) into *out.
 void value_forward(Calib& C, Trace& t, double* out) {
-  GemmCall gm{C.st};
+  GemmCall gm = C.gemm();
   const int g = C.c.g, D = kCD, dm = C.c.d_model;
   const long long r = (long long)g * t.nt, nTT = (long long)t.nt * t.T;
   q2_roundtrip(C, t.V, t.T, C.c.clip_v);
@@ -728,7 +809,7 @@ void value_forward(Calib& C, Trace& t, double* out) {
 
 // dR of L_V (after value_forward on the same trace and rotation).
 void value_backward(Calib& C, Trace& t) {
-  GemmCall gm{C.st};
+  GemmCall gm = C.gemm();
   const int g = C.c.g, D = kCD, dm = C.c.d_model;
   const long long r = (long long)g * t.nt, nTT = (long long)t.nt * t.T;
   gm(t.nt, D, dm, C.E, dm, false, C.W, D, false, C.U, D, 2.0 / ((double)dm * r), 0.0,
