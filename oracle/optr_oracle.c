@@ -32,11 +32,9 @@
 #define OR_D 128
 #define OR_G 32
 #define OR_P 16
-#define OR_CHUNK 1536
 #define OR_KC 0
 #define OR_VC 512
 #define OR_KM 1024
-#define OR_VM 1280
 
 /* ---------------------------------------------------------------- scalars */
 
@@ -120,20 +118,33 @@ static double dequant(int code, uint16_t scale_bits, uint16_t min_bits) {
 int oracle_code_byte(int ch) { return 4 * ((ch % OR_G) / 4) + ch / OR_G; }
 int oracle_code_shift(int ch) { return 2 * (ch % 4); }
 
-static uint8_t* chunk_of(uint8_t* pool, int page, int h_kv, int h) {
-  return pool + ((size_t)page * h_kv + h) * OR_CHUNK;
+/* Pool record layout per (page, KV head) as a function of the group size:
+ *   G = 32:  1536 bytes: K codes [16][32] at 0, V codes at 512, K meta
+ *            [16 slots][4 blocks][fp16 scale, fp16 min] at 1024, V meta at
+ *            1280 (16 bytes per slot);
+ *   G = 128: 1152 bytes (the paper's compact record, Sec. 5: one scale and
+ *            min per 128 channels, 2 + 0.25 bits per element): codes as
+ *            above, K meta [16 slots][fp16 scale, fp16 min] at 1024, V meta
+ *            at 1088 (4 bytes per slot). */
+static int chunk_bytes(int group) { return group == 128 ? 1152 : 1536; }
+static int vmeta_off(int group) { return group == 128 ? 1088 : 1280; }
+static int meta_stride(int group) { return group == 128 ? 4 : 16; }
+
+static uint8_t* chunk_of(uint8_t* pool, int page, int h_kv, int h, int group) {
+  return pool + ((size_t)page * h_kv + h) * chunk_bytes(group);
 }
 
 static void store_slot(uint8_t* chunk, int codes_off, int meta_off, int slot,
                        const uint8_t* codes /*[128]*/,
                        const uint16_t* scale /*[4]*/,
-                       const uint16_t* mn /*[4]*/) {
+                       const uint16_t* mn /*[4]*/, int group) {
   uint8_t* cb = chunk + codes_off + slot * 32;
   memset(cb, 0, 32);
   for (int ch = 0; ch < OR_D; ++ch)
     cb[oracle_code_byte(ch)] |= (uint8_t)(codes[ch] << oracle_code_shift(ch));
-  uint8_t* mb = chunk + meta_off + slot * 16;
-  for (int g = 0; g < OR_D / OR_G; ++g) {
+  uint8_t* mb = chunk + meta_off + slot * meta_stride(group);
+  /* G = 128: the four 32-channel blocks share one pair, stored once */
+  for (int g = 0; g < (group == 128 ? 1 : OR_D / OR_G); ++g) {
     mb[4 * g + 0] = (uint8_t)(scale[g] & 0xff);
     mb[4 * g + 1] = (uint8_t)(scale[g] >> 8);
     mb[4 * g + 2] = (uint8_t)(mn[g] & 0xff);
@@ -143,12 +154,12 @@ static void store_slot(uint8_t* chunk, int codes_off, int meta_off, int slot,
 
 /* Dequantized rotated vector of one slot (kind 0 = key, 1 = value). */
 static void load_slot(const uint8_t* chunk, int kind, int slot,
-                      double* out /*[128]*/) {
+                      double* out /*[128]*/, int group) {
   const uint8_t* cb = chunk + (kind ? OR_VC : OR_KC) + slot * 32;
-  const uint8_t* mb = chunk + (kind ? OR_VM : OR_KM) + slot * 16;
+  const uint8_t* mb = chunk + (kind ? vmeta_off(group) : OR_KM) + slot * meta_stride(group);
   for (int ch = 0; ch < OR_D; ++ch) {
     int code = (cb[oracle_code_byte(ch)] >> oracle_code_shift(ch)) & 3;
-    int g = ch / OR_G;
+    int g = group == 128 ? 0 : ch / OR_G;
     uint16_t s = (uint16_t)(mb[4 * g] | (mb[4 * g + 1] << 8));
     uint16_t m = (uint16_t)(mb[4 * g + 2] | (mb[4 * g + 3] << 8));
     out[ch] = dequant(code, s, m);
@@ -157,10 +168,11 @@ static void load_slot(const uint8_t* chunk, int kind, int slot,
 
 /* Exported for tests: dequantized K and V of one slot of the pool. */
 int oracle_read_slot(const uint8_t* pool, int h_kv, int page, int h, int slot,
-                     double* khat, double* vhat) {
-  const uint8_t* c = pool + ((size_t)page * h_kv + h) * OR_CHUNK;
-  load_slot(c, 0, slot, khat);
-  load_slot(c, 1, slot, vhat);
+                     double* khat, double* vhat, int group) {
+  if (group != 32 && group != 128) return -1;
+  const uint8_t* c = pool + ((size_t)page * h_kv + h) * chunk_bytes(group);
+  load_slot(c, 0, slot, khat, group);
+  load_slot(c, 1, slot, vhat, group);
   return 0;
 }
 
@@ -261,9 +273,9 @@ int oracle_kv_append(const uint16_t* k, const uint16_t* v, int n_tok,
       float* uv = u_out ? u_out + (((size_t)t * h_kv + h) * 2 + 1) * OR_D : NULL;
       quantize_vector(zk, clip_k, group, ck, sk, mk, uk);
       quantize_vector(zv, clip_v, group, cv, sv, mv, uv);
-      uint8_t* c = chunk_of(pool, page, h_kv, h);
-      store_slot(c, OR_KC, OR_KM, slot, ck, sk, mk);
-      store_slot(c, OR_VC, OR_VM, slot, cv, sv, mv);
+      uint8_t* c = chunk_of(pool, page, h_kv, h, group);
+      store_slot(c, OR_KC, OR_KM, slot, ck, sk, mk, group);
+      store_slot(c, OR_VC, vmeta_off(group), slot, cv, sv, mv, group);
     }
   }
   return bad ? -1 : 0;
@@ -397,7 +409,9 @@ int oracle_decode_attention_win(const uint16_t* q, const int32_t* block_table,
                                 const float* mu, const uint16_t* win,
                                 const int32_t* win_slot, int n_slots, int sink,
                                 int recent, double* out, const int32_t* sel_b,
-                                const int32_t* sel_j, int n_sel, double* p_out) {
+                                const int32_t* sel_j, int n_sel, double* p_out,
+                                int group) {
+  if (group != 32 && group != 128) return -1;
   int n_rows = n_sel > 0 ? n_sel : B * h_q;
   int ratio = h_q / h_kv;
   int bad = 0;
@@ -442,10 +456,10 @@ int oracle_decode_attention_win(const uint16_t* q, const int32_t* block_table,
       } else {
         int page = block_table[(size_t)b * max_pages + s / OR_P];
         if (page < 0 || page >= num_pages) { ok = 0; break; }
-        const uint8_t* c = pool + ((size_t)page * h_kv + h) * OR_CHUNK;
+        const uint8_t* c = pool + ((size_t)page * h_kv + h) * chunk_bytes(group);
         double kh[OR_D];
-        load_slot(c, 0, s % OR_P, kh);
-        load_slot(c, 1, s % OR_P, vs);
+        load_slot(c, 0, s % OR_P, kh, group);
+        load_slot(c, 1, s % OR_P, vs, group);
         for (int i = 0; i < OR_D; ++i) acc += qr[i] * kh[i];
         rot[s] = 1;
       }
@@ -487,11 +501,12 @@ int oracle_decode_attention(const uint16_t* q, const int32_t* block_table,
                             const uint8_t* pool, int num_pages, int h_q,
                             int h_kv, const float* R_k, const float* R_v,
                             double* out, const int32_t* sel_b,
-                            const int32_t* sel_j, int n_sel, double* p_out) {
+                            const int32_t* sel_j, int n_sel, double* p_out,
+                            int group) {
   return oracle_decode_attention_win(q, block_table, seq_lens, B, max_pages,
                                      pool, num_pages, h_q, h_kv, R_k, R_v,
                                      NULL, NULL, NULL, 0, 0, 0, out, sel_b,
-                                     sel_j, n_sel, p_out);
+                                     sel_j, n_sel, p_out, group);
 }
 
 /*

@@ -26,7 +26,21 @@ _lib = None
 D = 128
 G = 32
 P = 16
-CHUNK = 1536
+CHUNK = 1536  # record bytes per (page, KV head) with G = 32
+
+
+def chunk_bytes(group: int = 32) -> int:
+    """Record bytes per (page, KV head): 1536 for G = 32 (four scale/min
+    pairs per slot), 1152 for the compact G = 128 record (one pair)."""
+    return 1152 if group == 128 else 1536
+
+
+def _layout_group(pool) -> int:
+    """Group size implied by a pool's record size."""
+    n = pool.shape[-1]
+    if n not in (1152, 1536):
+        raise ValueError(f"pool record of {n} bytes: expected 1536 or 1152")
+    return 128 if n == 1152 else 32
 
 
 def build(force: bool = False) -> str:
@@ -63,11 +77,11 @@ def _declare(L):
                                    _P, _P, f, f, _P, i]
     L.oracle_kv_append.restype = i
     L.oracle_decode_attention.argtypes = [_P, _P, _P, i, i, _P, i, i, i, _P,
-                                          _P, _P, _P, _P, i, _P]
+                                          _P, _P, _P, _P, i, _P, i]
     L.oracle_decode_attention.restype = i
     L.oracle_decode_attention_win.argtypes = [_P, _P, _P, i, i, _P, i, i, i,
                                               _P, _P, _P, _P, _P, i, i, i, _P,
-                                              _P, _P, i, _P]
+                                              _P, _P, i, _P, i]
     L.oracle_decode_attention_win.restype = i
     L.oracle_window_write.argtypes = [_P, _P, i, _P, _P, i, _P, i, i, i, i, _P]
     L.oracle_window_write.restype = i
@@ -81,7 +95,7 @@ def _declare(L):
     L.oracle_rotate_quantize.restype = i
     L.oracle_rotate_quantize_g.argtypes = [_P, _P, f, _P, _P, _P, _P, _P, i]
     L.oracle_rotate_quantize_g.restype = i
-    L.oracle_read_slot.argtypes = [_P, i, i, i, i, _P, _P]
+    L.oracle_read_slot.argtypes = [_P, i, i, i, i, _P, _P, i]
     L.oracle_read_slot.restype = i
     L.oracle_code_byte.argtypes = [i]
     L.oracle_code_byte.restype = i
@@ -145,14 +159,15 @@ def rotate_quantize(x, R, clip: float = 1.0, group: int = 32):
 
 def kv_append(k_bits, v_bits, cu_new, pos0, block_table, pool, R_k, R_v, mu,
               clip_k=1.0, clip_v=1.0, want_u=False, group=32):
-    """Oracle cache write; ``pool`` (uint8 [num_pages][h_kv][1536]) is
-    modified in place.  Returns the pre-rounding values when want_u."""
+    """Oracle cache write; ``pool`` (uint8 [num_pages][h_kv][chunk_bytes(group)])
+    is modified in place.  Returns the pre-rounding values when want_u."""
     k_bits = _c(k_bits, np.uint16)
     v_bits = _c(v_bits, np.uint16)
     cu_new = _c(cu_new, np.int32)
     pos0 = _c(pos0, np.int32)
     bt = _c(block_table, np.int32)
     assert pool.dtype == np.uint8 and pool.flags["C_CONTIGUOUS"]
+    assert pool.shape[-1] == chunk_bytes(group), "pool record size vs group"
     n_tok, h_kv = k_bits.shape[0], k_bits.shape[1]
     B = pos0.size
     max_pages = bt.shape[1]
@@ -172,7 +187,8 @@ def kv_append(k_bits, v_bits, cu_new, pos0, block_table, pool, R_k, R_v, mu,
 def decode_attention(q_bits, block_table, seq_lens, pool, R_k, R_v, h_kv,
                      rows=None, want_p=False, win=None, win_slot=None, sink=0,
                      recent=0, mu=None):
-    """Oracle decode.  Returns float64 [B][h_q][128]; when ``rows`` (a list of
+    """Oracle decode (the pool's record size selects its layout: 1536 bytes
+    for G = 32, 1152 for G = 128).  Returns float64 [B][h_q][128]; when ``rows`` (a list of
     (b, j)) is given only those rows are computed (others stay zero).  With
     ``sink`` / ``recent`` > 0 the BF16 window positions are read from ``win``
     (uint16 bf16 bits [n_slots][h_kv][2][sink + recent][128]) at the slots
@@ -208,7 +224,7 @@ def decode_attention(q_bits, block_table, seq_lens, pool, R_k, R_v, h_kv,
         pool.shape[0], h_q, h_kv, _ptr(_c(R_k, np.float32)),
         _ptr(_c(R_v, np.float32)), _ptr(mu), _ptr(win), _ptr(win_slot),
         n_slots, int(sink), int(recent), _ptr(out), _ptr(sb), _ptr(sj), n_sel,
-        _ptr(p))
+        _ptr(p), _layout_group(pool))
     if rc != 0:
         raise ValueError("oracle_decode_attention: table entry or window slot out of range")
     return (out, p) if want_p else out
@@ -261,7 +277,7 @@ def read_slot(pool, page, h, slot):
     kh = np.zeros(D, np.float64)
     vh = np.zeros(D, np.float64)
     lib().oracle_read_slot(_ptr(pool), pool.shape[1], int(page), int(h),
-                           int(slot), _ptr(kh), _ptr(vh))
+                           int(slot), _ptr(kh), _ptr(vh), _layout_group(pool))
     return kh, vh
 
 

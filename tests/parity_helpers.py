@@ -41,14 +41,21 @@ def token_slots(cu, pos0, bt):
 
 
 def slot_codes(pool, pages, slots, kind):
-    """codes [n][h_kv][128] and (scale, min) float64 [n][h_kv][4]."""
-    chunk = pool[pages]  # [n, h_kv, 1536]
+    """codes [n][h_kv][128] and (scale, min) float64 [n][h_kv][4] (the
+    compact G = 128 record's one pair repeated in the four entries; the
+    pool's record size, 1536 or 1152 bytes, gives its layout)."""
+    chunk = pool[pages]  # [n, h_kv, 1536 or 1152]
+    compact = pool.shape[-1] == 1152
     off = 512 * kind
     idx = off + slots[:, None] * 32 + np.arange(32)[None]
     cb = np.take_along_axis(chunk, idx[:, None, :].repeat(chunk.shape[1], 1), 2)
     codes = (cb[..., CODE_BYTE] >> CODE_SHIFT) & 3
-    moff = 1024 + 256 * kind
-    midx = moff + slots[:, None] * 16 + np.arange(16)[None]
+    if compact:
+        moff = 1024 + 64 * kind
+        midx = moff + slots[:, None] * 4 + np.tile(np.arange(4), 4)[None]
+    else:
+        moff = 1024 + 256 * kind
+        midx = moff + slots[:, None] * 16 + np.arange(16)[None]
     mb = np.take_along_axis(chunk, midx[:, None, :].repeat(chunk.shape[1], 1), 2)
     meta = np.ascontiguousarray(mb).view(np.float16).astype(np.float64)
     return codes, meta[..., 0::2], meta[..., 1::2]
@@ -143,7 +150,8 @@ def gpu_decode(case, pool_np, variant=optr.OPTR_VARIANT_DEFAULT,
 
 def oracle_case(case, pool_init=None, group=32, clip_k=1.0, clip_v=1.0):
     """Oracle append of context and new tokens; returns (pool, u_ctx, u_new)."""
-    pool = (np.zeros((case["num_pages"], case["h_kv"], 1536), np.uint8)
+    pool = (np.zeros((case["num_pages"], case["h_kv"], oracle.chunk_bytes(group)),
+                     np.uint8)
             if pool_init is None else pool_init.copy())
     bt = case["block_table"].numpy()
     args = (case["R_k"].numpy(), case["R_v"].numpy(), case["mu"].numpy())
@@ -176,8 +184,8 @@ def oracle_decode(case, pool, rows=None, seq_lens=None, q=None):
 def dequant_records(pool, pages, slots, h, kind):
     """Dequantized rotated vectors code * scale + min (float64 [n][128]) of
     KV head h at the given (page, slot) records of a pool; kind 0 = keys,
-    1 = values.  G = 128 records hold their pair in all four entries, so the
-    same 32-channel reading serves both group sizes."""
+    1 = values (slot_codes repeats a compact record's pair per 32-channel
+    block, so one reading serves both layouts)."""
     codes, sc, mn = slot_codes(pool, pages, slots, kind)
     grp = _CH // 32
     return codes[:, h, :] * sc[:, h, grp] + mn[:, h, grp]

@@ -84,7 +84,7 @@ def test_paged_equals_dense_with_128_groups(oracle_mod):
     bt, num_pages = synth.page_tables(seq, True, 3)
     cu = np.concatenate([[0], np.cumsum(seq)]).astype(np.int32)
     pos0 = np.zeros(len(seq), np.int32)
-    pool = np.zeros((num_pages, h_kv, 1536), np.uint8)
+    pool = np.zeros((num_pages, h_kv, oracle_mod.chunk_bytes(128)), np.uint8)
     kb, vb = synth.bf16_bits(k), synth.bf16_bits(v)
     oracle_mod.kv_append(kb, vb, cu, pos0, bt.numpy(), pool, R_k.numpy(),
                          R_v.numpy(), mu, clip_k=0.96, clip_v=0.92, group=128)

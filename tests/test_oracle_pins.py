@@ -123,6 +123,38 @@ def test_slot_layout_golden(oracle_mod):
         assert not others.any()  # only slot 3 written
 
 
+def test_compact_g128_record_golden(oracle_mod):
+    """The compact G = 128 record (Sec. 5's one scale and min per 128
+    channels): 1152 bytes per (page, KV head), codes laid out as with G = 32,
+    one 4-byte (scale, min) per slot at 1024 (keys) and 1088 (values), and
+    nothing else written."""
+    meta = {name: (int(off), bytes.fromhex(hx.replace(" ", "")))
+            for name, off, hx in _read_golden("slot_layout_g128.txt")}
+    for name, formula, hexbytes in _read_golden("slot_layout.txt"):
+        ch = np.arange(D)
+        g, w, r = ch // 32, (ch % 32) // 4, ch % 4
+        z = {"r": r, "(r+g)%4": (r + g) % 4, "(r+w)%4": (r + w) % 4}[formula]
+        k = torch.tensor(z, dtype=torch.bfloat16).view(1, 1, D)
+        pool = np.zeros((1, 1, 1152), np.uint8)
+        oracle_mod.kv_append(_bits(k), _bits(k), [0, 1], [3], [[0]], pool,
+                             _identity(), _identity(), np.zeros((1, D)),
+                             group=128)
+        want = bytes.fromhex(hexbytes.replace(" ", ""))
+        assert bytes(pool[0, 0, 3 * 32:4 * 32]) == want, name
+        assert bytes(pool[0, 0, 512 + 96:512 + 128]) == want, name
+        for field, (off, val) in meta.items():
+            assert bytes(pool[0, 0, off:off + len(val)]) == val, (name, field)
+        rest = pool[0, 0].copy()
+        rest[3 * 32:4 * 32] = 0
+        rest[512 + 96:512 + 128] = 0
+        for off, val in meta.values():
+            rest[off:off + len(val)] = 0
+        assert not rest.any(), name  # only slot 3's codes and pairs written
+        kh, vh = oracle_mod.read_slot(pool, 0, 0, 3)
+        assert np.array_equal(kh, z.astype(np.float64)), name
+        assert np.array_equal(vh, z.astype(np.float64)), name
+
+
 def test_rotation_is_right_multiplication(oracle_mod):
     """Row-vector convention z' = z R (Intro and Sec. 3.1 Eq. 4): with R a
     permutation matrix R[i][pi(i)] = 1, channel i lands on channel pi(i)."""
