@@ -139,12 +139,19 @@ def traffic_for(kernel_key, files):
 
 # ------------------------------------------------------------ byte counts
 
-def decode_bytes(seq_lens, h_kv, h_q):
-    """Algorithmic bytes of one decode: 96 B per cached token and KV head
-    (32 + 32 code bytes, 16 + 16 metadata bytes), bf16 query, fp32 output."""
+def record_bytes(group=32):
+    """Cache bytes per token and KV head: 32 + 32 code bytes and 16 + 16
+    metadata bytes (G = 32), or 4 + 4 metadata bytes (the compact G = 128
+    record)."""
+    return 72 if group == 128 else 96
+
+
+def decode_bytes(seq_lens, h_kv, h_q, group=32):
+    """Algorithmic bytes of one decode: the cache records of every cached
+    token and KV head, bf16 query, fp32 output."""
     toks = int(sum(int(x) for x in seq_lens))
     B = len(seq_lens)
-    return toks * h_kv * 96 + B * h_q * D * 2 + B * h_q * D * 4
+    return toks * h_kv * record_bytes(group) + B * h_q * D * 2 + B * h_q * D * 4
 
 
 def decode_stream_bytes(seq_lens, h_kv):
@@ -152,9 +159,10 @@ def decode_stream_bytes(seq_lens, h_kv):
     return int(sum(int(x) for x in seq_lens)) * h_kv * 96
 
 
-def append_bytes(n_tok, h_kv):
-    """Append: bf16 K and V read (512 B) + 96 B written per token and head."""
-    return n_tok * h_kv * (512 + 96)
+def append_bytes(n_tok, h_kv, group=32):
+    """Append: bf16 K and V read (512 B) + the record written per token and
+    head."""
+    return n_tok * h_kv * (512 + record_bytes(group))
 
 
 def window_split(n, sink, recent):
@@ -166,17 +174,17 @@ def window_split(n, sink, recent):
     return n - nw, nw
 
 
-def decode_bytes_win(seq_lens, h_kv, h_q, sink, recent):
-    """Algorithmic bytes of one decode with BF16 windows: 96 B per INT2
-    token and KV head, 512 B (bf16 K and V rows) per window token and KV
-    head, bf16 query, fp32 output."""
+def decode_bytes_win(seq_lens, h_kv, h_q, sink, recent, group=32):
+    """Algorithmic bytes of one decode with BF16 windows: the record (96 or
+    72 B) per INT2 token and KV head, 512 B (bf16 K and V rows) per window
+    token and KV head, bf16 query, fp32 output."""
     i2 = wt = 0
     for x in seq_lens:
         a, b = window_split(int(x), sink, recent)
         i2 += a
         wt += b
     B = len(seq_lens)
-    return (i2 * h_kv * 96 + wt * h_kv * 512 + B * h_q * D * 2 +
+    return (i2 * h_kv * record_bytes(group) + wt * h_kv * 512 + B * h_q * D * 2 +
             B * h_q * D * 4)
 
 
@@ -387,7 +395,7 @@ def extra_workloads(args, dev):
         optr.optr_profile_enable(p, False)
         ms = float(np.mean(t))
         n_tok = k.shape[0]
-        nb = append_bytes(n_tok, case["h_kv"])
+        nb = append_bytes(n_tok, case["h_kv"], group)
         res[key] = {
             "tokens": n_tok, "group": group, "ms": round(ms, 4),
             "tokens_per_s": round(n_tok / (ms * 1e-3), 1),
@@ -571,11 +579,11 @@ def windows_step(args, dev, flush, hbm_peak, sink=64, recent=256, group=32,
     optr.optr_profile_enable(p, False)
     lens = case["seq_lens"].tolist()
     n_new = k_new.shape[0]
-    nb = (decode_bytes_win(lens, h_kv, h_q, sink, recent) +
-          append_bytes(n_new, h_kv) + n_new * h_kv * 512)  # + window copies
+    nb = (decode_bytes_win(lens, h_kv, h_q, sink, recent, group) +
+          append_bytes(n_new, h_kv, group) + n_new * h_kv * 512)  # + window copies
     i2 = sum(window_split(x, sink, recent)[0] for x in lens)
     wt = sum(window_split(x, sink, recent)[1] for x in lens)
-    pb = i2 * h_kv * 96 + wt * h_kv * 512  # what the partial kernel streams
+    pb = i2 * h_kv * record_bytes(group) + wt * h_kv * 512  # what the partial kernel streams
     pm = float(np.mean(part))
     return {"sink": sink, "recent": recent, "group": group,
             "clip_k": clip_k, "clip_v": clip_v, "step_ms": round(ms, 4),

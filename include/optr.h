@@ -72,9 +72,15 @@
  *      offset  512: V codes  [16 slots][32 bytes]
  *      offset 1024: K meta   [16 slots][4 groups] {fp16 scale, fp16 min}
  *      offset 1280: V meta   [16 slots][4 groups] {fp16 scale, fp16 min}
- * The metadata has one {scale, min} entry per 32-channel block; with
- * G = 128 the group's pair is stored in all four entries (the decode then
- * reads the same layout for both group sizes).
+ * The metadata has one {scale, min} entry per 32-channel block.  With
+ * G = 128 the record is the paper's compact one (Sec. 5: one fp16 scale and
+ * min per 128 channels, 2.25 bits per element), OPTR_PAGE_HEAD_BYTES_G128 =
+ * 1152 bytes per (page, KV head):
+ *      offset    0: K codes  [16 slots][32 bytes]
+ *      offset  512: V codes  [16 slots][32 bytes]
+ *      offset 1024: K meta   [16 slots] {fp16 scale, fp16 min}
+ *      offset 1088: V meta   [16 slots] {fp16 scale, fp16 min}
+ * and the pool is pool[num_pages][h_kv][1152] (optr_page_bytes).
  * Within a slot's 32 code bytes the groups are interleaved word-major:
  * channel ch = 32*g + 4*w + r  (group g in 0..3, w in 0..7, r in 0..3) is
  * stored in byte 4*w + g, bits [2r, 2r+1].  Byte 4*w + g therefore holds the
@@ -122,6 +128,9 @@ extern "C" {
 #define OPTR_V_CODES_OFFSET 512
 #define OPTR_K_META_OFFSET 1024
 #define OPTR_V_META_OFFSET 1280
+/* the compact record of G = 128 (one scale and min per 128 channels) */
+#define OPTR_PAGE_HEAD_BYTES_G128 1152
+#define OPTR_V_META_OFFSET_G128 1088
 
 typedef enum {
   OPTR_OK = 0,
@@ -192,7 +201,8 @@ optr_status optr_params_create(const optr_config* cfg, const float* R_k,
  * still uses it. */
 void optr_params_destroy(optr_params* p);
 
-/* Bytes of one page across all KV heads: h_kv * 1536. */
+/* Bytes of one page across all KV heads: h_kv * 1536 (G = 32) or
+ * h_kv * 1152 (the compact G = 128 record). */
 size_t optr_page_bytes(const optr_params* p);
 
 /*

@@ -55,7 +55,7 @@ append_cuda_core_kernel(const __nv_bfloat16* __restrict__ k,
     long long off = -1;
     if (tok < n_tok)
       off = resolve_slot(tok, h, cu_new, pos0, bt, B, max_pages, num_pages,
-                         h_kv, &slot, err);
+                         h_kv, &slot, err, chunk_bytes(group128 != 0));
     dst[tid] = off;
     dslot[tid] = slot;
   }
@@ -78,7 +78,8 @@ append_cuda_core_kernel(const __nv_bfloat16* __restrict__ k,
   const float sub = kind ? 0.f : __ldg(muR + h * kD + j);
   const float clip = kind ? clip_v : clip_k;
   const int codes_off = kind ? OPTR_V_CODES_OFFSET : OPTR_K_CODES_OFFSET;
-  const int meta_off = kind ? OPTR_V_META_OFFSET : OPTR_K_META_OFFSET;
+  const bool compact = group128 != 0;  // one (scale, min) pair per slot
+  const int meta_off = kind ? vmeta_offset(compact) : OPTR_K_META_OFFSET;
 #pragma unroll 1
   for (int t = 0; t < T; ++t) {
     const float z = __fsub_rn(acc[t], sub);
@@ -107,8 +108,9 @@ append_cuda_core_kernel(const __nv_bfloat16* __restrict__ k,
       const int slot = dslot[t];
       if ((lane & 3) == 0)
         chunk[codes_off + slot * 32 + 4 * (lane >> 2) + g] = (uint8_t)bits;
-      if (lane == 0)
-        *reinterpret_cast<__half2*>(chunk + meta_off + slot * 16 + 4 * g) =
+      if (lane == 0 && (!compact || g == 0))
+        *reinterpret_cast<__half2*>(chunk + meta_off + slot * meta_stride(compact) +
+                                    (compact ? 0 : 4 * g)) =
             __halves2half2(gq.scale, gq.min);
     }
   }

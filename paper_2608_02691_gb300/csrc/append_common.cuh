@@ -16,14 +16,14 @@ __device__ __forceinline__ int find_seq(const int32_t* __restrict__ cu_new,
   return lo;
 }
 
-// Byte offset in the pool of the chunk (page, h) and the slot of new token
-// `tok`, or -1 (after flagging the device error word) when a table entry,
+// Byte offset in the pool of the record (page, h) (records of `chunk`
+// bytes) and the slot of new token `tok`, or -1 (after flagging the device error word) when a table entry,
 // position or cu_new entry is out of range.
 __device__ __forceinline__ long long resolve_slot(int tok, int h, const int32_t* __restrict__ cu_new,
                                   const int32_t* __restrict__ pos0,
                                   const int32_t* __restrict__ bt, int B,
                                   int max_pages, int num_pages, int h_kv,
-                                  int* slot, unsigned* err) {
+                                  int* slot, unsigned* err, int chunk) {
   int b = find_seq(cu_new, B, tok);
   int c0 = __ldg(cu_new + b), c1 = __ldg(cu_new + b + 1);
   if (!(c0 <= tok && tok < c1)) {
@@ -41,7 +41,7 @@ __device__ __forceinline__ long long resolve_slot(int tok, int h, const int32_t*
     return -1;
   }
   *slot = (int)(pos % kPage);
-  return ((long long)page * h_kv + h) * kChunk;
+  return ((long long)page * h_kv + h) * chunk;
 }
 
 // resolve_slot() with cu_new[0..B] and pos0[0..B-1] already in shared
@@ -50,7 +50,7 @@ __device__ __forceinline__ long long resolve_slot(int tok, int h, const int32_t*
 __device__ __forceinline__ long long resolve_slot_cached(
     int tok, int h, const int* cu, const int* p0,
     const int32_t* __restrict__ bt, int B, int max_pages, int num_pages,
-    int h_kv, int* slot, unsigned* err) {
+    int h_kv, int* slot, unsigned* err, int chunk) {
   int lo = 0, hi = B;
   while (hi - lo > 1) {
     const int mid = (lo + hi) >> 1;
@@ -73,7 +73,7 @@ __device__ __forceinline__ long long resolve_slot_cached(
     return -1;
   }
   *slot = (int)(pos % kPage);
-  return ((long long)page * h_kv + h) * kChunk;
+  return ((long long)page * h_kv + h) * chunk;
 }
 
 }  // namespace optr

@@ -113,7 +113,7 @@ __device__ __forceinline__ void append_small_body(
       }
     } else {
       off = resolve_slot(my_tok, h, cu_new, pos0, bt, B, max_pages, num_pages,
-                         h_kv, &slot, err);
+                         h_kv, &slot, err, chunk_bytes(group128));
     }
   }
   if (identity) {
@@ -137,7 +137,7 @@ __device__ __forceinline__ void append_small_body(
       } else if (page < 0 || page >= num_pages) {
         atomicOr(err, OPTR_DEVERR_PAGE_ID);
       } else {
-        off = ((long long)page * h_kv + h) * kChunk;
+        off = ((long long)page * h_kv + h) * chunk_bytes(group128);
       }
     }
     dst[tid] = off;
@@ -152,7 +152,8 @@ __device__ __forceinline__ void append_small_body(
   const int wslot = dslot[warp];
   const float clip = kind ? clip_v : clip_k;
   const int codes_off = kind ? OPTR_V_CODES_OFFSET : OPTR_K_CODES_OFFSET;
-  const int meta_off = kind ? OPTR_V_META_OFFSET : OPTR_K_META_OFFSET;
+  // G = 128: the compact record, one (scale, min) pair per slot
+  const int meta_off = kind ? vmeta_offset(group128) : OPTR_K_META_OFFSET;
   uint8_t* chunk = pool + woff;
   float zv[kGroups];
 #pragma unroll
@@ -193,8 +194,9 @@ __device__ __forceinline__ void append_small_body(
     bits |= __shfl_xor_sync(0xffffffffu, bits, 2);
     if ((lane & 3) == 0)
       chunk[codes_off + wslot * 32 + 4 * (lane >> 2) + g] = (uint8_t)bits;
-    if (lane == 0)
-      *reinterpret_cast<__half2*>(chunk + meta_off + wslot * 16 + 4 * g) =
+    if (lane == 0 && (!group128 || g == 0))
+      *reinterpret_cast<__half2*>(chunk + meta_off + wslot * meta_stride(group128) +
+                                  (group128 ? 0 : 4 * g)) =
           __halves2half2(gq.scale, gq.min);
   }
 }

@@ -310,7 +310,8 @@ append_tc05_kernel(const __grid_constant__ CUtensorMap tmap_k,
     const int g = warp >> 3, q = warp & 3, hp = (warp >> 2) & 1, row = 32 * q + lane;
     const float clip = kind ? clip_v : clip_k;
     const int codes_off = kind ? OPTR_V_CODES_OFFSET : OPTR_K_CODES_OFFSET;
-    const int meta_off = kind ? OPTR_V_META_OFFSET : OPTR_K_META_OFFSET;
+    // G = 128: the compact record, one (scale, min) pair per slot
+    const int meta_off = kind ? vmeta_offset(kG128) : OPTR_K_META_OFFSET;
     const uint32_t lane_base = (uint32_t)(32 * q) << 16;
     const uint32_t tD = tmem + lane_base + kColD0 + 128u * g;
     const int n_mine = my_tiles > g ? (my_tiles - 1 - g) / 2 + 1 : 0;
@@ -324,9 +325,9 @@ append_tc05_kernel(const __grid_constant__ CUtensorMap tmap_k,
       long long d = -1;
       if (tok < n_tok)
         d = cached ? resolve_slot_cached(tok, h, S.cu, S.p0, bt, B, max_pages,
-                                         num_pages, h_kv, &slot, err)
+                                         num_pages, h_kv, &slot, err, chunk_bytes(kG128))
                    : resolve_slot(tok, h, cu_new, pos0, bt, B, max_pages,
-                                  num_pages, h_kv, &slot, err);
+                                  num_pages, h_kv, &slot, err, chunk_bytes(kG128));
       __syncwarp();  // converged for the warp-wide tensor-memory accesses
       return d;
     };
@@ -495,7 +496,14 @@ append_tc05_kernel(const __grid_constant__ CUtensorMap tmap_k,
           *reinterpret_cast<uint4*>(rec + codes_off + slot * 32 + 16) =
               make_uint4(word[4], word[5], word[6], word[7]);
         }
-        *reinterpret_cast<uint2*>(rec + meta_off + slot * 16 + 8 * hp) = make_uint2(meta[0], meta[1]);
+        if constexpr (kG128) {
+          // both half-row threads hold the group's one pair after the
+          // range exchange; the first writes it
+          if (!hp) *reinterpret_cast<uint32_t*>(rec + meta_off + slot * 4) = meta[0];
+        } else {
+          *reinterpret_cast<uint2*>(rec + meta_off + slot * 16 + 8 * hp) =
+              make_uint2(meta[0], meta[1]);
+        }
       }
       __syncwarp();
     }

@@ -295,8 +295,12 @@ partial_cuda_core_kernel(const uint8_t* __restrict__ pool,
                          const int* __restrict__ pref,
                          const int* __restrict__ nzpref,
                          float* __restrict__ part, int W, unsigned* err,
-                         int sink, int recent, WinPhase wp) {
+                         int sink, int recent, WinPhase wp, int compact) {
+  // compact: the G = 128 record (one scale/min pair per slot, 1152 bytes)
   __shared__ WarpSmemCC smem[4];
+  const int chunk = chunk_bytes(compact != 0);
+  const int mstride = meta_stride(compact != 0);
+  const int vmeta = vmeta_offset(compact != 0);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   WarpSmemCC& S = smem[warp];
   const int w = blockIdx.x * 4 + warp;
@@ -332,13 +336,14 @@ partial_cuda_core_kernel(const uint8_t* __restrict__ pool,
     }
     const int32_t* btb = bt + (size_t)b * max_pages;
     // 2-stage cp.async pipeline over the segment's pages
-    bool ok0 = issue_page(S.stage[0], pool, btb, poff + sg.p0, num_pages, h_kv, h, lane, err);
+    bool ok0 = issue_page(S.stage[0], pool, btb, poff + sg.p0, num_pages, h_kv, h, lane, err,
+                          chunk);
     bool okn = false;
     for (int i = 0; i < sg.n; ++i) {
       const bool ok = (i == 0) ? ok0 : okn;
       if (i + 1 < sg.n)
         okn = issue_page(S.stage[(i + 1) & 1], pool, btb, poff + sg.p0 + i + 1,
-                         num_pages, h_kv, h, lane, err);
+                         num_pages, h_kv, h, lane, err, chunk);
       else
         cp_async_commit();
       cp_async_wait_1();
@@ -354,7 +359,7 @@ partial_cuda_core_kernel(const uint8_t* __restrict__ pool,
       if (t < nvalid) {
         float a0 = 0.f, a1 = 0.f;
         const uint8_t* kc = st + OPTR_K_CODES_OFFSET + t * 32;
-        const __half2* km = reinterpret_cast<const __half2*>(st + OPTR_K_META_OFFSET + t * 16);
+        const __half2* km = reinterpret_cast<const __half2*>(st + OPTR_K_META_OFFSET + t * mstride);
 #pragma unroll
         for (int G = 0; G < kGroups; ++G) {
           float d0 = 0.f, d1 = 0.f;
@@ -369,7 +374,7 @@ partial_cuda_core_kernel(const uint8_t* __restrict__ pool,
               d1 = fmaf(S.qv[hp + 1][ch], c, d1);
             }
           }
-          const float2 sm = __half22float2(km[G]);
+          const float2 sm = __half22float2(km[compact ? 0 : G]);
           a0 += sm.x * d0 + sm.y * S.qsum[hp][G];
           a1 += sm.x * d1 + sm.y * S.qsum[hp + 1][G];
         }
@@ -422,7 +427,7 @@ partial_cuda_core_kernel(const uint8_t* __restrict__ pool,
       for (int tt = 0; tt < nvalid; ++tt) {
         const unsigned byte = st[OPTR_V_CODES_OFFSET + tt * 32 + lane];
         const float2 sm = __half22float2(
-            reinterpret_cast<const __half2*>(st + OPTR_V_META_OFFSET + tt * 16)[G]);
+            reinterpret_cast<const __half2*>(st + vmeta + tt * mstride)[compact ? 0 : G]);
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
           const float vv = fmaf((float)((byte >> (2 * c)) & 3u), sm.x, sm.y);
@@ -838,7 +843,8 @@ cudaError_t launch_decode(const optr_params* p, int variant,
     e = launch_pdl(windows ? partial_cuda_core_kernel<true> : partial_cuda_core_kernel<false>,
                    dim3(plan.W / 4), dim3(128), 0, s,
                    pool, bt, seq_lens, B, max_pages, num_pages, h_q, h_kv, qf,
-                   qs, pref, nzpref, part, plan.W, p->err, sink, recent, wp);
+                   qs, pref, nzpref, part, plan.W, p->err, sink, recent, wp,
+                   p->cfg.group == 128 ? 1 : 0);
   }
   if (e != cudaSuccess) return e;
   prof_mark(p, 4, s);

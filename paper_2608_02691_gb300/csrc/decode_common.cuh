@@ -84,8 +84,9 @@ __device__ __forceinline__ void cp_async_wait() {
 }
 __device__ __forceinline__ void cp_async_wait_1() { cp_async_wait<1>(); }
 
-// Stage the 1536-byte chunk (page, h) of logical page `page_idx` into shared
-// memory (three 16-byte copies per lane) and commit one cp.async group.  An
+// Stage the record (page, h) of logical page `page_idx` (`chunk` bytes: 1536,
+// or 1152 for the compact G = 128 record) into shared memory (up to three
+// 16-byte copies per lane) and commit one cp.async group.  An
 // out-of-range page id is flagged and not read; the group is still
 // committed so that group counting stays uniform.
 __device__ __forceinline__ bool issue_page(uint8_t* stage,
@@ -93,14 +94,15 @@ __device__ __forceinline__ bool issue_page(uint8_t* stage,
                                            const int32_t* __restrict__ btb,
                                            int page_idx, int num_pages,
                                            int h_kv, int h, int lane,
-                                           unsigned* err) {
+                                           unsigned* err, int chunk) {
   const int phys = __ldg(btb + page_idx);
   const bool ok = phys >= 0 && phys < num_pages;
   if (ok) {
-    const uint8_t* src = pool + ((size_t)phys * h_kv + h) * kChunk;
+    const uint8_t* src = pool + ((size_t)phys * h_kv + h) * chunk;
 #pragma unroll
     for (int c = 0; c < 3; ++c)
-      cp_async16(stage + (lane + 32 * c) * 16, src + (lane + 32 * c) * 16);
+      if ((lane + 32 * c) * 16 < chunk)
+        cp_async16(stage + (lane + 32 * c) * 16, src + (lane + 32 * c) * 16);
   } else if (lane == 0) {
     atomicOr(err, OPTR_DEVERR_PAGE_ID);
   }
@@ -112,13 +114,15 @@ __device__ __forceinline__ bool issue_page(uint8_t* stage,
 __device__ __forceinline__ bool issue_phys(uint8_t* stage,
                                            const uint8_t* __restrict__ pool,
                                            int phys, int num_pages, int h_kv,
-                                           int h, int lane, unsigned* err) {
+                                           int h, int lane, unsigned* err,
+                                           int chunk) {
   const bool ok = phys >= 0 && phys < num_pages;
   if (ok) {
-    const uint8_t* src = pool + ((size_t)phys * h_kv + h) * kChunk;
+    const uint8_t* src = pool + ((size_t)phys * h_kv + h) * chunk;
 #pragma unroll
     for (int c = 0; c < 3; ++c)
-      cp_async16(stage + (lane + 32 * c) * 16, src + (lane + 32 * c) * 16);
+      if ((lane + 32 * c) * 16 < chunk)
+        cp_async16(stage + (lane + 32 * c) * 16, src + (lane + 32 * c) * 16);
   } else if (lane == 0) {
     atomicOr(err, OPTR_DEVERR_PAGE_ID);
   }

@@ -223,8 +223,11 @@ __device__ __noinline__ void page_prefix(const int32_t* __restrict__ seq_lens,
 }
 
 // WIN: the BF16-window phase is compiled in (a separate instance, so that
-// the INT2-only kernel keeps its own register allocation).
-template <bool WIN>
+// the INT2-only kernel keeps its own register allocation).  CMP: the compact
+// G = 128 record (1152 bytes per page and KV head, one (scale, min) pair per
+// slot at 4-byte stride), read as the G = 32 record's four entries with the
+// pair repeated, so the page arithmetic is the same.
+template <bool WIN, bool CMP>
 __global__ void __launch_bounds__(kWarps * 32, 1)
 partial_tensor_kernel(const uint8_t* __restrict__ pool,
                       const int32_t* __restrict__ bt,
@@ -317,11 +320,12 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
       const int nv = __shfl_sync(0xffffffffu, chk.nvalid, j);
       // an invalid page (flagged, all tokens masked) is filled with zeros
       const bool ok = unit >= 0;
-      const uint8_t* src = pool + (size_t)(ok ? unit : 0) * kChunk + lane * 16;
+      const uint8_t* src = pool + (size_t)(ok ? unit : 0) * chunk_bytes(CMP) + lane * 16;
       uint8_t* dst = S.stage[s] + lane * 16;
       cp_async16_zfill(dst, src, ok);
       cp_async16_zfill(dst + 512, src + 512, ok);
-      cp_async16_zfill(dst + 1024, src + 1024, ok);
+      if (!CMP || lane < 8)  // the compact record's last 128 bytes
+        cp_async16_zfill(dst + 1024, src + 1024, ok);
       S.info[s] = make_int2(key, nv);  // same value from every lane
       ++f_issue;
     }
@@ -441,6 +445,17 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
 
   // ------------------------------------------------ parts of one page
   // logits of tokens g and g+8 (head c) of the page staged at st
+  // the four (scale, min) entries of slot t in a metadata region (the
+  // compact record's one pair repeated)
+  auto meta4 = [&](const uint8_t* region, int t) -> uint4 {
+    if constexpr (CMP) {
+      const uint32_t x = *reinterpret_cast<const uint32_t*>(region + t * 4);
+      return make_uint4(x, x, x, x);
+    } else {
+      return *reinterpret_cast<const uint4*>(region + t * 16);
+    }
+  };
+
   auto logits = [&](const uint8_t* st, float& sc0, float& sc1) {
     const uint2 k0 = *reinterpret_cast<const uint2*>(st + OPTR_K_CODES_OFFSET + g * 32 + 8 * c);
     const uint2 k1 = *reinterpret_cast<const uint2*>(st + OPTR_K_CODES_OFFSET + (g + 8) * 32 + 8 * c);
@@ -465,16 +480,18 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
         mma16816(s_acc[G], f0[par][2], f1[par][2], f0[par][3], f1[par][3], qv.z, qv.w);
       }
     }
-    const uint4 km0 = *reinterpret_cast<const uint4*>(st + OPTR_K_META_OFFSET + g * 16);
-    const uint4 km1 = *reinterpret_cast<const uint4*>(st + OPTR_K_META_OFFSET + (g + 8) * 16);
+    const uint4 km0 = meta4(st + OPTR_K_META_OFFSET, g);
+    const uint4 km1 = meta4(st + OPTR_K_META_OFFSET, g + 8);
     const uint32_t kmv0[4] = {km0.x, km0.y, km0.z, km0.w};
     const uint32_t kmv1[4] = {km1.x, km1.y, km1.z, km1.w};
     // sum_g min_g * sum(q' over g) on the tensor core: A row t = the 8
     // (scale, min) halves of token t, B = (0, Q_g) per (scale, min) pair
     float u[4] = {0.f, 0.f, 0.f, 0.f};
     {
-      const uint32_t w0 = *reinterpret_cast<const uint32_t*>(st + OPTR_K_META_OFFSET + g * 16 + 4 * c);
-      const uint32_t w1 = *reinterpret_cast<const uint32_t*>(st + OPTR_K_META_OFFSET + (g + 8) * 16 + 4 * c);
+      const uint32_t w0 = *reinterpret_cast<const uint32_t*>(
+          st + OPTR_K_META_OFFSET + g * meta_stride(CMP) + (CMP ? 0 : 4 * c));
+      const uint32_t w1 = *reinterpret_cast<const uint32_t*>(
+          st + OPTR_K_META_OFFSET + (g + 8) * meta_stride(CMP) + (CMP ? 0 : 4 * c));
       mma16816(u, w0, w1, 0u, 0u, bmin, 0u);
     }
     float t0 = 0.f, t1 = 0.f;
@@ -492,8 +509,8 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
   // value (scale, min) halves of tokens g (vm[0..3]) and g+8 (vm[4..7])
   // per group, kept packed; returns their largest scale
   auto vmeta = [&](const uint8_t* st, uint32_t (&vm)[2 * kGroups]) {
-    const uint4 m0 = *reinterpret_cast<const uint4*>(st + OPTR_V_META_OFFSET + g * 16);
-    const uint4 m1 = *reinterpret_cast<const uint4*>(st + OPTR_V_META_OFFSET + (g + 8) * 16);
+    const uint4 m0 = meta4(st + vmeta_offset(CMP), g);
+    const uint4 m1 = meta4(st + vmeta_offset(CMP), g + 8);
     vm[0] = m0.x; vm[1] = m0.y; vm[2] = m0.z; vm[3] = m0.w;
     vm[4] = m1.x; vm[5] = m1.y; vm[6] = m1.z; vm[7] = m1.w;
     __half2 mx = *reinterpret_cast<const __half2*>(&vm[0]);
@@ -701,7 +718,9 @@ cudaError_t launch_partial_tensor(const optr_params* p, const uint8_t* pool,
                                   const WinPhase& wp, cudaStream_t s) {
   const size_t dsmem = sizeof(WarpSmemTC) * kWarps;
   const bool win = wp.Ww > 0;
-  auto fn = win ? partial_tensor_kernel<true> : partial_tensor_kernel<false>;
+  const bool cmp = p->cfg.group == 128;
+  auto fn = win ? (cmp ? partial_tensor_kernel<true, true> : partial_tensor_kernel<true, false>)
+                : (cmp ? partial_tensor_kernel<false, true> : partial_tensor_kernel<false, false>);
   cudaError_t e = ensure_dynamic_smem(reinterpret_cast<const void*>(fn), dsmem);
   if (e != cudaSuccess) return e;
   return launch_pdl(fn, dim3(W / (win ? kWinIntWarps : kWarps)), dim3(kWarps * 32),

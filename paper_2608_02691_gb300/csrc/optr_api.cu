@@ -282,7 +282,7 @@ void optr_params_destroy(optr_params* p) {
 }
 
 size_t optr_page_bytes(const optr_params* p) {
-  return p ? (size_t)p->cfg.h_kv * kChunk : 0;
+  return p ? (size_t)p->cfg.h_kv * chunk_bytes(p->cfg.group == 128) : 0;
 }
 
 namespace {

@@ -14,7 +14,18 @@ constexpr int kD = OPTR_HEAD_DIM;        // 128
 constexpr int kG = OPTR_GROUP;           // 32
 constexpr int kGroups = kD / kG;         // 4
 constexpr int kPage = OPTR_PAGE_SIZE;    // 16
-constexpr int kChunk = OPTR_PAGE_HEAD_BYTES;
+constexpr int kChunk = OPTR_PAGE_HEAD_BYTES;       // G = 32 record
+constexpr int kChunk128 = OPTR_PAGE_HEAD_BYTES_G128;  // compact G = 128 record
+// Record layout by group size: bytes per (page, KV head), the value
+// metadata's offset and the metadata bytes per slot (four {scale, min}
+// pairs for G = 32, one for the compact G = 128 record).
+__host__ __device__ constexpr int chunk_bytes(bool compact) {
+  return compact ? kChunk128 : kChunk;
+}
+__host__ __device__ constexpr int vmeta_offset(bool compact) {
+  return compact ? OPTR_V_META_OFFSET_G128 : OPTR_V_META_OFFSET;
+}
+__host__ __device__ constexpr int meta_stride(bool compact) { return compact ? 4 : 16; }
 constexpr int kMaxRatio = 8;             // largest supported h_q / h_kv
 
 // Decode split-K: every decode launch uses this many warps per SM for the

@@ -23,7 +23,8 @@ _lock = threading.Lock()
 OPTR_VARIANT_DEFAULT = 0
 OPTR_VARIANT_CUDA_CORE = 1
 OPTR_VARIANT_TENSOR = 2
-PAGE_HEAD_BYTES = 1536
+PAGE_HEAD_BYTES = 1536       # record bytes per (page, KV head), G = 32
+PAGE_HEAD_BYTES_G128 = 1152  # the compact G = 128 record
 HEAD_DIM = 128
 # device error bits (optr_device_error)
 OPTR_DEVERR_PAGE_ID = 1
@@ -385,9 +386,10 @@ def optr_profile_last(p: Params) -> dict:
 
 
 def new_pool(p: Params, num_pages: int, device="cuda") -> torch.Tensor:
-    """A zero-filled pool tensor [num_pages][h_kv][1536] (uint8)."""
-    return torch.zeros(num_pages, p.h_kv, PAGE_HEAD_BYTES, dtype=torch.uint8,
-                       device=device)
+    """A zero-filled pool tensor [num_pages][h_kv][record bytes] (uint8):
+    1536 bytes per (page, KV head) for G = 32, 1152 for G = 128."""
+    rec = PAGE_HEAD_BYTES_G128 if p.cfg.group == 128 else PAGE_HEAD_BYTES
+    return torch.zeros(num_pages, p.h_kv, rec, dtype=torch.uint8, device=device)
 
 
 def new_workspace(p: Params, B: int, max_pages: int, device="cuda"):

@@ -132,9 +132,11 @@ def gpu_case(case, variant=optr.OPTR_VARIANT_DEFAULT, append_variant=0,
 
 def gpu_decode(case, pool_np, variant=optr.OPTR_VARIANT_DEFAULT,
                seq_lens=None, dev="cuda"):
-    """GPU decode over a given (oracle-written) host pool."""
+    """GPU decode over a given (oracle-written) host pool (its record size,
+    1536 or 1152 bytes, selects the G = 32 or the compact G = 128 layout)."""
+    group = 128 if pool_np.shape[-1] == 1152 else 32
     p = optr.optr_params_create(case["R_k"], case["R_v"], case["mu"],
-                                case["h_q"], decode_variant=variant)
+                                case["h_q"], decode_variant=variant, group=group)
     pool = torch.from_numpy(pool_np).to(dev)
     bt = case["block_table"].to(dev)
     lens = case["seq_lens"] if seq_lens is None else seq_lens
