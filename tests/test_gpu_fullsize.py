@@ -32,17 +32,20 @@ SEED = 0
 _cache: dict = {}
 
 
-def _gpu_full(name):
+def _gpu_full(name, group=32, clip_k=1.0, clip_v=1.0):
     """Full-size workload generated and appended on the GPU (as bench.py
     builds it), with the sampled sequences overwritten by oracle records.
-    Returns (case, pool, per-sample (oracle output, b))."""
-    if name in _cache:
-        return _cache[name]
+    Returns (case, pool, per-sample (oracle output, b)).  group = 128 uses
+    the compact record (1152 bytes per page and KV head) with the clips."""
+    key = (name, group, clip_k, clip_v)
+    if key in _cache:
+        return _cache[key]
     dev = "cuda"
     wl = synth.workload(name, SEED)
     case = synth.build_case(wl, SEED, device=dev)
     p = optr.optr_params_create(case["R_k"], case["R_v"], case["mu"],
-                                case["h_q"])
+                                case["h_q"], group=group, clip_k=clip_k,
+                                clip_v=clip_v)
     pool = optr.new_pool(p, case["num_pages"], device=dev)
     bt = case["block_table"].to(dev)
     optr.optr_kv_append(p, case["k_ctx"], case["v_ctx"],
@@ -70,10 +73,11 @@ def _gpu_full(name):
             synth.plant_needles(k, [0, n], case["mu"], q_cpu, SEED)
         npg = (n + 15) // 16
         obt = np.arange(npg, dtype=np.int32)[None]
-        opool = np.zeros((npg, h_kv, 1536), np.uint8)
+        opool = np.zeros((npg, h_kv, oracle.chunk_bytes(group)), np.uint8)
         oracle.kv_append(synth.bf16_bits(k), synth.bf16_bits(v),
                          np.array([0, n], np.int32), np.zeros(1, np.int32),
-                         obt, opool, R_k, R_v, mu)
+                         obt, opool, R_k, R_v, mu, clip_k=clip_k,
+                         clip_v=clip_v, group=group)
         ref = oracle.decode_attention(synth.bf16_bits(q_cpu[b:b + 1]), obt,
                                       np.array([n], np.int32), opool, R_k, R_v,
                                       h_kv)[0]
@@ -81,8 +85,8 @@ def _gpu_full(name):
         pool.index_copy_(0, phys, torch.from_numpy(opool).to(dev))
         refs.append((b, ref))
     torch.cuda.synchronize()
-    _cache[name] = (case, pool, refs)
-    return _cache[name]
+    _cache[key] = (case, pool, refs)
+    return _cache[key]
 
 
 @pytest.mark.parametrize("variant", DECODE_VARIANTS)
@@ -107,6 +111,33 @@ def test_full_size_decode(name, variant):
         err = float(np.abs(got[b] - ref).max())
         print(f"{name} variant {variant} seq {b}: err/rms {err / rms:.2e}")
         assert err <= OUT_TOL * rms, (name, variant, b, err / rms)
+
+
+@pytest.mark.parametrize("variant", DECODE_VARIANTS)
+def test_full_size_decode_compact_g128(variant):
+    """decode8k at full size with the paper's quantizer settings (G = 128,
+    clips 0.96 / 0.92) in the compact record: 72 B per token and KV head."""
+    case, pool, refs = _gpu_full("decode8k", 128, 0.96, 0.92)
+    assert pool.shape[-1] == 1152
+    dev = "cuda"
+    p = optr.optr_params_create(case["R_k"], case["R_v"], case["mu"],
+                                case["h_q"], decode_variant=variant, group=128,
+                                clip_k=0.96, clip_v=0.92)
+    bt = case["block_table"].to(dev)
+    out = torch.full((case["B"], case["h_q"], 128), 7.0, dtype=torch.float32,
+                     device=dev)
+    ws = optr.new_workspace(p, case["B"], bt.shape[1], device=dev)
+    optr.optr_decode_attention(p, case["q"], bt, case["seq_lens"].to(dev),
+                               pool, out, ws)
+    torch.cuda.synchronize()
+    assert optr.optr_device_error(p) == 0
+    got = out.cpu().double().numpy()
+    assert np.all(np.isfinite(got))
+    for b, ref in refs:
+        rms = float(np.sqrt(np.mean(ref ** 2)))
+        err = float(np.abs(got[b] - ref).max())
+        print(f"decode8k G=128 variant {variant} seq {b}: err/rms {err / rms:.2e}")
+        assert err <= OUT_TOL * rms, (variant, b, err / rms)
 
 
 @pytest.mark.parametrize("append_variant",
