@@ -38,8 +38,9 @@ constexpr int kCD = 128;  // head dimension d
 
 // ------------------------------------------------------------------ GEMM
 // C[b] = alpha op(A[b]) op(B[b]) + beta C[b] + diag I, float64, row-major
-// with leading dimensions; op = transpose when tA / tB.  64 x 64 tiles,
-// 16-deep k slices in shared memory, 256 threads of 4 x 4 outputs each.
+// with leading dimensions; op = transpose when tA / tB.  Square output tiles
+// of 64, 32 or 16 (gemm_f64_kernel below), 16-deep k slices in shared
+// memory, 256 threads per CTA.
 // gate: when non-null and gate_idx >= *gate, the launch instead copies
 // `pass` into C (or does nothing when pass is null); this lets a fixed
 // number of launches apply a device-decided number of squarings.
