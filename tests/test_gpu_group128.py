@@ -138,3 +138,45 @@ def test_paper_default_configuration_step(dvar):
                               win_slot=slots, sink=sink, recent=recent)
     strict, mean_bar = ph.assert_rows_within_bar(got, ref, bound, "paper defaults")
     print(f"paper defaults: strict rows {strict:.2f}, mean bar {mean_bar:.3f} x strict")
+
+
+def test_compact_step_replays_from_a_cuda_graph():
+    """The decode step on the compact G = 128 record (single-token write of
+    one pair per slot, decode reading 1152-byte records) captured in a CUDA
+    graph and replayed gives the bytes and output of direct calls."""
+    c = synth.build_case(synth.workload("decode8k", 0, 1 / 32), 0)
+    dev = "cuda"
+    res = []
+    for use_graph in (False, True):
+        p = optr.optr_params_create(c["R_k"], c["R_v"], c["mu"], c["h_q"],
+                                    clip_k=CK, clip_v=CV, group=128)
+        pool = optr.new_pool(p, c["num_pages"], device=dev)
+        assert pool.shape[-1] == 1152
+        bt = c["block_table"].to(dev)
+        optr.optr_kv_append(p, c["k_ctx"].to(dev), c["v_ctx"].to(dev),
+                            c["cu_ctx"].to(dev), c["pos0_ctx"].to(dev), bt, pool)
+        args = [c["q"].to(dev), c["k_new"].to(dev), c["v_new"].to(dev),
+                c["cu_new"].to(dev), c["pos0_new"].to(dev), bt,
+                c["seq_lens"].to(dev)]
+        out = torch.empty(c["B"], c["h_q"], 128, dtype=torch.float32, device=dev)
+        ws = optr.new_workspace(p, c["B"], bt.shape[1], device=dev)
+        torch.cuda.synchronize()
+        if use_graph:
+            s = torch.cuda.Stream()
+            s.wait_stream(torch.cuda.current_stream())
+            with torch.cuda.stream(s):  # warm-up outside the capture
+                optr.optr_decode_step(p, *args, pool, out, ws)
+            torch.cuda.current_stream().wait_stream(s)
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g):
+                optr.optr_decode_step(p, *args, pool, out, ws)
+            out.zero_()
+            g.replay()
+        else:
+            optr.optr_decode_step(p, *args, pool, out, ws)
+            optr.optr_decode_step(p, *args, pool, out, ws)
+        torch.cuda.synchronize()
+        assert optr.optr_device_error(p) == 0
+        res.append((pool.cpu(), out.cpu()))
+    assert torch.equal(res[0][0], res[1][0])
+    assert torch.equal(res[0][1], res[1][1])
