@@ -35,6 +35,7 @@
 // The quantizer is quant.cuh's float32 formula.
 #include "append_common.cuh"
 #include "decode_common.cuh"
+#include "f32x2.cuh"
 #include "quant.cuh"
 #include "tc05.cuh"
 
@@ -87,7 +88,7 @@ struct Smem {
   // token rows, bf16: [channel half][row][128 B], 16-byte chunk c of row r
   // at chunk position c ^ (r % 8) (the TMA 128-byte swizzle)
   uint8_t stage[kStages][kStageBytes];
-  alignas(16) float mu[kD];               // mu R_k (keys) or 0 (values)
+  alignas(16) float nmu[kD];              // -mu R_k (keys) or 0 (values)
   int cu[kCuCache + 1];
   int p0[kCuCache];
   uint4 xchg[2][kRows][2];               // second-half code words per row
@@ -112,13 +113,12 @@ __device__ __forceinline__ uint32_t bf16x2_to_f16x2(uint32_t u) {
 
 // Quantizer parameters of one group (quant.cuh's formula: mn = c lo,
 // mx = c hi, r = mx - mn, degenerate unless 1e-30 < r <= FLT_MAX), with the
-// two divisions done as reciprocal multiplies: inv4 = (3 / r) / 4 from
-// rcp.approx (within ~2 ulp of quant.cuh's correctly rounded 3 / r, which
-// moves only code decisions within ~1e-6 of a rounding boundary) and the
-// stored scale fp16(r * (1/3)) (at most one fp16 ulp from fp16(r / 3)).
-// A degenerate group gets inv4 = 0, which makes every code 0 below.
+// two divisions done as reciprocal multiplies: inv = 3 / r from rcp.approx
+// (within ~2 ulp of quant.cuh's correctly rounded 3 / r, which moves only
+// code decisions within ~1e-6 of a rounding boundary) and the stored scale
+// fp16(r * (1/3)) (at most one fp16 ulp from fp16(r / 3)).
 struct FastQuant {
-  float mn, mx, inv4;
+  float mn, mx, inv;
   uint32_t meta;  // (scale, min) as half2
   bool degenerate;
 };
@@ -131,7 +131,7 @@ __device__ __forceinline__ FastQuant fast_quant_params(float lo, float hi, float
   q.degenerate = !(r > 1e-30f) || !(r <= 3.402823466e38f);
   float rc;
   asm("rcp.approx.f32 %0, %1;" : "=f"(rc) : "f"(r));
-  q.inv4 = q.degenerate ? 0.f : __fmul_rn(0.75f, rc);
+  q.inv = q.degenerate ? 0.f : __fmul_rn(3.0f, rc);
   const __half2 sm = __halves2half2(
       q.degenerate ? __float2half_rn(0.f) : __float2half_rn(__fmul_rn(r, 1.0f / 3.0f)),
       __float2half_rn(q.mn));
@@ -141,30 +141,37 @@ __device__ __forceinline__ FastQuant fast_quant_params(float lo, float hi, float
 
 // Code bytes of the 32 values x of one group: byte[w] holds the codes of
 // channels 4w + r (r = 0..3) at bits 2r, in its low byte (bits 8-21 zero).
-// In x's scale (mn, mx and inv4 = inv / 4 scaled alike):
-//   v = sat((x - mn) * inv4)   u = (x - mn) * inv rounded to float, / 4
-//                              exact, clamped to [0, 1]: NaN (and every
-//                              value of a degenerate group) -> 0
-//   v * 4 + 1.5 * 2^23         rounds u to the nearest integer (ties to
-//                              even, as rint) into the low mantissa bits:
-//                              bits = 0x4B400000 + code, code <= 3
+// In x's scale (mn, mx and inv scaled alike), two values per packed
+// instruction:
+//   d = x - mn                  rounded as quant.cuh's subtraction; in
+//                               [0, r] (x lies in [mn, mx]: the group's own
+//                               extremes, or clamped to them when c < 1)
+//   d * inv + 1.5 * 2^23        one rounding takes d * inv (<= 3 + 2^-20)
+//                               to the nearest integer (ties to even, as
+//                               rint) in the low mantissa bits:
+//                               bits = 0x4B400000 + code, code <= 3
 // and sum_r bits_r 4^r = 85 * 0x4B400000 + byte, whose constant part lies
-// above bit 21.  With c = 1, x lies in [mn, mx], so no clamp of x is needed.
+// above bit 21.  Rounding d * inv once instead of twice (to float, then to
+// an integer) moves only decisions within ~2e-7 of a rounding boundary.
+// A degenerate group (also any group holding a NaN or infinity: the
+// rotation spreads one to every channel of the row) gets code 0 throughout.
 template <bool kClamp>
 __device__ __forceinline__ void code_bytes(const float (&x)[32], const FastQuant& q,
                                            uint32_t (&byte)[8]) {
+  if (q.degenerate) {
+#pragma unroll
+    for (int w = 0; w < 8; ++w) byte[w] = 0u;
+    return;
+  }
+  const float2 mn2 = make_float2(q.mn, q.mn), inv2 = make_float2(q.inv, q.inv);
+  const float2 mag2 = make_float2(12582912.0f, 12582912.0f);
+  auto xc = [&](int j) { return kClamp ? fminf(fmaxf(x[j], q.mn), q.mx) : x[j]; };
 #pragma unroll
   for (int w = 0; w < 8; ++w) {
-    uint32_t b[4];
-#pragma unroll
-    for (int r = 0; r < 4; ++r) {
-      const float xv = x[4 * w + r];
-      const float xc = kClamp ? fminf(fmaxf(xv, q.mn), q.mx) : xv;
-      float v;
-      asm("mul.rn.sat.f32 %0, %1, %2;" : "=f"(v) : "f"(__fsub_rn(xc, q.mn)), "f"(q.inv4));
-      b[r] = __float_as_uint(__fmaf_rn(v, 4.0f, 12582912.0f));
-    }
-    byte[w] = b[0] + 4u * b[1] + 16u * b[2] + 64u * b[3];
+    const float2 b01 = fma2(sub2(make_float2(xc(4 * w), xc(4 * w + 1)), mn2), inv2, mag2);
+    const float2 b23 = fma2(sub2(make_float2(xc(4 * w + 2), xc(4 * w + 3)), mn2), inv2, mag2);
+    byte[w] = __float_as_uint(b01.x) + 4u * __float_as_uint(b01.y) +
+              16u * __float_as_uint(b23.x) + 64u * __float_as_uint(b23.y);
   }
 }
 
@@ -218,7 +225,7 @@ append_tc05_kernel(const __grid_constant__ CUtensorMap tmap_k,
       cp_async16_zfill(dst + i, src + i, true);
     cp_async_commit();
   }
-  if (tid < kD) S.mu[tid] = kind ? 0.f : __ldg(muR + h * kD + tid);
+  if (tid < kD) S.nmu[tid] = kind ? 0.f : -__ldg(muR + h * kD + tid);
   if (tid == 0) {
     for (int s = 0; s < kStages; ++s) {
       tc05::bar_init(&S.full[s], 1);
@@ -394,14 +401,21 @@ append_tc05_kernel(const __grid_constant__ CUtensorMap tmap_k,
         auto row_values = [&](int e, const uint32_t (&a)[32], float (&x)[32]) {
           const int G = G2 + e;
           if (kind == 0) {
-            const float4* mu4 = reinterpret_cast<const float4*>(S.mu + 32 * G);
+            const float4* nmu4 = reinterpret_cast<const float4*>(S.nmu + 32 * G);
+            const float2 s64 = make_float2(1.0f / 64.0f, 1.0f / 64.0f);
 #pragma unroll
             for (int j4 = 0; j4 < 8; ++j4) {
-              const float4 m = mu4[j4];
-              x[4 * j4 + 0] = fmaf(__uint_as_float(a[4 * j4 + 0]), 1.0f / 64.0f, -m.x);
-              x[4 * j4 + 1] = fmaf(__uint_as_float(a[4 * j4 + 1]), 1.0f / 64.0f, -m.y);
-              x[4 * j4 + 2] = fmaf(__uint_as_float(a[4 * j4 + 2]), 1.0f / 64.0f, -m.z);
-              x[4 * j4 + 3] = fmaf(__uint_as_float(a[4 * j4 + 3]), 1.0f / 64.0f, -m.w);
+              const float4 m = nmu4[j4];
+              const float2 x01 = fma2(make_float2(__uint_as_float(a[4 * j4 + 0]),
+                                                  __uint_as_float(a[4 * j4 + 1])),
+                                      s64, make_float2(m.x, m.y));
+              const float2 x23 = fma2(make_float2(__uint_as_float(a[4 * j4 + 2]),
+                                                  __uint_as_float(a[4 * j4 + 3])),
+                                      s64, make_float2(m.z, m.w));
+              x[4 * j4 + 0] = x01.x;
+              x[4 * j4 + 1] = x01.y;
+              x[4 * j4 + 2] = x23.x;
+              x[4 * j4 + 3] = x23.y;
             }
           } else {
 #pragma unroll
@@ -413,7 +427,7 @@ append_tc05_kernel(const __grid_constant__ CUtensorMap tmap_k,
           range_err |= q.degenerate && !(fabsf(hi - lo) <= 3.402823466e38f);
           q.mn *= xs;
           q.mx *= xs;
-          q.inv4 *= 1.0f / xs;
+          q.inv *= 1.0f / xs;
           return q;
         };
         if constexpr (kG128) {
