@@ -99,6 +99,20 @@
  * device memory of the current CUDA device; "host" pointers are read
  * synchronously before the call returns.
  *
+ * Activations in host memory
+ * --------------------------
+ * The per-step activations -- k and v of a cache write, q and out of a
+ * decode, all four of a decode step ("device or pinned host" below) -- may
+ * instead be page-locked host memory (cudaHostAlloc, or host memory
+ * registered with cudaHostRegister) that the runtime maps into the
+ * device's address space.  The kernels then read and write them in place
+ * over the host link (NVLink-C2C on a Grace host), so a step's host-device
+ * transfers happen inside its own kernels, with no staging copies.
+ * Pageable host memory, or a pointer the CUDA runtime does not know, is
+ * refused with OPTR_ERR_INVALID_ARG before any launch.  A cache write of
+ * more than 256 tokens from host memory runs on the CUDA-core kernel (the
+ * tensor-core kernel loads its input by TMA from device memory).
+ *
  * Errors
  * ------
  * Argument errors are detected on the host before any launch and return a
@@ -207,7 +221,8 @@ size_t optr_page_bytes(const optr_params* p);
 
 /*
  * Cache write (Sec. 4.1; Appendix, key-mean estimation and application).
- *   k, v        device bf16 [n_tok][h_kv][D]: new keys (post-RoPE) and values.
+ *   k, v        device or pinned host bf16 [n_tok][h_kv][D]: new keys
+ *               (post-RoPE) and values.
  *   n_tok       host; total new tokens (0 is a no-op).
  *   cu_new      device int32 [B+1]: tokens of sequence b are rows
  *               cu_new[b] .. cu_new[b+1]-1 of k / v; cu_new[0] = 0,
@@ -239,11 +254,13 @@ size_t optr_decode_workspace_size(const optr_params* p, int B, int max_pages);
 /*
  * Decode attention over the paged INT2 cache (Sec. 3 Eq. 1-2; Appendix,
  * rotated-query implementation and equivalent inference implementation).
- *   q           device bf16 [B][h_q][D]: post-RoPE queries, one per sequence.
+ *   q           device or pinned host bf16 [B][h_q][D]: post-RoPE queries,
+ *               one per sequence.
  *   block_table device int32 [B][max_pages].
  *   seq_lens    device int32 [B]: cached tokens per sequence, 0 .. max_pages*16.
  *   pool        device bytes [num_pages][h_kv][1536] (read only).
- *   out         device float32 [B][h_q][D]: attention output o = o' R_v^T.
+ *   out         device or pinned host float32 [B][h_q][D]: attention output
+ *               o = o' R_v^T.
  *   workspace   device, at least optr_decode_workspace_size(p, B, max_pages)
  *               bytes, 256-byte aligned; contents need no initialisation and
  *               are scratch between calls (concurrent calls need distinct

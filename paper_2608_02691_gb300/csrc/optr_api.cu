@@ -26,6 +26,30 @@ optr_status cuda_status(cudaError_t e) {
 
 size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
+// A per-step activation (k, v, q or out) as the kernels address it: device
+// or managed memory as given; page-locked host memory through its device
+// mapping (*host set), which the kernels then read or write in place over
+// the host link.  Pageable host memory, or a pointer the runtime does not
+// know, is refused (false), so no kernel ever dereferences it.
+bool io_pointer(const void* ptr, const void** dev, bool* host) {
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, ptr) != cudaSuccess) {
+    (void)cudaGetLastError();  // the failed query leaves no error behind
+    return false;
+  }
+  if (a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged) {
+    *dev = ptr;
+    if (host) *host = false;
+    return true;
+  }
+  if (a.type == cudaMemoryTypeHost && a.devicePointer != nullptr) {
+    *dev = a.devicePointer;
+    if (host) *host = true;
+    return true;
+  }
+  return false;
+}
+
 }  // namespace
 
 namespace optr {
@@ -334,14 +358,18 @@ optr_status optr_kv_append_win(const optr_params* p, const void* k,
     return OPTR_ERR_INVALID_ARG;
   if (!aligned(pool, 16) || !aligned(k, 16) || !aligned(v, 16))
     return OPTR_ERR_INVALID_ARG;
+  bool k_host = false, v_host = false;
+  if (!io_pointer(k, &k, &k_host) || !io_pointer(v, &v, &v_host))
+    return OPTR_ERR_INVALID_ARG;
   if ((long long)max_pages * kPage > (1LL << 30)) return OPTR_ERR_OUT_OF_RANGE;
   const int variant = p->cfg.append_variant;
   prof_mark(p, 0, stream);
   cudaError_t e;
   // decode-step sized appends (<= 256 tokens) use the slice-parallel
   // CUDA-core kernel under every variant; larger ones the tensor-core kernel
-  // unless the CUDA-core variant is requested
-  if (variant == OPTR_VARIANT_CUDA_CORE || n_tok <= 256)
+  // unless the CUDA-core variant is requested or the input is in host
+  // memory (the tensor-core kernel loads it by TMA from device memory)
+  if (variant == OPTR_VARIANT_CUDA_CORE || n_tok <= 256 || k_host || v_host)
     e = launch_append_cuda_core(p, (const __nv_bfloat16*)k,
                                 (const __nv_bfloat16*)v, n_tok, cu_new, pos0,
                                 block_table, B, max_pages, pool, num_pages,
@@ -387,6 +415,12 @@ optr_status optr_decode_attention_win(const optr_params* p, const void* q,
   const optr_status st = decode_args_status(p, q, block_table, seq_lens, B,
                                             max_pages, pool, num_pages, out);
   if (st != OPTR_OK) return st;
+  {
+    const void* od = nullptr;
+    if (!io_pointer(q, &q, nullptr) || !io_pointer(out, &od, nullptr))
+      return OPTR_ERR_INVALID_ARG;
+    out = static_cast<float*>(const_cast<void*>(od));
+  }
   WinArgs wbuf;
   bool bad = false;
   const WinArgs* wa = window_args(p, const_cast<void*>(win), win_slot, n_slots,
@@ -456,6 +490,13 @@ optr_status optr_decode_step_win(const optr_params* p, const void* q,
     return optr_decode_attention_win(p, q, block_table, seq_lens, B, max_pages,
                                      pool, num_pages, win, win_slot, n_slots,
                                      out, workspace, ws_bytes, stream);
+  }
+  {
+    const void* od = nullptr;
+    if (!io_pointer(q, &q, nullptr) || !io_pointer(k, &k, nullptr) ||
+        !io_pointer(v, &v, nullptr) || !io_pointer(out, &od, nullptr))
+      return OPTR_ERR_INVALID_ARG;
+    out = static_cast<float*>(const_cast<void*>(od));
   }
   StepAppend app{(const __nv_bfloat16*)k, (const __nv_bfloat16*)v, n_tok,
                  cu_new, pos0, pool};

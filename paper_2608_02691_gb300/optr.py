@@ -140,9 +140,16 @@ def _stream(stream):
     return ctypes.c_void_p(stream.cuda_stream)
 
 
+# per-step activations: CUDA tensors or pinned host tensors, which the
+# kernels read or write in place
+_IO = ("q", "k", "v", "out")
+
+
 def _dev(t, dtype, name):
-    if not (t.is_cuda and t.dtype == dtype and t.is_contiguous()):
-        raise ValueError(f"{name} must be a contiguous CUDA {dtype} tensor")
+    where = t.is_cuda or (name in _IO and t.is_pinned())
+    if not (where and t.dtype == dtype and t.is_contiguous()):
+        kind = "CUDA or pinned host" if name in _IO else "CUDA"
+        raise ValueError(f"{name} must be a contiguous {kind} {dtype} tensor")
     return t
 
 
