@@ -429,6 +429,11 @@ def extra_workloads(args, dev):
                                                   group=128, clip_k=0.96,
                                                   clip_v=0.92)
     torch.cuda.empty_cache()
+    # the compact G = 128 record (72 B per token and KV head) without windows
+    res["decode8k_g128"] = windows_step(args, dev, flush, hbm_peak, sink=0,
+                                        recent=0, group=128, clip_k=0.96,
+                                        clip_v=0.92)
+    torch.cuda.empty_cache()
 
     for name in ("long128k", "ragged"):
         wl, case, p, pool, bt = setup_decode(name, args.seed, dev, args.variant,
@@ -545,7 +550,8 @@ def windows_step(args, dev, flush, hbm_peak, sink=64, recent=256, group=32,
                  clip_k=1.0, clip_v=1.0):
     """The decode8k step with the paper's BF16 windows (64 sink, 256 recent
     tokens; Sec. 5), optionally with its G = 128 and clip ratios:
-    optr_decode_step_win, L2 flushed before every step."""
+    optr_decode_step_win, L2 flushed before every step.  sink = recent = 0:
+    the same step without windows (optr_decode_step)."""
     from paper_2608_02691_gb300 import optr, synth
     wl = synth.workload("decode8k", args.seed)
     case = synth.build_case(wl, args.seed, device=dev)
@@ -556,12 +562,17 @@ def windows_step(args, dev, flush, hbm_peak, sink=64, recent=256, group=32,
                                 clip_v=clip_v)
     B, h_q, h_kv = case["B"], case["h_q"], case["h_kv"]
     pool = optr.new_pool(p, case["num_pages"], device=dev)
-    win = optr.new_windows(p, B, device=dev)
-    slot = torch.arange(B, dtype=torch.int32, device=dev)
+    windows = sink > 0 or recent > 0
     bt = case["block_table"].to(dev)
-    optr.optr_kv_append_win(p, case["k_ctx"], case["v_ctx"],
-                            case["cu_ctx"].to(dev), case["pos0_ctx"].to(dev),
-                            bt, pool, win, slot)
+    if windows:
+        win = optr.new_windows(p, B, device=dev)
+        slot = torch.arange(B, dtype=torch.int32, device=dev)
+        optr.optr_kv_append_win(p, case["k_ctx"], case["v_ctx"],
+                                case["cu_ctx"].to(dev), case["pos0_ctx"].to(dev),
+                                bt, pool, win, slot)
+    else:
+        optr.optr_kv_append(p, case["k_ctx"], case["v_ctx"], case["cu_ctx"].to(dev),
+                            case["pos0_ctx"].to(dev), bt, pool)
     seq = case["seq_lens"].to(dev)
     q = case["q"].to(dev)
     k_new, v_new = case["k_new"].to(dev), case["v_new"].to(dev)
@@ -571,8 +582,12 @@ def windows_step(args, dev, flush, hbm_peak, sink=64, recent=256, group=32,
     stream = torch.cuda.current_stream()
 
     def step():
-        optr.optr_decode_step_win(p, q, k_new, v_new, cu_new, pos0, bt, seq,
-                                  pool, win, slot, out, ws)
+        if windows:
+            optr.optr_decode_step_win(p, q, k_new, v_new, cu_new, pos0, bt, seq,
+                                      pool, win, slot, out, ws)
+        else:
+            optr.optr_decode_step(p, q, k_new, v_new, cu_new, pos0, bt, seq,
+                                  pool, out, ws)
 
     for _ in range(3):
         flush()
@@ -599,7 +614,8 @@ def windows_step(args, dev, flush, hbm_peak, sink=64, recent=256, group=32,
     lens = case["seq_lens"].tolist()
     n_new = k_new.shape[0]
     nb = (decode_bytes_win(lens, h_kv, h_q, sink, recent, group) +
-          append_bytes(n_new, h_kv, group) + n_new * h_kv * 512)  # + window copies
+          append_bytes(n_new, h_kv, group) +
+          (n_new * h_kv * 512 if windows else 0))  # + window copies
     i2 = sum(window_split(x, sink, recent)[0] for x in lens)
     wt = sum(window_split(x, sink, recent)[1] for x in lens)
     pb = i2 * h_kv * record_bytes(group) + wt * h_kv * 512  # what the partial kernel streams

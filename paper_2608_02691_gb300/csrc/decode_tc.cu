@@ -376,7 +376,7 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
 #pragma unroll
     for (int o = 4; o < 32; o <<= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
 #pragma unroll
-    for (int G = 0; G < kGroups; ++G)
+    for (int G = 0; G < (CMP ? 1 : kGroups); ++G)
 #pragma unroll
       for (int o = 4; o < 32; o <<= 1)
         mv[G] += __shfl_xor_sync(0xffffffffu, mv[G], o);
@@ -387,11 +387,12 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
     for (int G = 0; G < kGroups; ++G) {
       // rows g (r = 2*half) and g+8 (r = 2*half+1) of tile (G, half) are
       // channels 32G + 4g + r
+      const float mvG = mv[CMP ? 0 : G];  // CMP: one (scale, min) per token
       float4 o4;
-      o4.x = (acc_o[G][0][0] + acc_o[G][0][1]) + mv[G];
-      o4.y = (acc_o[G][0][2] + acc_o[G][0][3]) + mv[G];
-      o4.z = (acc_o[G][1][0] + acc_o[G][1][1]) + mv[G];
-      o4.w = (acc_o[G][1][2] + acc_o[G][1][3]) + mv[G];
+      o4.x = (acc_o[G][0][0] + acc_o[G][0][1]) + mvG;
+      o4.y = (acc_o[G][0][2] + acc_o[G][0][3]) + mvG;
+      o4.z = (acc_o[G][1][0] + acc_o[G][1][1]) + mvG;
+      o4.w = (acc_o[G][1][2] + acc_o[G][1][3]) + mvG;
       *reinterpret_cast<float4*>(dst + 32 * G + 4 * g) = o4;
     }
     if (g == 0) {
@@ -414,10 +415,18 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
       const float4* ko = reinterpret_cast<const float4*>(
           koff + ((size_t)cb * h_kv + ch) * 32 + c * 8);
       const float4 k01 = __ldcg(ko), k23 = __ldcg(ko + 1);
-      S.kq[0][lane] = make_float4(-k01.x, -k01.y, -k01.x, -k01.y);
-      S.kq[1][lane] = make_float4(-k01.z, -k01.w, -k01.z, -k01.w);
-      S.kq[2][lane] = make_float4(-k23.x, -k23.y, -k23.x, -k23.y);
-      S.kq[3][lane] = make_float4(-k23.z, -k23.w, -k23.z, -k23.w);
+      if constexpr (CMP) {
+        // one scale per token: the four groups share one accumulator,
+        // started from the sum of their offsets
+        const float hi = -((k01.x + k01.z) + (k23.x + k23.z));
+        const float lo = -((k01.y + k01.w) + (k23.y + k23.w));
+        S.kq[0][lane] = make_float4(hi, lo, hi, lo);
+      } else {
+        S.kq[0][lane] = make_float4(-k01.x, -k01.y, -k01.x, -k01.y);
+        S.kq[1][lane] = make_float4(-k01.z, -k01.w, -k01.z, -k01.w);
+        S.kq[2][lane] = make_float4(-k23.x, -k23.y, -k23.x, -k23.y);
+        S.kq[3][lane] = make_float4(-k23.z, -k23.w, -k23.z, -k23.w);
+      }
     }
     const size_t row = (size_t)cb * h_q + 4 * ch + c;
     {
@@ -465,6 +474,10 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
     const uint32_t y01_1 = __byte_perm(k1.x, k1.y, 0x5410);
     const uint32_t y23_1 = __byte_perm(k1.x, k1.y, 0x7632);
     float s_acc[kGroups][4];
+    if constexpr (CMP) {
+      const float4 kv = S.kq[0][lane];
+      s_acc[0][0] = kv.x; s_acc[0][1] = kv.y; s_acc[0][2] = kv.z; s_acc[0][3] = kv.w;
+    }
 #pragma unroll
     for (int j = 0; j < 2; ++j) {  // groups 2j, 2j+1
       uint32_t f0[2][4], f1[2][4];  // token rows g, g+8
@@ -473,34 +486,41 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
 #pragma unroll
       for (int par = 0; par < 2; ++par) {
         const int G = 2 * j + par;
+        const int A = CMP ? 0 : G;  // accumulator of the group's scale
         const uint4 qv = S.qfr[G][lane];
-        const float4 kv = S.kq[G][lane];
-        s_acc[G][0] = kv.x; s_acc[G][1] = kv.y; s_acc[G][2] = kv.z; s_acc[G][3] = kv.w;
-        mma16816(s_acc[G], f0[par][0], f1[par][0], f0[par][1], f1[par][1], qv.x, qv.y);
-        mma16816(s_acc[G], f0[par][2], f1[par][2], f0[par][3], f1[par][3], qv.z, qv.w);
+        if constexpr (!CMP) {
+          const float4 kv = S.kq[G][lane];
+          s_acc[G][0] = kv.x; s_acc[G][1] = kv.y; s_acc[G][2] = kv.z; s_acc[G][3] = kv.w;
+        }
+        mma16816(s_acc[A], f0[par][0], f1[par][0], f0[par][1], f1[par][1], qv.x, qv.y);
+        mma16816(s_acc[A], f0[par][2], f1[par][2], f0[par][3], f1[par][3], qv.z, qv.w);
       }
     }
-    const uint4 km0 = meta4(st + OPTR_K_META_OFFSET, g);
-    const uint4 km1 = meta4(st + OPTR_K_META_OFFSET, g + 8);
-    const uint32_t kmv0[4] = {km0.x, km0.y, km0.z, km0.w};
-    const uint32_t kmv1[4] = {km1.x, km1.y, km1.z, km1.w};
     // sum_g min_g * sum(q' over g) on the tensor core: A row t = the 8
     // (scale, min) halves of token t, B = (0, Q_g) per (scale, min) pair
     float u[4] = {0.f, 0.f, 0.f, 0.f};
-    {
-      const uint32_t w0 = *reinterpret_cast<const uint32_t*>(
-          st + OPTR_K_META_OFFSET + g * meta_stride(CMP) + (CMP ? 0 : 4 * c));
-      const uint32_t w1 = *reinterpret_cast<const uint32_t*>(
-          st + OPTR_K_META_OFFSET + (g + 8) * meta_stride(CMP) + (CMP ? 0 : 4 * c));
-      mma16816(u, w0, w1, 0u, 0u, bmin, 0u);
-    }
+    const uint32_t w0 = *reinterpret_cast<const uint32_t*>(
+        st + OPTR_K_META_OFFSET + g * meta_stride(CMP) + (CMP ? 0 : 4 * c));
+    const uint32_t w1 = *reinterpret_cast<const uint32_t*>(
+        st + OPTR_K_META_OFFSET + (g + 8) * meta_stride(CMP) + (CMP ? 0 : 4 * c));
+    mma16816(u, w0, w1, 0u, 0u, bmin, 0u);
     float t0 = 0.f, t1 = 0.f;
+    if constexpr (CMP) {
+      // the one (scale, min) pair of tokens g and g+8 is w0 and w1
+      t0 = __low2float(*reinterpret_cast<const __half2*>(&w0)) * (s_acc[0][0] + s_acc[0][1]);
+      t1 = __low2float(*reinterpret_cast<const __half2*>(&w1)) * (s_acc[0][2] + s_acc[0][3]);
+    } else {
+      const uint4 km0 = meta4(st + OPTR_K_META_OFFSET, g);
+      const uint4 km1 = meta4(st + OPTR_K_META_OFFSET, g + 8);
+      const uint32_t kmv0[4] = {km0.x, km0.y, km0.z, km0.w};
+      const uint32_t kmv1[4] = {km1.x, km1.y, km1.z, km1.w};
 #pragma unroll
-    for (int G = 0; G < kGroups; ++G) {
-      const float a = __low2float(*reinterpret_cast<const __half2*>(&kmv0[G]));   // scale, token g
-      const float bb = __low2float(*reinterpret_cast<const __half2*>(&kmv1[G]));  // token g+8
-      t0 = fmaf(a, s_acc[G][0] + s_acc[G][1], t0);
-      t1 = fmaf(bb, s_acc[G][2] + s_acc[G][3], t1);
+      for (int G = 0; G < kGroups; ++G) {
+        const float a = __low2float(*reinterpret_cast<const __half2*>(&kmv0[G]));   // scale, token g
+        const float bb = __low2float(*reinterpret_cast<const __half2*>(&kmv1[G]));  // token g+8
+        t0 = fmaf(a, s_acc[G][0] + s_acc[G][1], t0);
+        t1 = fmaf(bb, s_acc[G][2] + s_acc[G][3], t1);
+      }
     }
     sc0 = fmaf(inv_s, t0, u[0] + u[1]);
     sc1 = fmaf(inv_s, t1, u[2] + u[3]);
@@ -508,15 +528,25 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
 
   // value (scale, min) halves of tokens g (vm[0..3]) and g+8 (vm[4..7])
   // per group, kept packed; returns their largest scale
+  // (CMP: the one pair of tokens g and g+8 in vm[0] and vm[kGroups])
   auto vmeta = [&](const uint8_t* st, uint32_t (&vm)[2 * kGroups]) {
-    const uint4 m0 = meta4(st + vmeta_offset(CMP), g);
-    const uint4 m1 = meta4(st + vmeta_offset(CMP), g + 8);
-    vm[0] = m0.x; vm[1] = m0.y; vm[2] = m0.z; vm[3] = m0.w;
-    vm[4] = m1.x; vm[5] = m1.y; vm[6] = m1.z; vm[7] = m1.w;
-    __half2 mx = *reinterpret_cast<const __half2*>(&vm[0]);
+    if constexpr (CMP) {
+      const uint8_t* region = st + vmeta_offset(true);
+      vm[0] = *reinterpret_cast<const uint32_t*>(region + g * 4);
+      vm[kGroups] = *reinterpret_cast<const uint32_t*>(region + (g + 8) * 4);
+      const __half2 mx = __hmax2(*reinterpret_cast<const __half2*>(&vm[0]),
+                                 *reinterpret_cast<const __half2*>(&vm[kGroups]));
+      return __low2float(mx);
+    } else {
+      const uint4 m0 = meta4(st + vmeta_offset(CMP), g);
+      const uint4 m1 = meta4(st + vmeta_offset(CMP), g + 8);
+      vm[0] = m0.x; vm[1] = m0.y; vm[2] = m0.z; vm[3] = m0.w;
+      vm[4] = m1.x; vm[5] = m1.y; vm[6] = m1.z; vm[7] = m1.w;
+      __half2 mx = *reinterpret_cast<const __half2*>(&vm[0]);
 #pragma unroll
-    for (int i = 1; i < 2 * kGroups; ++i) mx = __hmax2(mx, *reinterpret_cast<const __half2*>(&vm[i]));
-    return __low2float(mx);  // scales are >= 0 (fp16 max ignores a NaN min half)
+      for (int i = 1; i < 2 * kGroups; ++i) mx = __hmax2(mx, *reinterpret_cast<const __half2*>(&vm[i]));
+      return __low2float(mx);  // scales are >= 0 (fp16 max ignores a NaN min half)
+    }
   };
 
   // Lazy reference: p = 2^(l - m_ref) with m_ref = m_lazy + k_s - 15,
@@ -548,7 +578,7 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
         l_lane *= alpha;
 #pragma unroll
         for (int G = 0; G < kGroups; ++G) {
-          mv[G] *= alpha;
+          if (!CMP || G == 0) mv[G] *= alpha;
 #pragma unroll
           for (int hf = 0; hf < 2; ++hf)
 #pragma unroll
@@ -563,7 +593,7 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
   auto vprod = [&](float p0, float p1, const uint32_t (&vm)[2 * kGroups],
                    uint32_t (&pt)[kGroups][kPage][4]) {
 #pragma unroll
-    for (int G = 0; G < kGroups; ++G) {
+    for (int G = 0; G < (CMP ? 1 : kGroups); ++G) {  // CMP: one pair per token
       const float2 va = h2f(vm[G]), vb = h2f(vm[kGroups + G]);  // tokens g, g+8
       // the MMA sees centered codes (code - 1.5): the min term carries
       // min + 1.5 * scale
@@ -579,10 +609,15 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
     uint32_t bv[kGroups][2];
     {
       // lanes 0-7 address rows 0-7 of group G, 8-15 rows 8-15, 16-31 the
-      // same for group G+1
-      const int r = lane & 15, gsel = lane >> 4;
+      // same for group G+1 (CMP: every group's operand is group 0's)
+      const int r = lane & 15, gsel = CMP ? 0 : lane >> 4;
       ldsm_x4_trans(bv[0][0], bv[0][1], bv[1][0], bv[1][1], &pt[gsel][r][0]);
-      ldsm_x4_trans(bv[2][0], bv[2][1], bv[3][0], bv[3][1], &pt[2 + gsel][r][0]);
+      if constexpr (CMP) {
+        bv[2][0] = bv[0][0]; bv[2][1] = bv[0][1];
+        bv[3][0] = bv[0][0]; bv[3][1] = bv[0][1];
+      } else {
+        ldsm_x4_trans(bv[2][0], bv[2][1], bv[3][0], bv[3][1], &pt[2 + gsel][r][0]);
+      }
     }
     const uint8_t* vc = st + OPTR_V_CODES_OFFSET + 4 * g;
     const uint32_t x0 = *reinterpret_cast<const uint32_t*>(vc + (2 * c) * 32);
@@ -625,14 +660,18 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
     }
     float smax = vmeta(st, vm);
     if (!FULL) {
+      constexpr int nG = CMP ? 1 : kGroups;
 #pragma unroll
-      for (int G = 0; G < kGroups; ++G) {
+      for (int G = 0; G < nG; ++G) {
         vm[G] = v0 ? vm[G] : 0u;
         vm[kGroups + G] = v1 ? vm[kGroups + G] : 0u;
       }
       __half2 mx = *reinterpret_cast<const __half2*>(&vm[0]);
 #pragma unroll
-      for (int i = 1; i < 2 * kGroups; ++i) mx = __hmax2(mx, *reinterpret_cast<const __half2*>(&vm[i]));
+      for (int G = 0; G < nG; ++G) {
+        mx = __hmax2(mx, *reinterpret_cast<const __half2*>(&vm[G]));
+        mx = __hmax2(mx, *reinterpret_cast<const __half2*>(&vm[kGroups + G]));
+      }
       smax = __low2float(mx);
     }
     reference(fmaxf(sc0, sc1), smax);
