@@ -796,6 +796,10 @@ def main():
                     for k, v in m["case"].items()}
         del m["pool"], m["case"]
         cpu = cpu_baseline(case_cpu, args.cpu_seqs, os.cpu_count() or 1)
+        # the same oracle on one host core, on one sequence of the batch
+        one = cpu_baseline(case_cpu, 1, 1)
+        cpu["single_thread"] = {k: one[k] for k in ("value", "unit", "cores",
+                                                    "seconds_per_step", "sample")}
     if rank == 0:
         value = job_value(m["bytes"], m["ms"], world)
         e2e = (None if not np.isfinite(m["e2e_ms"]) else
