@@ -174,30 +174,41 @@ __device__ __forceinline__ void append_small_body(
     }
     g128 = group_quant_params(lo, hi, clip);
   }
+  // the four groups' range reductions, parameters and codes interleaved
+  // (four independent shuffle chains instead of one after another)
+  GroupQuant gq[kGroups];
+  if (group128) {
+#pragma unroll
+    for (int g = 0; g < kGroups; ++g) gq[g] = g128;
+  } else {
+    float lo[kGroups], hi[kGroups];
+#pragma unroll
+    for (int g = 0; g < kGroups; ++g) lo[g] = hi[g] = zv[g];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1)
+#pragma unroll
+      for (int g = 0; g < kGroups; ++g) {
+        lo[g] = fminf(lo[g], __shfl_xor_sync(0xffffffffu, lo[g], o));
+        hi[g] = fmaxf(hi[g], __shfl_xor_sync(0xffffffffu, hi[g], o));
+      }
+#pragma unroll
+    for (int g = 0; g < kGroups; ++g) gq[g] = group_quant_params(lo[g], hi[g], clip);
+  }
+  unsigned bits[kGroups];
+#pragma unroll
+  for (int g = 0; g < kGroups; ++g) bits[g] = (unsigned)quant_code(zv[g], gq[g]) << (2 * (lane & 3));
+#pragma unroll
+  for (int g = 0; g < kGroups; ++g) bits[g] |= __shfl_xor_sync(0xffffffffu, bits[g], 1);
+#pragma unroll
+  for (int g = 0; g < kGroups; ++g) bits[g] |= __shfl_xor_sync(0xffffffffu, bits[g], 2);
 #pragma unroll
   for (int g = 0; g < kGroups; ++g) {
-    const float z = zv[g];
-    GroupQuant gq;
-    if (group128) {
-      gq = g128;
-    } else {
-      float lo = z, hi = z;
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) {
-        lo = fminf(lo, __shfl_xor_sync(0xffffffffu, lo, o));
-        hi = fmaxf(hi, __shfl_xor_sync(0xffffffffu, hi, o));
-      }
-      gq = group_quant_params(lo, hi, clip);
-    }
-    unsigned bits = (unsigned)quant_code(z, gq) << (2 * (lane & 3));
-    bits |= __shfl_xor_sync(0xffffffffu, bits, 1);
-    bits |= __shfl_xor_sync(0xffffffffu, bits, 2);
     if ((lane & 3) == 0)
-      chunk[codes_off + wslot * 32 + 4 * (lane >> 2) + g] = (uint8_t)bits;
+      chunk[codes_off + wslot * 32 + 4 * (lane >> 2) + g] = (uint8_t)bits[g];
     if (lane == 0 && (!group128 || g == 0))
       *reinterpret_cast<__half2*>(chunk + meta_off + wslot * meta_stride(group128) +
                                   (group128 ? 0 : 4 * g)) =
-          __halves2half2(gq.scale, gq.min);
+          __halves2half2(gq[g].scale, gq[g].min);
   }
 }
 
