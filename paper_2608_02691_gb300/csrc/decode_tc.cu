@@ -196,13 +196,23 @@ __device__ __forceinline__ void load_chunk(PageChunk& ch, int base, int f1,
 }
 
 // spref[b] = pages of sequences < b (b <= B <= kPrefCache; invalid lengths
-// count as empty), by one block-wide scan; ends with __syncthreads().
+// count as empty), by one block-wide scan; ends with __syncthreads().  In a
+// decode step (step_cu set) also sstep[0][b] = the step's new tokens of
+// sequence b and sstep[1][b] = their first position, loaded together with
+// the lengths.
 __device__ __noinline__ void page_prefix(const int32_t* __restrict__ seq_lens,
                                          int B, int max_pages, int* spref,
-                                         int* wsum, int sink, int recent) {
+                                         int* wsum, int sink, int recent,
+                                         const int32_t* __restrict__ step_cu,
+                                         const int32_t* __restrict__ step_pos0,
+                                         int (*sstep)[kPrefCache]) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   int np = 0;
   if ((int)threadIdx.x < B) {
+    if (step_cu != nullptr) {
+      sstep[0][threadIdx.x] = __ldg(step_cu + threadIdx.x + 1) - __ldg(step_cu + threadIdx.x);
+      sstep[1][threadIdx.x] = __ldg(step_pos0 + threadIdx.x);
+    }
     const int len = __ldg(seq_lens + threadIdx.x);
     if (len >= 0 && (long long)len <= (long long)max_pages * kPage)
       np = int2_pages(len, sink, recent);
@@ -249,6 +259,7 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
   extern __shared__ __align__(16) unsigned char dsm_[];
   WarpSmemTC* smem = reinterpret_cast<WarpSmemTC*>(dsm_);  // [kWarps]
   __shared__ int spref[kPrefCache + 1];
+  __shared__ int sstep[2][kPrefCache];  // decode step: new tokens, first position
   __shared__ int wsum[kWarps];
   uint32_t e1024;
   asm volatile("mov.b32 %0, 0x64006400;" : "=r"(e1024));
@@ -275,7 +286,8 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
   static_assert(kPrefCache < kWarps * 32, "one thread per sequence");
   int F;
   if (cached) {
-    page_prefix(seq_lens, B, max_pages, spref, wsum, sink, recent);
+    page_prefix(seq_lens, B, max_pages, spref, wsum, sink, recent, step_cu, step_pos0,
+                sstep);
     F = spref[B] * h_kv;
   } else {
     pdl_wait();
@@ -347,8 +359,9 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
     bool safe = true;
     if (lane < 2 && f0 + lane < f1 && chk.key >= 0) {
       const int b = chk.key / h_kv;
-      const long long n = (long long)__ldg(step_cu + b + 1) - __ldg(step_cu + b);
-      const long long s0 = __ldg(step_pos0 + b);
+      const long long n = cached ? sstep[0][b]
+                                 : (long long)__ldg(step_cu + b + 1) - __ldg(step_cu + b);
+      const long long s0 = cached ? sstep[1][b] : __ldg(step_pos0 + b);
       const long long t0 = (long long)lpage * kPage;
       safe = n <= 0 || s0 >= t0 + kPage || s0 + n <= t0;
     }
@@ -496,20 +509,8 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
         mma16816(s_acc[A], f0[par][2], f1[par][2], f0[par][3], f1[par][3], qv.z, qv.w);
       }
     }
-    // sum_g min_g * sum(q' over g) on the tensor core: A row t = the 8
-    // (scale, min) halves of token t, B = (0, Q_g) per (scale, min) pair
-    float u[4] = {0.f, 0.f, 0.f, 0.f};
-    const uint32_t w0 = *reinterpret_cast<const uint32_t*>(
-        st + OPTR_K_META_OFFSET + g * meta_stride(CMP) + (CMP ? 0 : 4 * c));
-    const uint32_t w1 = *reinterpret_cast<const uint32_t*>(
-        st + OPTR_K_META_OFFSET + (g + 8) * meta_stride(CMP) + (CMP ? 0 : 4 * c));
-    mma16816(u, w0, w1, 0u, 0u, bmin, 0u);
     float t0 = 0.f, t1 = 0.f;
-    if constexpr (CMP) {
-      // the one (scale, min) pair of tokens g and g+8 is w0 and w1
-      t0 = __low2float(*reinterpret_cast<const __half2*>(&w0)) * (s_acc[0][0] + s_acc[0][1]);
-      t1 = __low2float(*reinterpret_cast<const __half2*>(&w1)) * (s_acc[0][2] + s_acc[0][3]);
-    } else {
+    if constexpr (!CMP) {
       const uint4 km0 = meta4(st + OPTR_K_META_OFFSET, g);
       const uint4 km1 = meta4(st + OPTR_K_META_OFFSET, g + 8);
       const uint32_t kmv0[4] = {km0.x, km0.y, km0.z, km0.w};
@@ -521,6 +522,19 @@ partial_tensor_kernel(const uint8_t* __restrict__ pool,
         t0 = fmaf(a, s_acc[G][0] + s_acc[G][1], t0);
         t1 = fmaf(bb, s_acc[G][2] + s_acc[G][3], t1);
       }
+    }
+    // sum_g min_g * sum(q' over g) on the tensor core: A row t = the 8
+    // (scale, min) halves of token t, B = (0, Q_g) per (scale, min) pair
+    float u[4] = {0.f, 0.f, 0.f, 0.f};
+    const uint32_t w0 = *reinterpret_cast<const uint32_t*>(
+        st + OPTR_K_META_OFFSET + g * meta_stride(CMP) + (CMP ? 0 : 4 * c));
+    const uint32_t w1 = *reinterpret_cast<const uint32_t*>(
+        st + OPTR_K_META_OFFSET + (g + 8) * meta_stride(CMP) + (CMP ? 0 : 4 * c));
+    mma16816(u, w0, w1, 0u, 0u, bmin, 0u);
+    if constexpr (CMP) {
+      // the one (scale, min) pair of tokens g and g+8 is w0 and w1
+      t0 = __low2float(*reinterpret_cast<const __half2*>(&w0)) * (s_acc[0][0] + s_acc[0][1]);
+      t1 = __low2float(*reinterpret_cast<const __half2*>(&w1)) * (s_acc[0][2] + s_acc[0][3]);
     }
     sc0 = fmaf(inv_s, t0, u[0] + u[1]);
     sc1 = fmaf(inv_s, t1, u[2] + u[3]);
