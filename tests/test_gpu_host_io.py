@@ -145,3 +145,33 @@ def test_pageable_host_memory_is_refused():
     assert torch.all(out_d == 3.0)
     with pytest.raises(ValueError):
         optr.optr_decode_attention(p, q_pageable, bt, seq, pool, out_d, ws)
+
+
+def test_windowed_step_with_host_activations_is_bit_identical():
+    """The paper's default configuration (G = 128, clips 0.96 / 0.92, BF16
+    sink 64 / recent 256 windows): a step from pinned host buffers writes
+    the same pool and window bytes and returns the same output."""
+    c = synth.build_case(synth.workload("decode8k", 0, 1 / 16), 0)
+    p = optr.optr_params_create(c["R_k"], c["R_v"], c["mu"], c["h_q"], group=128,
+                                clip_k=0.96, clip_v=0.92, sink=64, recent=256)
+    bt = c["block_table"].to(DEV)
+    slot = torch.arange(c["B"], dtype=torch.int32, device=DEV)
+    pool = optr.new_pool(p, c["num_pages"], device=DEV)
+    win = optr.new_windows(p, c["B"], device=DEV)
+    optr.optr_kv_append_win(p, c["k_ctx"].to(DEV), c["v_ctx"].to(DEV), c["cu_ctx"].to(DEV),
+                            c["pos0_ctx"].to(DEV), bt, pool, win, slot)
+    pool_h, win_h = pool.clone(), win.clone()
+    seq = c["seq_lens"].to(DEV)
+    cu, pos0 = c["cu_new"].to(DEV), c["pos0_new"].to(DEV)
+    ws = optr.new_workspace(p, c["B"], bt.shape[1], device=DEV)
+    out_d = torch.empty(c["B"], c["h_q"], 128, dtype=torch.float32, device=DEV)
+    out_h = torch.zeros(c["B"], c["h_q"], 128, dtype=torch.float32).pin_memory()
+    optr.optr_decode_step_win(p, c["q"].to(DEV), c["k_new"].to(DEV), c["v_new"].to(DEV),
+                              cu, pos0, bt, seq, pool, win, slot, out_d, ws)
+    optr.optr_decode_step_win(p, _pinned(c["q"]), _pinned(c["k_new"]), _pinned(c["v_new"]),
+                              cu, pos0, bt, seq, pool_h, win_h, slot, out_h, ws)
+    torch.cuda.synchronize()
+    assert optr.optr_device_error(p) == 0
+    assert torch.equal(pool, pool_h)
+    assert torch.equal(win, win_h)
+    assert torch.equal(out_d.cpu(), out_h)
