@@ -848,7 +848,10 @@ cudaError_t launch_decode(const optr_params* p, int variant,
   }
   if (e != cudaSuccess) return e;
   prof_mark(p, 4, s);
-  const size_t cmb_bytes = sizeof(float) * kD * kD;
+  // R_v^T (64 KB) plus padding: more than half of an SM's shared memory,
+  // so no two combine CTAs share an SM (in a decode step they take SMs as
+  // the partial kernel's CTAs leave them)
+  const size_t cmb_bytes = 120 * 1024;
   e = ensure_dynamic_smem(reinterpret_cast<const void*>(&combine_kernel),
                           cmb_bytes);
   if (e != cudaSuccess) return e;
