@@ -720,6 +720,108 @@ combine_kernel(const float* __restrict__ part, const int* __restrict__ pref,
   }
 }
 
+// The one-CTA-per-segment combine (S = 1, no BF16 windows) without
+// block-wide merging steps: grid (B, h_kv), 512 threads, warp (r, qq) =
+// (query head 4h + r, channels 32qq .. 32qq + 31).  Every warp merges the
+// segment's partials for its own head and channels on its own (the
+// maxima, weights and sums by shuffles), with the headers and its o'
+// values of up to kFastBatch partials requested at once; a single barrier
+// then hands the normalised o' to the rotation, in which warp (r, qq)
+// produces outputs 32qq + lane of head r over all 128 input channels.
+constexpr int kFastBatch = 32;
+
+__global__ void __launch_bounds__(kCombineThreads)
+combine_fast_kernel(const float* __restrict__ part, const int* __restrict__ pref,
+                    const int* __restrict__ nzpref, int B, int h_q, int h_kv, int W,
+                    const float* __restrict__ R_vT, float* __restrict__ out,
+                    int fold_v) {
+  extern __shared__ float4 dsm[];
+  float* rts = reinterpret_cast<float*>(dsm);  // [128][128] R_v^T[h]
+  __shared__ __align__(16) float orot[4][kD];
+  const int b = blockIdx.x, h = blockIdx.y;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int r = warp >> 2, ch = 32 * (warp & 3) + lane;
+  if (!fold_v) {
+    const float4* src = reinterpret_cast<const float4*>(R_vT + (size_t)h * kD * kD);
+#pragma unroll
+    for (int u = 0; u < kD * kD / 4 / kCombineThreads; ++u)
+      cp_async16(&dsm[tid + u * kCombineThreads], src + tid + u * kCombineThreads);
+  }
+  cp_async_commit();
+  // the page prefix sums come from the query rotation, two kernels back
+  // (complete before the partial kernel let this grid launch)
+  const int np = __ldcg(pref + b + 1) - __ldcg(pref + b);
+  const long long F = (long long)__ldcg(pref + B) * h_kv;
+  const long long fs = (long long)__ldcg(pref + b) * h_kv + (long long)h * np;
+  const int nzb = __ldcg(nzpref + b);
+  int w0 = 0, n = 0;
+  if (np > 0) {
+    w0 = warp_of(fs, F, W);
+    n = warp_of(fs + np - 1, F, W) - w0 + 1;
+  }
+  const bool sparse = F < W;
+  const float* pbase = part + ((size_t)nzb * h_kv + h + w0) * kPartFloats;
+  pdl_wait();
+  pdl_trigger();
+  float* ob = out + ((size_t)b * h_q + 4 * h) * kD;
+  if (np == 0) {  // no cached token: the output is 0
+    ob[tid] = 0.f;
+    cp_async_wait<0>();
+    return;
+  }
+  // running maximum M, sum L and accumulator o of head r, channel ch
+  float M = -INFINITY, L = 0.f, o = 0.f;
+  for (int i0 = 0; i0 < n; i0 += kFastBatch) {
+    const int cnt = min(kFastBatch, n - i0);
+    // lane i: header of partial i0 + i; every lane: o' of all cnt partials
+    float m = -INFINITY, l = 0.f;
+    if (lane < cnt && !(sparse && warp_empty(w0 + i0 + lane, F, W))) {
+      const float* pp = pbase + (size_t)(i0 + lane) * kPartFloats;
+      m = __ldcg(pp + kPartM + r);
+      l = __ldcg(pp + kPartL + r);
+    }
+    float ov[kFastBatch];
+#pragma unroll
+    for (int i = 0; i < kFastBatch; ++i)
+      ov[i] = i < cnt ? __ldcg(pbase + (size_t)(i0 + i) * kPartFloats + r * kD + ch) : 0.f;
+    float bm = m;
+#pragma unroll
+    for (int x = 16; x > 0; x >>= 1) bm = fmaxf(bm, __shfl_xor_sync(0xffffffffu, bm, x));
+    const float Mn = fmaxf(M, bm);
+    const float alpha = merge_weight(M, Mn);
+    const float wgt = merge_weight(m, Mn);  // 0 for an empty partial
+    float wl = wgt * l;
+#pragma unroll
+    for (int x = 16; x > 0; x >>= 1) wl += __shfl_xor_sync(0xffffffffu, wl, x);
+    L = L * alpha + wl;
+    o *= alpha;
+#pragma unroll
+    for (int i = 0; i < kFastBatch; ++i) {
+      const float wi = __shfl_sync(0xffffffffu, wgt, i);
+      if (wi != 0.f) o = fmaf(ov[i], wi, o);
+    }
+    M = Mn;
+  }
+  orot[r][ch] = o * (L > 0.f ? 1.f / L : 0.f);
+  cp_async_wait<0>();
+  __syncthreads();
+  if (fold_v) {  // output in the folded value basis: no R_v^T
+    ob[r * kD + ch] = orot[r][ch];
+    return;
+  }
+  // out[r][i] = sum_k o'[r][k] R_v^T[k][i], i = ch
+  float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+#pragma unroll 8
+  for (int k = 0; k < kD; k += 4) {
+    const float4 ok = *reinterpret_cast<const float4*>(&orot[r][k]);
+    a0 = fmaf(ok.x, rts[(k + 0) * kD + ch], a0);
+    a1 = fmaf(ok.y, rts[(k + 1) * kD + ch], a1);
+    a2 = fmaf(ok.z, rts[(k + 2) * kD + ch], a2);
+    a3 = fmaf(ok.w, rts[(k + 3) * kD + ch], a3);
+  }
+  ob[r * kD + ch] = (a0 + a1) + (a2 + a3);
+}
+
 }  // namespace
 
 cudaError_t launch_partial_tensor(const optr_params* p, const uint8_t* pool,
@@ -852,6 +954,18 @@ cudaError_t launch_decode(const optr_params* p, int variant,
   // so no two combine CTAs share an SM (in a decode step they take SMs as
   // the partial kernel's CTAs leave them)
   const size_t cmb_bytes = 120 * 1024;
+  if (plan.S == 1 && plan.Ww == 0) {
+    e = ensure_dynamic_smem(reinterpret_cast<const void*>(&combine_fast_kernel),
+                            cmb_bytes);
+    if (e != cudaSuccess) return e;
+    e = launch_pdl(combine_fast_kernel, dim3(B, h_kv), dim3(kCombineThreads),
+                   cmb_bytes, s, (const float*)part, (const int*)pref,
+                   (const int*)nzpref, B, h_q, h_kv, plan.W, (const float*)p->R_vT,
+                   out, p->fold_v);
+    if (e != cudaSuccess) return e;
+    prof_mark(p, 5, s);
+    return cudaSuccess;
+  }
   e = ensure_dynamic_smem(reinterpret_cast<const void*>(&combine_kernel),
                           cmb_bytes);
   if (e != cudaSuccess) return e;

@@ -192,6 +192,25 @@ def test_split_invariance(variant):
         assert float((a - bb).abs().max()) <= 1e-5 * rms
 
 
+@pytest.mark.parametrize("variant", VARIANTS)
+@pytest.mark.parametrize("short", [16, 48])
+def test_one_long_sequence_among_short_ones(variant, short):
+    """One sequence far longer than the rest of a 128-sequence batch: its
+    segments span more than 32 split-K partials while the plan keeps one
+    combine CTA per segment, so the merge runs over several batches of
+    partials; with 16-token neighbours the batch has fewer pages than warps
+    (some warps own nothing), with 48-token neighbours it has more."""
+    c, pool_ref, _, _ = _case("ragged", 1 / 32)
+    ctx = c["seq_lens_ctx"].clone()
+    b_long = int(torch.argmax(ctx))
+    lens = torch.minimum(ctx, torch.full_like(ctx, short))
+    lens[b_long] = ctx[b_long]
+    assert int(ctx[b_long]) // 16 > 32
+    got = ph.gpu_decode(c, pool_ref, variant, seq_lens=lens)
+    ref = ph.oracle_decode(c, pool_ref, seq_lens=lens)
+    ph.assert_decode_close(got, ref, f"long among {short}-token sequences")
+
+
 def test_needle_is_retrieved():
     """long-context workload: the planted key wins the softmax of its
     group's first query head, and the GPU output matches the oracle."""
