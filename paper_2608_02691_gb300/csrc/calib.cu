@@ -66,18 +66,22 @@ constexpr int kTK = 16;
 // The host picks the largest tile, then a split of K into kc chunks, so that
 // a call covers about two CTAs per SM (float64 runs at a few FMAs per clock
 // per SM on this GPU).  With kc > 1 chunk z of a product writes its raw sum
-// to P[z][b] and gemm_f64_reduce_kernel adds the chunks in a fixed order.
+// to P[z][b]; the last of the tile's kc CTAs to finish (a per-tile arrival
+// counter, left at 0 again) adds the chunks in a fixed order, z = 0 .. kc-1,
+// so the result does not depend on which CTA that is.
 template <int TILE>
-__global__ void __launch_bounds__(256) gemm_f64_kernel(Gemm g, int kc, double* P) {
+__global__ void __launch_bounds__(256) gemm_f64_kernel(Gemm g, int kc, double* P,
+                                                       int* tcnt) {
   constexpr int R = TILE / 16;  // outputs per thread per dimension
   __shared__ double As[kTK][TILE + 1];
   __shared__ double Bs[kTK][TILE + 1];
+  __shared__ int s_last;
   const int b = blockIdx.z / kc, z = blockIdx.z % kc;
   const int m0 = blockIdx.y * TILE, n0 = blockIdx.x * TILE;
   const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
   double* C = g.C + (long long)b * g.sC;
   if (g.gate != nullptr && g.gate_idx >= *g.gate) {
-    if (g.pass != nullptr && kc == 1) {
+    if (g.pass != nullptr && z == 0) {
       for (int i = tid; i < TILE * TILE; i += 256) {
         const int r = m0 + i / TILE, c = n0 + i % TILE;
         if (r < g.M && c < g.N) C[r * g.ldc + c] = g.pass[r * g.ldc + c];
@@ -146,33 +150,28 @@ __global__ void __launch_bounds__(256) gemm_f64_kernel(Gemm g, int kc, double* P
       C[r * g.ldc + c] = x;
     }
   }
-}
-
-// C[b] = alpha sum_z P[z][b] + beta C[b] + diag I (the chunks in order).
-__global__ void gemm_f64_reduce_kernel(Gemm g, int kc, int batch, const double* P) {
-  const long long mn = (long long)g.M * g.N;
-  if (g.gate != nullptr && g.gate_idx >= *g.gate) {
-    if (g.pass == nullptr) return;
-    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < mn * batch;
-         i += (long long)gridDim.x * blockDim.x) {
-      const long long b = i / mn, e = i % mn;
-      const int r = (int)(e / g.N), c = (int)(e % g.N);
-      g.C[b * g.sC + r * g.ldc + c] = g.pass[r * g.ldc + c];
-    }
-    return;
-  }
-  for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < mn * batch;
-       i += (long long)gridDim.x * blockDim.x) {
-    const long long b = i / mn, e = i % mn;
-    const int r = (int)(e / g.N), c = (int)(e % g.N);
-    double s = 0.0;
-    for (int z = 0; z < kc; ++z) s += P[((long long)z * batch + b) * mn + e];
-    double* C = g.C + b * g.sC + r * g.ldc + c;
-    double x = g.alpha * s;
-    if (g.beta != 0.0) x += g.beta * *C;
+  if (kc == 1) return;
+  // split K: the tile's last CTA to arrive adds the kc chunk sums in order
+  __threadfence();
+  __syncthreads();
+  const int tile_id = (b * gridDim.y + blockIdx.y) * gridDim.x + blockIdx.x;
+  if (tid == 0) s_last = atomicAdd(tcnt + tile_id, 1) == kc - 1;
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  const int batch = gridDim.z / kc;
+  for (int i = tid; i < TILE * TILE; i += 256) {
+    const int r = m0 + i / TILE, c = n0 + i % TILE;
+    if (r >= g.M || c >= g.N) continue;
+    double sum = 0.0;
+    for (int zz = 0; zz < kc; ++zz)
+      sum += __ldcg(P + (((long long)zz * batch + b) * g.M + r) * g.N + c);
+    double x = g.alpha * sum;
+    if (g.beta != 0.0) x += g.beta * C[r * g.ldc + c];
     if (r == c) x += g.diag;
-    *C = x;
+    C[r * g.ldc + c] = x;
   }
+  if (tid == 0) tcnt[tile_id] = 0;
 }
 
 // ------------------------------------------------------- small kernels
@@ -527,11 +526,13 @@ inline int nblk(long long n, int t = 256) {
 }
 
 constexpr long long kGemmScratch = 1 << 21;  // split-K doubles (16 MiB)
+constexpr int kGemmTiles = 512;  // K is split only while a call has < 300 tiles
 
 struct GemmCall {
   cudaStream_t s;
   double* scratch;        // split-K partial sums
   long long scratch_len;  // doubles
+  int* tcnt;              // split-K arrival counters, one per output tile (0)
   void operator()(int M, int N, int K, const double* A, long long lda, bool tA,
                   const double* B, long long ldb, bool tB, double* C, long long ldc,
                   double alpha = 1.0, double beta = 0.0, int batch = 1,
@@ -550,14 +551,9 @@ struct GemmCall {
            (long long)(2 * kc) * batch * M * N <= scratch_len)
       kc *= 2;
     const dim3 grid((N + tile - 1) / tile, (M + tile - 1) / tile, batch * kc);
-    if (tile == 64) gemm_f64_kernel<64><<<grid, 256, 0, s>>>(g, kc, scratch);
-    else if (tile == 32) gemm_f64_kernel<32><<<grid, 256, 0, s>>>(g, kc, scratch);
-    else gemm_f64_kernel<16><<<grid, 256, 0, s>>>(g, kc, scratch);
-    if (kc > 1) {
-      const long long n = (long long)batch * M * N;
-      const int blocks = (int)std::min<long long>((n + 255) / 256, 4096);
-      gemm_f64_reduce_kernel<<<blocks, 256, 0, s>>>(g, kc, batch, scratch);
-    }
+    if (tile == 64) gemm_f64_kernel<64><<<grid, 256, 0, s>>>(g, kc, scratch, tcnt);
+    else if (tile == 32) gemm_f64_kernel<32><<<grid, 256, 0, s>>>(g, kc, scratch, tcnt);
+    else gemm_f64_kernel<16><<<grid, 256, 0, s>>>(g, kc, scratch, tcnt);
   }
 };
 
@@ -591,8 +587,9 @@ struct Calib {
   unsigned* err;
   const double* W;  // [g][d_model][d]
   double* gsc;      // split-K scratch of the GEMMs
+  int* gcnt;        // split-K arrival counters (kGemmTiles, zero between calls)
   cudaStream_t st;
-  GemmCall gemm() const { return GemmCall{st, gsc, kGemmScratch}; }
+  GemmCall gemm() const { return GemmCall{st, gsc, kGemmScratch, gcnt}; }
 };
 
 struct Layout {
@@ -640,6 +637,7 @@ size_t carve(Calib& C, char* base) {
   C.U = L.take<double>(g * nm * D);
   C.E = L.take<double>(g * nm * c.d_model);
   C.gsc = L.take<double>(kGemmScratch);
+  C.gcnt = L.take<int>(kGemmTiles);
   double** dd[] = {&C.R0[0], &C.R0[1], &C.A, &C.m, &C.v, &C.dA, &C.S, &C.Xs,
                    &C.Hs, &C.T1[0], &C.T1[1], &C.T2[0], &C.T2[1], &C.R, &C.dR,
                    &C.dE, &C.best};
@@ -931,7 +929,8 @@ extern "C" optr_status optr_calibrate_head(
   Calib C;
   calib_init(C, c, workspace, W_O, stream);
   const int n = kCD * kCD;
-  if (cudaMemsetAsync(C.err, 0, sizeof(unsigned), stream) != cudaSuccess)
+  if (cudaMemsetAsync(C.err, 0, sizeof(unsigned), stream) != cudaSuccess ||
+      cudaMemsetAsync(C.gcnt, 0, sizeof(int) * kGemmTiles, stream) != cudaSuccess)
     return OPTR_ERR_CUDA;
   col_mean_kernel<<<1, kCD, 0, stream>>>(K, c->T, mu);
   const double* r0[2] = {R0_K, R0_V};
@@ -974,7 +973,8 @@ extern "C" optr_status optr_calib_loss_grad(
   Calib C;
   calib_init(C, c, workspace, W_O, stream);
   const int n = kCD * kCD;
-  if (cudaMemsetAsync(C.err, 0, sizeof(unsigned), stream) != cudaSuccess)
+  if (cudaMemsetAsync(C.err, 0, sizeof(unsigned), stream) != cudaSuccess ||
+      cudaMemsetAsync(C.gcnt, 0, sizeof(int) * kGemmTiles, stream) != cudaSuccess)
     return OPTR_ERR_CUDA;
   C.tr[0].q = q; C.tr[0].K = K; C.tr[0].V = V; C.tr[0].tpos = t_pos;
   C.tr[0].T = c->T; C.tr[0].nt = c->nt;
