@@ -720,21 +720,25 @@ combine_kernel(const float* __restrict__ part, const int* __restrict__ pref,
   }
 }
 
-// The one-CTA-per-segment combine (S = 1, no BF16 windows) without
-// block-wide merging steps: grid (B, h_kv), 512 threads, warp (r, qq) =
-// (query head 4h + r, channels 32qq .. 32qq + 31).  Every warp merges the
-// segment's partials for its own head and channels on its own (the
-// maxima, weights and sums by shuffles), with the headers and its o'
-// values of up to kFastBatch partials requested at once; a single barrier
-// then hands the normalised o' to the rotation, in which warp (r, qq)
-// produces outputs 32qq + lane of head r over all 128 input channels.
+// The one-CTA-per-segment combine (S = 1) without block-wide merging steps:
+// grid (B, h_kv), 512 threads, warp (r, qq) = (query head 4h + r, channels
+// 32qq .. 32qq + 31).  Every warp merges the segment's partials for its own
+// head and channels on its own (the maxima, weights and sums by shuffles),
+// with the headers and its o' values of up to kFastBatch partials requested
+// at once, then the BF16-window partials of the segment (if any) into a
+// second accumulator under the same running maxima; a single barrier then
+// hands the normalised o' to the rotation, in which warp (r, qq) produces
+// outputs 32qq + lane of head r over all 128 input channels (the window
+// part, computed on the unrotated values, is added after it).
 constexpr int kFastBatch = 32;
 
 __global__ void __launch_bounds__(kCombineThreads)
 combine_fast_kernel(const float* __restrict__ part, const int* __restrict__ pref,
                     const int* __restrict__ nzpref, int B, int h_q, int h_kv, int W,
                     const float* __restrict__ R_vT, float* __restrict__ out,
-                    int fold_v) {
+                    int fold_v, const float* __restrict__ wpart,
+                    const int32_t* __restrict__ seq_lens, int max_pages, int sink,
+                    int recent, int Uw, int Ww) {
   extern __shared__ float4 dsm[];
   float* rts = reinterpret_cast<float*>(dsm);  // [128][128] R_v^T[h]
   __shared__ __align__(16) float orot[4][kD];
@@ -761,29 +765,47 @@ combine_fast_kernel(const float* __restrict__ part, const int* __restrict__ pref
   }
   const bool sparse = F < W;
   const float* pbase = part + ((size_t)nzb * h_kv + h + w0) * kPartFloats;
+  // BF16-window partials of (b, h): the window warps that own its units
+  // 0 .. nwu - 1 (window.cuh), one slot each, no gaps
+  int wn = 0;
+  const float* wbase = nullptr;
+  if (Ww > 0) {
+    int len = __ldg(seq_lens + b);
+    if (len < 0 || (long long)len > (long long)max_pages * kPage) len = 0;
+    const int nwu = (win_count(len, sink, recent) + kWinUnit - 1) / kWinUnit;
+    if (nwu > 0) {
+      const long long U = (long long)B * h_kv * Uw;
+      const long long u0 = ((long long)b * h_kv + h) * Uw;
+      const int ww0 = warp_of(u0, U, Ww);
+      wn = warp_of(u0 + nwu - 1, U, Ww) - ww0 + 1;
+      wbase = wpart + (size_t)(ww0 + b * h_kv + h) * kPartFloats;
+    }
+  }
   pdl_wait();
   pdl_trigger();
   float* ob = out + ((size_t)b * h_q + 4 * h) * kD;
-  if (np == 0) {  // no cached token: the output is 0
+  if (np == 0 && wn == 0) {  // no cached token: the output is 0
     ob[tid] = 0.f;
     cp_async_wait<0>();
     return;
   }
-  // running maximum M, sum L and accumulator o of head r, channel ch
-  float M = -INFINITY, L = 0.f, o = 0.f;
-  for (int i0 = 0; i0 < n; i0 += kFastBatch) {
-    const int cnt = min(kFastBatch, n - i0);
-    // lane i: header of partial i0 + i; every lane: o' of all cnt partials
+  // running maximum M and sum L of head r; accumulators of channel ch:
+  // o (INT2 partials) and ow (window partials)
+  float M = -INFINITY, L = 0.f, o = 0.f, ow = 0.f;
+  // one batch of up to kFastBatch partials at base (empty slots skipped
+  // when sparse: only the INT2 slots of warps that own no page); the
+  // accumulator acc takes the batch, both are rescaled to the new maximum
+  auto merge = [&](const float* base, int cnt, bool sp, int wfirst, float& acc) {
     float m = -INFINITY, l = 0.f;
-    if (lane < cnt && !(sparse && warp_empty(w0 + i0 + lane, F, W))) {
-      const float* pp = pbase + (size_t)(i0 + lane) * kPartFloats;
+    if (lane < cnt && !(sp && warp_empty(wfirst + lane, F, W))) {
+      const float* pp = base + (size_t)lane * kPartFloats;
       m = __ldcg(pp + kPartM + r);
       l = __ldcg(pp + kPartL + r);
     }
     float ov[kFastBatch];
 #pragma unroll
     for (int i = 0; i < kFastBatch; ++i)
-      ov[i] = i < cnt ? __ldcg(pbase + (size_t)(i0 + i) * kPartFloats + r * kD + ch) : 0.f;
+      ov[i] = i < cnt ? __ldcg(base + (size_t)i * kPartFloats + r * kD + ch) : 0.f;
     float bm = m;
 #pragma unroll
     for (int x = 16; x > 0; x >>= 1) bm = fmaxf(bm, __shfl_xor_sync(0xffffffffu, bm, x));
@@ -795,18 +817,25 @@ combine_fast_kernel(const float* __restrict__ part, const int* __restrict__ pref
     for (int x = 16; x > 0; x >>= 1) wl += __shfl_xor_sync(0xffffffffu, wl, x);
     L = L * alpha + wl;
     o *= alpha;
+    ow *= alpha;
 #pragma unroll
     for (int i = 0; i < kFastBatch; ++i) {
       const float wi = __shfl_sync(0xffffffffu, wgt, i);
-      if (wi != 0.f) o = fmaf(ov[i], wi, o);
+      if (wi != 0.f) acc = fmaf(ov[i], wi, acc);
     }
     M = Mn;
-  }
-  orot[r][ch] = o * (L > 0.f ? 1.f / L : 0.f);
+  };
+  for (int i0 = 0; i0 < n; i0 += kFastBatch)
+    merge(pbase + (size_t)i0 * kPartFloats, min(kFastBatch, n - i0), sparse, w0 + i0, o);
+  for (int j0 = 0; j0 < wn; j0 += kFastBatch)
+    merge(wbase + (size_t)j0 * kPartFloats, min(kFastBatch, wn - j0), false, 0, ow);
+  const float il = L > 0.f ? 1.f / L : 0.f;
+  orot[r][ch] = o * il;
+  const float owin = ow * il;  // window part (values unrotated)
   cp_async_wait<0>();
   __syncthreads();
   if (fold_v) {  // output in the folded value basis: no R_v^T
-    ob[r * kD + ch] = orot[r][ch];
+    ob[r * kD + ch] = orot[r][ch] + owin;
     return;
   }
   // out[r][i] = sum_k o'[r][k] R_v^T[k][i], i = ch
@@ -819,7 +848,7 @@ combine_fast_kernel(const float* __restrict__ part, const int* __restrict__ pref
     a2 = fmaf(ok.z, rts[(k + 2) * kD + ch], a2);
     a3 = fmaf(ok.w, rts[(k + 3) * kD + ch], a3);
   }
-  ob[r * kD + ch] = (a0 + a1) + (a2 + a3);
+  ob[r * kD + ch] = ((a0 + a1) + (a2 + a3)) + owin;
 }
 
 }  // namespace
@@ -954,14 +983,15 @@ cudaError_t launch_decode(const optr_params* p, int variant,
   // so no two combine CTAs share an SM (in a decode step they take SMs as
   // the partial kernel's CTAs leave them)
   const size_t cmb_bytes = 120 * 1024;
-  if (plan.S == 1 && plan.Ww == 0) {
+  if (plan.S == 1) {
     e = ensure_dynamic_smem(reinterpret_cast<const void*>(&combine_fast_kernel),
                             cmb_bytes);
     if (e != cudaSuccess) return e;
     e = launch_pdl(combine_fast_kernel, dim3(B, h_kv), dim3(kCombineThreads),
                    cmb_bytes, s, (const float*)part, (const int*)pref,
                    (const int*)nzpref, B, h_q, h_kv, plan.W, (const float*)p->R_vT,
-                   out, p->fold_v);
+                   out, p->fold_v, (const float*)wp.wpart, seq_lens, max_pages,
+                   sink, recent, plan.Uw, plan.Ww);
     if (e != cudaSuccess) return e;
     prof_mark(p, 5, s);
     return cudaSuccess;
