@@ -1,8 +1,8 @@
-// Packed float32 pair arithmetic: the .f32x2 forms of add, sub, mul and fma
-// (sm_100 and later) issue one instruction for two independent float32
-// operations, each rounded exactly as its scalar .rn counterpart (no flush
-// of subnormals).  The kernels are issue-bound, so pairing independent
-// float32 operations halves their share of the issue slots.
+// Packed float32 pair arithmetic: the .f32x2 forms of sub and fma (sm_100
+// and later) issue one instruction for two independent float32 operations,
+// each rounded exactly as its scalar .rn counterpart (no flush of
+// subnormals).  Where a kernel is issue-bound and its values come in
+// register pairs, pairing them halves their share of the issue slots.
 #pragma once
 
 namespace optr {
@@ -17,31 +17,11 @@ __device__ __forceinline__ float2 fma2(float2 a, float2 b, float2 c) {
   return d;
 }
 
-__device__ __forceinline__ float2 add2(float2 a, float2 b) {
-  float2 d;
-  asm("{\n\t.reg .b64 ra, rb, rd;\n\t"
-      "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
-      "add.rn.f32x2 rd, ra, rb;\n\tmov.b64 {%0, %1}, rd;\n\t}"
-      : "=f"(d.x), "=f"(d.y)
-      : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
-  return d;
-}
-
 __device__ __forceinline__ float2 sub2(float2 a, float2 b) {
   float2 d;
   asm("{\n\t.reg .b64 ra, rb, rd;\n\t"
       "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
       "sub.rn.f32x2 rd, ra, rb;\n\tmov.b64 {%0, %1}, rd;\n\t}"
-      : "=f"(d.x), "=f"(d.y)
-      : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
-  return d;
-}
-
-__device__ __forceinline__ float2 mul2(float2 a, float2 b) {
-  float2 d;
-  asm("{\n\t.reg .b64 ra, rb, rd;\n\t"
-      "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
-      "mul.rn.f32x2 rd, ra, rb;\n\tmov.b64 {%0, %1}, rd;\n\t}"
       : "=f"(d.x), "=f"(d.y)
       : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
   return d;
