@@ -175,3 +175,28 @@ def test_windowed_step_with_host_activations_is_bit_identical():
     assert torch.equal(pool, pool_h)
     assert torch.equal(win, win_h)
     assert torch.equal(out_d.cpu(), out_h)
+
+
+def test_windowed_prefill_from_host_inputs():
+    """A windowed cache write of a whole context (more than 256 tokens:
+    the CUDA-core kernel, then the window-copy kernel) from pinned host k, v
+    writes the same pool and window bytes as from device inputs."""
+    c = synth.build_case(synth.workload("decode8k", 0, 1 / 16), 0)
+    out = []
+    for host in (False, True):
+        p = optr.optr_params_create(c["R_k"], c["R_v"], c["mu"], c["h_q"],
+                                    append_variant=optr.OPTR_VARIANT_CUDA_CORE,
+                                    sink=64, recent=256)
+        pool = optr.new_pool(p, c["num_pages"], device=DEV)
+        win = optr.new_windows(p, c["B"], device=DEV)
+        slot = torch.arange(c["B"], dtype=torch.int32, device=DEV)
+        k = _pinned(c["k_ctx"]) if host else c["k_ctx"].to(DEV)
+        v = _pinned(c["v_ctx"]) if host else c["v_ctx"].to(DEV)
+        optr.optr_kv_append_win(p, k, v, c["cu_ctx"].to(DEV), c["pos0_ctx"].to(DEV),
+                                c["block_table"].to(DEV), pool, win, slot)
+        torch.cuda.synchronize()
+        assert optr.optr_device_error(p) == 0
+        out.append((pool, win))
+    assert c["k_ctx"].shape[0] > 256
+    assert torch.equal(out[0][0], out[1][0])
+    assert torch.equal(out[0][1], out[1][1])
