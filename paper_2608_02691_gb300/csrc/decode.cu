@@ -236,9 +236,18 @@ step_prologue_kernel(
     int* __restrict__ nzpref, int* __restrict__ cnt_ws, unsigned* err, int fold_v,
     int n_wcp, __nv_bfloat16* __restrict__ win,
     const int32_t* __restrict__ win_slot, int n_slots, int sink, int recent,
-    int group128) {
+    int group128, int lead) {
   extern __shared__ __align__(16) unsigned char dsm_[];
-  const int bid = blockIdx.x;
+  // Block order: `lead` query-rotation CTAs, the cache-write CTAs, then the
+  // remaining query-rotation CTAs.  With lead = SMs - write CTAs, the first
+  // wave gives every write CTA (the longest) an SM of its own and the CTAs
+  // beyond one per SM are query rotations.
+  int bid = blockIdx.x;
+  if (bid < lead) {
+    bid += n_app + n_wcp;  // a query rotation
+  } else if (bid < lead + n_app + n_wcp) {
+    bid -= lead;           // a cache write or window copy
+  }
   if (bid < n_app) {
     const int tblk = bid % app_tiles, hk = (bid / app_tiles) % h_kv,
               kind = bid / (app_tiles * h_kv);
@@ -949,7 +958,8 @@ cudaError_t launch_decode(const optr_params* p, int variant,
                    windows ? win->win : (__nv_bfloat16*)nullptr,
                    windows ? win->slot : (const int32_t*)nullptr,
                    windows ? win->n_slots : 0, sink, recent,
-                   p->cfg.group == 128 ? 1 : 0);
+                   p->cfg.group == 128 ? 1 : 0,
+                   std::max(0, std::min(B * h_kv, p->num_sms - n_app - n_wcp)));
     if (e != cudaSuccess) return e;
     prof_mark(p, 1, s);  // the append stage covers the fused launch,
     prof_mark(p, 2, s);  // the query-rotation stage is empty
